@@ -1,0 +1,206 @@
+"""Python loader for the NetKV CPU oracle (``netkv_oracle.cpp``).
+
+TEST INFRASTRUCTURE ONLY: imported by ``tests/``, ``__graft_entry__.smoke()`` and
+the benchmark's CPU-baseline leg.  The product path never imports this package.
+
+The oracle is plain C++ in double precision compiled with g++ (OpenMP across
+independent units only).  ``build()`` compiles it; the functions below marshal
+numpy arrays to it and return numpy results.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import subprocess
+from typing import Optional, Sequence
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "netkv_oracle.cpp")
+_LIB = os.path.join(_HERE, "libnetkv_oracle.so")
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + f".tmp{os.getpid()}"
+        subprocess.check_call(["g++", "-O2", "-std=c++17", "-fopenmp", "-shared", "-fPIC",
+                               _SRC, "-o", tmp])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        build()
+        _lib = C.CDLL(_LIB)
+        _declare(_lib)
+    return _lib
+
+
+P = C.c_void_p
+U32, U64, I64, F64, INT = C.c_uint32, C.c_uint64, C.c_int64, C.c_double, C.c_int
+
+
+def _declare(l):
+    l.oracle_kv_bytes_per_token.restype = F64
+    l.oracle_kv_bytes_per_token.argtypes = [U32, U32, U32, U32]
+    l.oracle_beff_tier.restype = F64
+    l.oracle_beff_tier.argtypes = [F64, F64, F64]
+    l.oracle_transfer_time.restype = F64
+    l.oracle_transfer_time.argtypes = [F64, F64, F64]
+    l.oracle_s_eff.restype = F64
+    l.oracle_s_eff.argtypes = [F64, F64, F64]
+    l.oracle_tier.restype = INT
+    l.oracle_tier.argtypes = [P, U64, U64]
+    l.oracle_path_links.restype = INT
+    l.oracle_path_links.argtypes = [P, U64, U64, P, P]
+    l.oracle_used_links.restype = U64
+    l.oracle_used_links.argtypes = [P]
+    l.oracle_cost_matrix.restype = None
+    l.oracle_cost_matrix.argtypes = [P, P, P, P, P, U64, U64, F64, P]
+    l.oracle_cost_entries.restype = None
+    l.oracle_cost_entries.argtypes = [P, P, P, P, P, U64, P, P, P, U64, F64, P]
+    l.oracle_up_bottleneck.restype = None
+    l.oracle_up_bottleneck.argtypes = [P, P, P, U64, U64, P]
+    l.oracle_prefix_match.restype = None
+    l.oracle_prefix_match.argtypes = [P, P, U32, P, P, U32, P, U32, P]
+    l.oracle_prefix_match_one.restype = None
+    l.oracle_prefix_match_one.argtypes = [P, U64, P, P, U64, P]
+    l.oracle_schedule_stream.restype = None
+    l.oracle_schedule_stream.argtypes = [P, P, P, P, P, U64, P, P, P, P, P, U64, F64, F64, F64,
+                                         F64, I64, U64, P, P, F64, P, P, P, P, P]
+
+
+def _p(a: Optional[np.ndarray]):
+    return None if a is None else a.ctypes.data_as(C.c_void_p)
+
+
+def _c(a, dt):
+    return np.ascontiguousarray(np.asarray(a, dtype=dt))
+
+
+# ------------------------------------------------------------------ closed forms
+def kv_bytes_per_token(n_layers=80, n_kv_heads=8, d_head=128, b_elem=2) -> float:
+    return lib().oracle_kv_bytes_per_token(n_layers, n_kv_heads, d_head, b_elem)
+
+
+def beff_tier(B, c, n_inflight=0.0) -> float:
+    return lib().oracle_beff_tier(B, c, n_inflight)
+
+
+def transfer_time(s, B_eff, L=0.0) -> float:
+    return lib().oracle_transfer_time(s, B_eff, L)
+
+
+def s_eff(s_r, lam, l_r) -> float:
+    return lib().oracle_s_eff(s_r, lam, l_r)
+
+
+# ------------------------------------------------------------------ topology
+def tier(fanout: Sequence[int], i: int, j: int) -> int:
+    f = _c(fanout, np.uint32)
+    return lib().oracle_tier(_p(f), i, j)
+
+
+def path_links(fanout: Sequence[int], i: int, j: int):
+    f = _c(fanout, np.uint32)
+    links = np.zeros(8, np.uint64)
+    levels = np.zeros(8, np.int32)
+    n = lib().oracle_path_links(_p(f), i, j, _p(links), _p(levels))
+    return links[:n], levels[:n]
+
+
+def used_links(fanout) -> int:
+    f = _c(fanout, np.uint32)
+    return int(lib().oracle_used_links(_p(f)))
+
+
+# ------------------------------------------------------------------ oracle matrix
+def cost_matrix(fanout, role, bw, lat, util, kv_bytes) -> np.ndarray:
+    f, ro = _c(fanout, np.uint32), _c(role, np.uint8)
+    b, la = _c(bw, np.float64), _c(lat, np.float64)
+    u = _c(util, np.float32)
+    S, L = u.shape
+    P = int((ro == 0).sum()); D = int((ro == 1).sum())
+    out = np.zeros((S, P, D), np.float64)
+    lib().oracle_cost_matrix(_p(f), _p(ro), _p(b), _p(la), _p(u), L, S, float(kv_bytes), _p(out))
+    return out
+
+
+def cost_entries(fanout, role, bw, lat, util, s, p, d, kv_bytes) -> np.ndarray:
+    f, ro = _c(fanout, np.uint32), _c(role, np.uint8)
+    b, la = _c(bw, np.float64), _c(lat, np.float64)
+    u = _c(util, np.float32)
+    s, p, d = _c(s, np.uint64), _c(p, np.uint64), _c(d, np.uint64)
+    out = np.zeros(len(s), np.float64)
+    lib().oracle_cost_entries(_p(f), _p(ro), _p(b), _p(la), _p(u), u.shape[1], _p(s), _p(p),
+                              _p(d), len(s), float(kv_bytes), _p(out))
+    return out
+
+
+def up_bottleneck(fanout, bw, util) -> np.ndarray:
+    f, b, u = _c(fanout, np.uint32), _c(bw, np.float64), _c(util, np.float32)
+    S, L = u.shape
+    n = int(np.prod(np.asarray(fanout, dtype=np.int64)))
+    out = np.zeros((S, n, 4), np.float64)
+    lib().oracle_up_bottleneck(_p(f), _p(b), _p(u), L, S, _p(out))
+    return out
+
+
+# ------------------------------------------------------------------ prefix match
+def prefix_match(keys, key_off, D, chains, chain_off, set_off) -> np.ndarray:
+    k, ko = _c(keys, np.uint64), _c(key_off, np.uint64)
+    ch, co = _c(chains, np.uint64), _c(chain_off, np.uint64)
+    so = _c(set_off, np.uint32)
+    R = len(co) - 1
+    out = np.zeros((R, D), np.uint16)
+    lib().oracle_prefix_match(_p(k), _p(ko), D, _p(ch), _p(co), R, _p(so), len(so) - 1, _p(out))
+    return out
+
+
+def prefix_match_one(keys, chains, chain_off) -> np.ndarray:
+    k = _c(keys, np.uint64)
+    ch, co = _c(chains, np.uint64), _c(chain_off, np.uint64)
+    out = np.zeros(len(co) - 1, np.uint16)
+    lib().oracle_prefix_match_one(_p(k), len(k), _p(ch), _p(co), len(co) - 1, _p(out))
+    return out
+
+
+# ------------------------------------------------------------------ greedy
+class StreamResult:
+    def __init__(self, dec, best, second, load, near_ties, mismatches, rejects):
+        self.dec, self.best, self.second, self.load = dec, best, second, load
+        self.near_ties, self.mismatches, self.rejects = near_ties, mismatches, rejects
+
+
+def schedule_stream(fanout, role, bw, lat, util, length, prefill, snap, M, events,
+                    w_net, w_prefix, w_load, theta, cap, bytes_per_token,
+                    load_init=None, hint=None, rel_tol=1e-5, dec_inout=None) -> StreamResult:
+    """Run one stream's events.  Arrays are indexed by global request index r.
+
+    ``dec_inout`` (int32 [R]) carries decisions across streams that share request
+    arrays; entries for this stream's requests are written.
+    """
+    f, ro = _c(fanout, np.uint32), _c(role, np.uint8)
+    b, la = _c(bw, np.float64), _c(lat, np.float64)
+    u = _c(util, np.float32)
+    ln, pf, sn = _c(length, np.uint32), _c(prefill, np.uint32), _c(snap, np.uint32)
+    m = _c(M, np.uint16)
+    ev = _c(events, np.uint32)
+    R = len(ln)
+    D = int((ro == 1).sum())
+    dec = np.full(R, -1, np.int32) if dec_inout is None else dec_inout
+    best = np.full(R, np.inf); second = np.full(R, np.inf)
+    load = np.zeros(D, np.int64)
+    counts = np.zeros(3, np.int64)
+    li = None if load_init is None else _c(load_init, np.int64)
+    h = None if hint is None else _c(hint, np.int32)
+    lib().oracle_schedule_stream(_p(f), _p(ro), _p(b), _p(la), _p(u), u.shape[1], _p(ln), _p(pf),
+                                 _p(sn), _p(m), _p(ev), len(ev), float(w_net), float(w_prefix),
+                                 float(w_load), float(theta), int(cap), int(bytes_per_token),
+                                 _p(li), _p(h), float(rel_tol), _p(dec), _p(best), _p(second),
+                                 _p(load), _p(counts))
+    return StreamResult(dec, best, second, load, int(counts[0]), int(counts[1]), int(counts[2]))

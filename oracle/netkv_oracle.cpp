@@ -1,0 +1,325 @@
+// NetKV CPU oracle: a plain, slow, double-precision statement of what the
+// decode-instance scoring path computes (arXiv 2606.03910, "NetKV").
+//
+// TEST INFRASTRUCTURE ONLY.  Nothing in the product path may call, link or
+// load this file; only the tests, the package's smoke check and the benchmark's
+// CPU-baseline leg use it.  It shares no code with the CUDA library: it knows
+// the instance tree only through the documented link-numbering convention and
+// computes everything by the definitions below, in double precision.
+//
+// What it states, with the paper's passage for each part:
+//   * KV size, Eq. 1 (Sec. III-B): s = 2 * n_layers * n_kv_heads * d_head * l * b_elem.
+//   * Locality tier tau(p,d) in {0,1,2,3} (Sec. III-A): same node / leaf / pod / other,
+//     found here by climbing the tree from both instances until their ancestors meet.
+//   * Effective bandwidth, Eq. 4 (Sec. III-D), generalised per link: the bottleneck
+//     of B_level(e) * (1 - u_e) over every link e on the up and down path, with the
+//     self-contention count n_inflight = 0 (the paper allows n_inflight == 0 when
+//     telemetry already covers the scheduler's flows).  With one utilisation per tier
+//     this is exactly B_tau * (1 - c_tau) (Sec. III-D, per-tier collapse).
+//   * Transfer time, Eq. 3: T = s / B_eff + L_tau.
+//   * Block-level prefix hit (Sec. III-B): lambda = 16 * |LCP_block(h_r, K_d)|, the number
+//     of leading blocks of the request's hash chain that are all in decode d's cache.
+//   * Effective transfer size, Eq. 2: s_eff = s * (1 - lambda / l).
+//   * Algorithm 1 (Sec. IV-A) as a weighted score: filter by capacity (line 1), reject
+//     when nothing is feasible (line 2), score every candidate (lines 3-11), take the
+//     argmin with the lowest index among equal scores (line 13), then update load.
+//
+// Parity: pinned by the not-gpu tests (worked example of Sec. III-D, closed forms of
+// Eq. 1, the per-tier special case of Eq. 4, brute force on tiny instances,
+// Propositions 1 and 2, first-miss LCP semantics).
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <limits>
+#include <unordered_set>
+#include <vector>
+
+namespace {
+
+struct Tree {
+  uint32_t f[4];  // instances per node, nodes per leaf, leaves per pod, pods
+  uint64_t n;     // instances
+  uint64_t n_node, n_leaf, n_pod;
+};
+
+Tree make_tree(const uint32_t* fanout) {
+  Tree t;
+  for (int k = 0; k < 4; ++k) t.f[k] = fanout[k];
+  t.n_pod = t.f[3];
+  t.n_leaf = t.n_pod * t.f[2];
+  t.n_node = t.n_leaf * t.f[1];
+  t.n = t.n_node * t.f[0];
+  return t;
+}
+
+// Ancestor of instance i at height h: h=0 the instance, 1 its node, 2 its leaf,
+// 3 its pod, 4 the spine (index 0).
+uint64_t ancestor(const Tree& t, uint64_t i, int h) {
+  uint64_t a = i;
+  for (int k = 0; k < h && k < 4; ++k) a /= t.f[k];
+  return h >= 4 ? 0 : a;
+}
+
+// Link from the height-h ancestor of i up to its parent.  Links are numbered in
+// consecutive blocks per level: instance-node links [0, N), node-leaf links
+// [N, N + n_node), leaf-pod links next, pod-spine links last.
+uint64_t uplink(const Tree& t, uint64_t i, int h) {
+  uint64_t base = 0;
+  const uint64_t block[4] = {t.n, t.n_node, t.n_leaf, t.n_pod};
+  for (int k = 0; k < h; ++k) base += block[k];
+  return base + ancestor(t, i, h);
+}
+
+// Locality tier: the lowest height h such that i and j share their height-(h+1) ancestor.
+int tier(const Tree& t, uint64_t i, uint64_t j) {
+  for (int h = 0; h < 4; ++h)
+    if (ancestor(t, i, h + 1) == ancestor(t, j, h + 1)) return h;
+  return 3;
+}
+
+// Bottleneck residual bandwidth over the unique tree path between i and j.
+double path_bottleneck(const Tree& t, const double* bw, const float* u_row,
+                       uint64_t i, uint64_t j, int* tau_out) {
+  const int tau = tier(t, i, j);
+  double b = std::numeric_limits<double>::infinity();
+  for (int h = 0; h <= tau; ++h) {
+    const uint64_t ei = uplink(t, i, h), ej = uplink(t, j, h);
+    const double ri = bw[h] * (1.0 - (double)u_row[ei]);
+    const double rj = bw[h] * (1.0 - (double)u_row[ej]);
+    if (ri < b) b = ri;
+    if (rj < b) b = rj;
+  }
+  if (tau_out) *tau_out = tau;
+  return b;
+}
+
+void ranks(const uint8_t* role, uint64_t n, std::vector<uint64_t>& pre, std::vector<uint64_t>& dec) {
+  pre.clear();
+  dec.clear();
+  for (uint64_t i = 0; i < n; ++i) (role[i] ? dec : pre).push_back(i);
+}
+
+}  // namespace
+
+extern "C" {
+
+// ---------------------------------------------------------------- closed forms
+// Eq. 1: bytes of KV cache per token, s_r / l_r.
+double oracle_kv_bytes_per_token(uint32_t n_layers, uint32_t n_kv_heads, uint32_t d_head,
+                                 uint32_t b_elem) {
+  return 2.0 * n_layers * n_kv_heads * d_head * (double)b_elem;
+}
+
+// Eq. 4: per-tier effective bandwidth with the self-contention count.
+double oracle_beff_tier(double B_tau, double c_tau, double n_inflight) {
+  return B_tau * (1.0 - c_tau) / (1.0 + n_inflight);
+}
+
+// Eq. 3: transfer time of s bytes.
+double oracle_transfer_time(double s, double B_eff, double L_tau) { return s / B_eff + L_tau; }
+
+// Eq. 2: effective transfer size after a lambda-token prefix hit.
+double oracle_s_eff(double s_r, double lambda, double l_r) { return s_r * (1.0 - lambda / l_r); }
+
+// ---------------------------------------------------------------- topology
+int oracle_tier(const uint32_t* fanout, uint64_t i, uint64_t j) {
+  return tier(make_tree(fanout), i, j);
+}
+
+// Links on the path between instances i and j (at most 8); returns the count.
+int oracle_path_links(const uint32_t* fanout, uint64_t i, uint64_t j, uint64_t* links, int* levels) {
+  const Tree t = make_tree(fanout);
+  const int tau = tier(t, i, j);
+  int n = 0;
+  for (int h = 0; h <= tau; ++h) {
+    links[n] = uplink(t, i, h); levels[n++] = h;
+    links[n] = uplink(t, j, h); levels[n++] = h;
+  }
+  return n;
+}
+
+uint64_t oracle_used_links(const uint32_t* fanout) {
+  const Tree t = make_tree(fanout);
+  return t.n + t.n_node + t.n_leaf + t.n_pod;
+}
+
+// ---------------------------------------------------------------- oracle matrix
+// C[s][p][d] = kv / Bbot(s,p,d) + L_tau(p,d), p over prefill ranks, d over decode
+// ranks (ranks = role order), util [n_snap][n_links].
+void oracle_cost_matrix(const uint32_t* fanout, const uint8_t* role, const double* bw,
+                        const double* lat, const float* util, uint64_t n_links,
+                        uint64_t n_snap, double kv_bytes, double* C) {
+  const Tree t = make_tree(fanout);
+  std::vector<uint64_t> pre, dec;
+  ranks(role, t.n, pre, dec);
+  const uint64_t P = pre.size(), D = dec.size();
+#pragma omp parallel for collapse(2) schedule(static)
+  for (uint64_t s = 0; s < n_snap; ++s)
+    for (uint64_t p = 0; p < P; ++p)
+      for (uint64_t d = 0; d < D; ++d) {
+        int tau = 0;
+        const double b = path_bottleneck(t, bw, util + s * n_links, pre[p], dec[d], &tau);
+        C[(s * P + p) * D + d] = kv_bytes / b + lat[tau];
+      }
+}
+
+// Selected entries (s[k], p[k], d[k]) of the same matrix; util rows indexed by s[k].
+void oracle_cost_entries(const uint32_t* fanout, const uint8_t* role, const double* bw,
+                         const double* lat, const float* util, uint64_t n_links,
+                         const uint64_t* s, const uint64_t* p, const uint64_t* d, uint64_t n,
+                         double kv_bytes, double* out) {
+  const Tree t = make_tree(fanout);
+  std::vector<uint64_t> pre, dec;
+  ranks(role, t.n, pre, dec);
+#pragma omp parallel for schedule(static)
+  for (uint64_t k = 0; k < n; ++k) {
+    int tau = 0;
+    const double b = path_bottleneck(t, bw, util + s[k] * n_links, pre[p[k]], dec[d[k]], &tau);
+    out[k] = kv_bytes / b + lat[tau];
+  }
+}
+
+// Bottleneck of the up path from instance i to its height-(k+1) ancestor, for every
+// instance and k = 0..3: UB[s][i][k] = min over h <= k of bw[h] * (1 - u[s][uplink(i,h)]).
+void oracle_up_bottleneck(const uint32_t* fanout, const double* bw, const float* util,
+                          uint64_t n_links, uint64_t n_snap, double* UB) {
+  const Tree t = make_tree(fanout);
+#pragma omp parallel for collapse(2) schedule(static)
+  for (uint64_t s = 0; s < n_snap; ++s)
+    for (uint64_t i = 0; i < t.n; ++i) {
+      double b = std::numeric_limits<double>::infinity();
+      for (int k = 0; k < 4; ++k) {
+        const double r = bw[k] * (1.0 - (double)util[s * n_links + uplink(t, i, k)]);
+        if (r < b) b = r;
+        UB[(s * t.n + i) * 4 + k] = b;
+      }
+    }
+}
+
+// ---------------------------------------------------------------- prefix match
+// M[r][d] = number of leading blocks of chain r found in cache K_{g(r),d}, where the
+// cache of (set g, decode d) is the key list keys[key_off[g*D+d] .. key_off[g*D+d+1]),
+// and set g serves requests [set_off[g], set_off[g+1]).  The scan stops at the first
+// block that is not cached.
+void oracle_prefix_match(const uint64_t* keys, const uint64_t* key_off, uint32_t D,
+                         const uint64_t* chains, const uint64_t* chain_off, uint32_t R,
+                         const uint32_t* set_off, uint32_t n_sets, uint16_t* M) {
+  for (uint32_t g = 0; g < n_sets; ++g) {
+    std::vector<std::unordered_set<uint64_t>> K(D);
+    for (uint32_t d = 0; d < D; ++d) {
+      const uint64_t t = (uint64_t)g * D + d;
+      K[d].reserve(key_off[t + 1] - key_off[t]);
+      for (uint64_t j = key_off[t]; j < key_off[t + 1]; ++j) K[d].insert(keys[j]);
+    }
+#pragma omp parallel for schedule(dynamic, 16)
+    for (int64_t r = set_off[g]; r < (int64_t)set_off[g + 1]; ++r) {
+      for (uint32_t d = 0; d < D; ++d) {
+        uint64_t m = 0;
+        for (uint64_t j = chain_off[r]; j < chain_off[r + 1]; ++j) {
+          if (K[d].count(chains[j]) == 0) break;
+          ++m;
+        }
+        M[(uint64_t)r * D + d] = (uint16_t)m;
+      }
+    }
+  }
+  (void)R;
+}
+
+// Prefix match of selected requests against ONE cache (key list), for sampled checks:
+// out[k] = leading blocks of chain k (chains[chain_off[k]..chain_off[k+1])) found in keys.
+void oracle_prefix_match_one(const uint64_t* keys, uint64_t n_keys, const uint64_t* chains,
+                             const uint64_t* chain_off, uint64_t n, uint16_t* out) {
+  std::unordered_set<uint64_t> K(keys, keys + n_keys);
+  for (uint64_t k = 0; k < n; ++k) {
+    uint64_t m = 0;
+    for (uint64_t j = chain_off[k]; j < chain_off[k + 1]; ++j) {
+      if (K.count(chains[j]) == 0) break;
+      ++m;
+    }
+    out[k] = (uint16_t)m;
+  }
+}
+
+// ---------------------------------------------------------------- greedy
+// One stream of Algorithm 1 with the weighted score
+//   score(d) = w_net * T_xfer(d) + w_prefix * miss(d) + w_load * theta * load[d],
+//   T_xfer(d) = s_eff(d) / Bbot(k_r, p_r, d) + L_tau,  s_eff(d) = (l - 16 M[r][d]) * bpt,
+//   miss(d)   = (l - 16 M[r][d]) / l,
+// feasible iff load[d] + l <= cap.  Events are processed in order: a departure of a
+// dispatched request releases its tokens; an arrival picks the feasible candidate of
+// minimum score (lowest index among equal scores) or is rejected (-1), then adds its
+// tokens to the chosen decode.
+//
+// hint (nullable): decisions of another implementation.  Where hint[r] differs from the
+// oracle's choice, the step is a near-tie when hint[r] is feasible and its score is
+// within rel_tol * best of the best score, and a mismatch otherwise; in both cases the
+// oracle continues from hint[r] so that later steps are compared from the same state.
+// counts[0] += near-ties, counts[1] += mismatches, counts[2] += rejects.
+//
+// best/second: the minimum score and the minimum over the other feasible candidates
+// (+inf when absent), both from the oracle's own scores.
+void oracle_schedule_stream(const uint32_t* fanout, const uint8_t* role, const double* bw,
+                            const double* lat, const float* util, uint64_t n_links,
+                            const uint32_t* len, const uint32_t* prefill, const uint32_t* snap,
+                            const uint16_t* M, const uint32_t* events, uint64_t n_events,
+                            double w_net, double w_prefix, double w_load, double theta,
+                            int64_t cap, uint64_t bytes_per_token, const int64_t* load_init,
+                            const int32_t* hint, double rel_tol, int32_t* dec, double* best,
+                            double* second, int64_t* load_out, int64_t* counts) {
+  const Tree t = make_tree(fanout);
+  std::vector<uint64_t> pre, decs;
+  ranks(role, t.n, pre, decs);
+  const uint64_t D = decs.size();
+  std::vector<int64_t> load(D, 0);
+  if (load_init)
+    for (uint64_t d = 0; d < D; ++d) load[d] = load_init[d];
+  std::vector<double> score(D);
+  const double inf = std::numeric_limits<double>::infinity();
+
+  for (uint64_t e = 0; e < n_events; ++e) {
+    const uint32_t code = events[e];
+    const uint32_t r = code & 0x7fffffffu;
+    const int64_t l = len[r];
+    if (code >> 31) {  // departure
+      if (dec[r] >= 0) load[dec[r]] -= l;
+      continue;
+    }
+    const float* u_row = util + (uint64_t)snap[r] * n_links;
+    const uint64_t p = pre[prefill[r]];
+    int32_t arg = -1;
+    for (uint64_t d = 0; d < D; ++d) {
+      if (load[d] + l > cap) { score[d] = inf; continue; }
+      int tau = 0;
+      const double b = path_bottleneck(t, bw, u_row, p, decs[d], &tau);
+      const int64_t lam = 16 * (int64_t)M[(uint64_t)r * D + d];
+      const double s_eff = (double)((l - lam) * (int64_t)bytes_per_token);
+      const double T = s_eff / b + lat[tau];
+      const double miss = (double)(l - lam) / (double)l;
+      score[d] = w_net * T + w_prefix * miss + w_load * (theta * (double)load[d]);
+      if (arg < 0 || score[d] < score[arg]) arg = (int32_t)d;
+    }
+    double b1 = inf, b2 = inf;
+    if (arg >= 0) {
+      b1 = score[arg];
+      for (uint64_t d = 0; d < D; ++d)
+        if ((int32_t)d != arg && score[d] < b2) b2 = score[d];
+    }
+    int32_t chosen = arg;
+    if (hint && hint[r] != arg) {
+      const int32_t h = hint[r];
+      const bool near = (arg >= 0 && h >= 0 && (uint64_t)h < D && score[h] != inf &&
+                         score[h] - b1 <= rel_tol * std::fabs(b1));
+      counts[near ? 0 : 1] += 1;
+      chosen = (h >= 0 && (uint64_t)h < D) ? h : -1;
+    }
+    if (chosen < 0) counts[2] += 1;
+    dec[r] = chosen;
+    best[r] = b1;
+    second[r] = b2;
+    if (chosen >= 0) load[chosen] += l;
+  }
+  for (uint64_t d = 0; d < D; ++d) load_out[d] = load[d];
+}
+
+}  // extern "C"

@@ -1,0 +1,132 @@
+"""A second, deliberately naive evaluator used only to pin the C++ oracle.
+
+It shares nothing with the oracle: the instance tree is built as an explicit
+graph (named vertices, adjacency lists), paths come from breadth-first search,
+prefix hits from a list scan, and scores are exact rationals (``fractions``),
+so every comparison is free of rounding.  Only tiny instances are feasible.
+"""
+from __future__ import annotations
+
+from collections import deque
+from fractions import Fraction
+from typing import Dict, List, Sequence, Tuple
+
+import numpy as np
+
+
+class ExplicitTree:
+    """Vertices: ('inst', i), ('node', n), ('leaf', l), ('pod', q), ('spine',).
+
+    Edge ids follow the link numbering of the library's interface: instance-node
+    links first (by instance), then node-leaf links (by node), leaf-pod links (by
+    leaf), pod-spine links (by pod).  Each edge also records its level 0..3.
+    """
+
+    def __init__(self, fanout: Sequence[int]):
+        f0, f1, f2, f3 = fanout
+        self.n = f0 * f1 * f2 * f3
+        n_node, n_leaf, n_pod = self.n // f0, self.n // (f0 * f1), f3
+        self.adj: Dict[tuple, List[Tuple[tuple, int]]] = {}
+        self.level: Dict[int, int] = {}
+        eid = 0
+
+        def add(a, b, lvl):
+            nonlocal eid
+            self.adj.setdefault(a, []).append((b, eid))
+            self.adj.setdefault(b, []).append((a, eid))
+            self.level[eid] = lvl
+            eid += 1
+
+        for i in range(self.n):
+            add(("inst", i), ("node", i // f0), 0)
+        for nd in range(n_node):
+            add(("node", nd), ("leaf", nd // f1), 1)
+        for lf in range(n_leaf):
+            add(("leaf", lf), ("pod", lf // f2), 2)
+        for q in range(n_pod):
+            add(("pod", q), ("spine",), 3)
+        self.n_edges = eid
+
+    def path(self, i: int, j: int) -> List[int]:
+        src, dst = ("inst", i), ("inst", j)
+        prev = {src: None}
+        q = deque([src])
+        while q:
+            v = q.popleft()
+            if v == dst:
+                break
+            for w, e in self.adj[v]:
+                if w not in prev:
+                    prev[w] = (v, e)
+                    q.append(w)
+        edges = []
+        v = dst
+        while prev[v] is not None:
+            v, e = prev[v]
+            edges.append(e)
+        return edges[::-1]
+
+    def tier(self, i: int, j: int) -> int:
+        # the highest level among the path's edges is the tier of the pair
+        return max(self.level[e] for e in self.path(i, j))
+
+
+def frac(x) -> Fraction:
+    return Fraction(float(x))
+
+
+def bottleneck(tree: ExplicitTree, bw, u_row, i, j) -> Fraction:
+    return min(frac(bw[tree.level[e]]) * (1 - frac(u_row[e])) for e in tree.path(i, j))
+
+
+def cost(tree, bw, lat, u_row, i, j, kv) -> Fraction:
+    return frac(kv) / bottleneck(tree, bw, u_row, i, j) + frac(lat[tree.tier(i, j)])
+
+
+def lcp_blocks(chain: Sequence[int], cache: Sequence[int]) -> int:
+    m = 0
+    for h in chain:
+        if h not in cache:
+            break
+        m += 1
+    return m
+
+
+def greedy_exact(tree, role, bw, lat, util, length, prefill, snap, M, events,
+                 w, theta, cap, bpt):
+    """Exact-rational Algorithm 1 with the weighted score; returns (dec, best_scores)."""
+    pre = [i for i in range(tree.n) if role[i] == 0]
+    dec_inst = [i for i in range(tree.n) if role[i] == 1]
+    D = len(dec_inst)
+    load = [0] * D
+    R = len(length)
+    dec = [-1] * R
+    best = [None] * R
+    wn, wp, wl = (frac(x) for x in w)
+    th = frac(theta)
+    for code in events:
+        code = int(code)
+        r = code & 0x7FFFFFFF
+        l = int(length[r])
+        if code >> 31:
+            if dec[r] >= 0:
+                load[dec[r]] -= l
+            continue
+        p = pre[int(prefill[r])]
+        u_row = util[int(snap[r])]
+        scores = []
+        for d in range(D):
+            if load[d] + l > cap:
+                scores.append(None)
+                continue
+            miss_tok = l - 16 * int(M[r][d])
+            T = Fraction(miss_tok * bpt) / bottleneck(tree, bw, u_row, p, dec_inst[d]) \
+                + frac(lat[tree.tier(p, dec_inst[d])])
+            scores.append(wn * T + wp * Fraction(miss_tok, l) + wl * th * load[d])
+        cands = [(s, d) for d, s in enumerate(scores) if s is not None]
+        if cands:
+            s, d = min(cands)
+            dec[r] = d
+            best[r] = s
+            load[d] += l
+    return dec, best, load
