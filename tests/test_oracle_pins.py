@@ -488,3 +488,34 @@ def test_proposition2_ranking_robustness():
             assert not order(a, b)
             tested += 1
     assert tested > 30
+
+
+def test_prefix_match_tables_with_holes():
+    """Multi-table form: two sets of two caches each, caches with holes in the chain."""
+    chains = np.array([1, 2, 3, 4, 5,   1, 2, 3,   9, 2, 3], np.uint64)
+    chain_off = np.array([0, 5, 8, 11], np.uint64)
+    set_off = np.array([0, 2, 3], np.uint32)           # set 0: requests 0,1; set 1: request 2
+    caches = [[1, 2, 4, 5], [1, 2, 3, 4, 5],           # set 0, decodes 0 and 1
+              [2, 3, 9], [9, 3]]                       # set 1, decodes 0 and 1
+    keys = np.concatenate([np.array(c, np.uint64) for c in caches])
+    key_off = np.concatenate([[0], np.cumsum([len(c) for c in caches])]).astype(np.uint64)
+    M = oracle.prefix_match(keys, key_off, 2, chains, chain_off, set_off)
+    expect = [[2, 5], [2, 3], [3, 1]]
+    np.testing.assert_array_equal(M, np.array(expect, np.uint16))
+    for r in range(3):
+        g = 0 if r < 2 else 1
+        for d in range(2):
+            assert M[r, d] == naive.lcp_blocks(list(chains[chain_off[r]:chain_off[r + 1]]),
+                                               caches[2 * g + d])
+
+
+def test_greedy_capacity_boundary_is_inclusive():
+    """Line 1 of Algorithm 1 keeps a candidate whose free capacity equals the demand."""
+    pb = _tiny_problem(4, R=6)
+    l0 = int(pb["length"][0])
+    pb["cap"] = l0
+    res = _run_oracle(pb, (1.0, 1.0, 1.0))
+    assert res.dec[0] >= 0
+    pb["cap"] = l0 - 1
+    res = _run_oracle(pb, (1.0, 1.0, 1.0))
+    assert res.dec[0] == -1
