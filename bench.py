@@ -1,0 +1,351 @@
+#!/usr/bin/env python
+"""Benchmark of the NetKV scoring path on GB300.
+
+Workload: 4,096 independent replicas of the single-stream 64-GPU cluster
+(8 prefill + 8 decode instances at TP=4, 1,000 requests each, decode caches of
+200K block hashes in 2^19-slot tables), run as 4,096 concurrent streams whose
+score weights cover a 16x16x16 grid.  One step is the whole hot path over all
+streams: level bottlenecks of every telemetry snapshot (netkv_oracle_build),
+prefix hits of every (request, decode) pair (netkv_prefix_match) and the greedy
+of every stream (netkv_schedule_streams).  The decode caches are resident state
+built once before timing (netkv_cache_build).
+
+Prints one JSON line.  ``--impl reference`` times the CPU oracle instead, on a
+bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "decisions/sec"
+UNIT = "decisions/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="netkv", choices=["netkv", "reference"])
+    ap.add_argument("--streams", type=int, default=4096)
+    ap.add_argument("--cpu-streams", type=int, default=24)
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--table-batch", type=int, default=256)
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def workload_config(streams, world, extra=None):
+    cfg = {"workload": f"{streams} replicas x 64-GPU four-tier tree (8P+8D, TP=4), "
+                       "1,000 requests/stream, 2^19-slot caches of 200K blocks",
+           "streams_per_gpu": streams, "requests_per_stream": 1000, "decodes": 8,
+           "prefills": 8, "parallelism": f"replicas{world}",
+           "l2": "inputs larger than L2 (tables 128 GiB + chains 27 GB per GPU)"}
+    if extra:
+        cfg.update(extra)
+    return cfg
+
+
+# ------------------------------------------------------------------ clocks
+class Clocks:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+# ------------------------------------------------------------------ CPU oracle
+def cpu_oracle_sample(w, streams, theta, cap, bpt):
+    """Time the CPU oracle on whole streams of the workload; returns (decisions, seconds)."""
+    from oracle.workload import run_stream
+    t0 = time.perf_counter()
+    dec = 0
+    for s in streams:
+        res = run_stream(w, int(s), theta, cap, bpt)
+        dec += int(res.dec.shape[0])
+    return dec, time.perf_counter() - t0
+
+
+def cpu_cores():
+    return int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+
+
+# ------------------------------------------------------------------ reference arm
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    import synth
+    spec = synth.config1(args.streams)
+    w = synth.make_workload(spec)
+    theta = float(np.float32(synth.THETA_S_PER_TOKEN))
+    per_step = max(1, min(4, args.streams))
+    order = np.random.default_rng(1).permutation(args.streams)
+    k = 0
+    for _ in range(args.warmup):
+        cpu_oracle_sample(w, order[k:k + per_step], theta, spec.cap_tokens, synth.BYTES_PER_TOKEN_SHARD)
+        k = (k + per_step) % args.streams
+    dec_total, secs = 0, 0.0
+    for _ in range(args.steps):
+        d, s = cpu_oracle_sample(w, order[k:k + per_step], theta, spec.cap_tokens,
+                                 synth.BYTES_PER_TOKEN_SHARD)
+        dec_total += d
+        secs += s
+        k = (k + per_step) % args.streams
+    value = dec_total / secs
+    sample = f"{per_step} whole streams per step (prefix match + greedy + level bottlenecks)"
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * secs / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(args.streams, world),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------ GPU arm
+def run_netkv(args):
+    import torch
+    import synth
+    import synth.device as sdev
+    from synth import stage
+    import __graft_entry__
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    __graft_entry__.build()
+    from paper_2606_03910_gb300.pipeline import Scorer, StepInputs, weights_tensor
+
+    spec = synth.config1(args.streams)
+    spec.seed0 = rank * args.streams               # weak scaling: each GPU its own replicas
+    w = synth.make_workload(spec)
+    theta = float(np.float32(synth.THETA_S_PER_TOKEN))
+    bpt = synth.BYTES_PER_TOKEN_SHARD
+
+    # resident caches, built in batches of table sets
+    sc = Scorer(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, w.L, w.n_sets, spec.log2_cap,
+                device=dev)
+    for g0 in range(0, w.n_sets, args.table_batch):
+        g1 = min(w.n_sets, g0 + args.table_batch)
+        keys = sdev.keys(w, g0, g1, device=dev)
+        sc.load_caches(keys, stage.key_offsets(w, (g1 - g0) * w.D, device=dev), set0=g0,
+                       n_sets=g1 - g0)
+        del keys
+    torch.cuda.synchronize()
+
+    ra = stage.request_arrays(w, device=dev)
+    chains, _ = sdev.chains(w, device=dev)
+    x = StepInputs(util=sdev.util(w, device=dev), chains=chains, chain_off=ra["chain_off"],
+                   set_off=ra["set_off"], length=ra["length"], prefill=ra["prefill"],
+                   snap=ra["snap"], events=ra["events"], event_off=ra["event_off"],
+                   weights=weights_tensor(w.weights, theta, spec.cap_tokens, bpt, device=dev))
+    out = sc.alloc_outputs(x.n_snap, x.R, x.n_streams)
+    stream = torch.cuda.current_stream(dev)
+    for _ in range(args.warmup):
+        sc.step(x, out, stream)
+    torch.cuda.synchronize()
+    if int(out.status.item()) != 0:
+        raise RuntimeError(f"device status {int(out.status.item())} after warm-up")
+
+    # ---- timed region: device-resident inputs
+    names = ("oracle_build", "prefix_match", "schedule")
+    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in names] for _ in range(args.steps)]
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = Clocks(local)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    t0.record(stream)
+    for k in range(args.steps):
+        for j, fn in enumerate((sc.oracle_build, sc.prefix_match, sc.schedule)):
+            ev[k][j][0].record(stream)
+            fn(x, out, stream)
+            ev[k][j][1].record(stream)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    if world > 1:
+        dist.barrier()
+    ms = t0.elapsed_time(t1) / args.steps
+    per_kernel = {n: sum(ev[k][j][0].elapsed_time(ev[k][j][1]) for k in range(args.steps)) / args.steps
+                  for j, n in enumerate(names)}
+    if world > 1:
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    status = int(out.status.item())
+    if status != 0:
+        raise RuntimeError(f"device status {status} in the timed region")
+
+    R, D = x.R, sc.D
+    decisions = R * world
+    value = decisions / (ms / 1e3)
+
+    # ---- roofline of the dominant kernel
+    M = out.M.to(torch.int32) & 0xFFFF
+    nblk = (x.chain_off[1:] - x.chain_off[:-1]).to(torch.int32)
+    probes = int(torch.minimum(M + 1, nblk[:, None]).sum().item())
+    n_arr = R
+    n_dep = R
+    algo = {
+        # 8-byte chain block + 8-byte table slot per probe, 2-byte M store per pair
+        "prefix_match": 16 * probes + 2 * R * D,
+        # per snapshot: the utilisation row (L floats), 16-byte UB of every instance
+        "oracle_build": x.n_snap * (4 * w.L + 16 * sc.N),
+        # per arrival: event, len/prefill/snap, UB of the prefill, per candidate M (2 B)
+        # and its UB entry (4 B), dec/best/second stores; per departure: event, len, dec
+        "schedule": n_arr * (4 + 12 + 16 + D * 6 + 12) + n_dep * 12 + 2 * 8 * D * x.n_streams,
+    }
+    dom = max(per_kernel, key=per_kernel.get)
+    peak, peak_src = measured_peaks()
+    achieved = algo[dom] / (per_kernel[dom] / 1e3) / 1e9
+    roofline = {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+                "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": None,
+                "peak_source": peak_src,
+                "algorithmic_bytes_per_launch": algo[dom],
+                "kernel_ms": {k: round(v, 4) for k, v in per_kernel.items()},
+                "probes_per_launch": probes}
+
+    # ---- end to end through the public API with pinned host buffers
+    e2e = None
+    if not args.no_e2e:
+        import dataclasses
+        xh = StepInputs(**{f.name: (getattr(x, f.name).cpu().pin_memory()
+                                    if isinstance(getattr(x, f.name), torch.Tensor) else None)
+                           for f in dataclasses.fields(StepInputs)})
+        res_h = {k: torch.empty_like(getattr(out, k), device="cpu").pin_memory()
+                 for k in ("dec", "best", "second", "load_final")}
+        h2d = xh.nbytes()
+        d2h = sum(int(t.numel() * t.element_size()) for t in res_h.values())
+        for _ in range(max(1, args.warmup)):
+            sc.step_host(xh, x, out, res_h, stream)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            sc.step_host(xh, x, out, res_h, stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ems = e0.elapsed_time(e1) / args.steps
+        if world > 1:
+            tt = torch.tensor([ems], device=dev)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            ems = float(tt.item())
+        e2e = {"value": decisions / (ems / 1e3), "unit": UNIT, "ms_per_step": round(ems, 3),
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    # ---- CPU oracle baseline, rank 0 at N=1 only
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        sample = np.random.default_rng(0).choice(args.streams, size=min(args.cpu_streams, args.streams),
+                                                 replace=False)
+        d, secs = cpu_oracle_sample(w, sample, theta, spec.cap_tokens, bpt)
+        cpu = {"value": d / secs, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+               "sample": f"{len(sample)} of {args.streams} streams, whole streams "
+                         f"({d} decisions in {secs:.1f} s)"}
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": "f32", "data": "synthetic",
+                "config": workload_config(args.streams, world),
+                "scores_per_s": value * D, "gpu_launches": 3 * args.steps,
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_netkv(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

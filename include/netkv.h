@@ -1,0 +1,212 @@
+/*
+ * netkv.h -- C ABI of the NetKV decode-instance scoring library (sm_103a).
+ *
+ * NetKV (arXiv 2606.03910) places each prefilled request on the decode instance
+ * that minimises a cost made of the KV-cache transfer time over the network
+ * (Sec. III-D, Eq. 3 and Eq. 4), the prefix-cache locality (Sec. III-B, Eq. 2)
+ * and the compute load (Sec. IV-A), by a per-request greedy over the decode pool
+ * (Algorithm 1, Sec. V-A).  This library runs that scoring path on one GPU:
+ *
+ *   netkv_topology_create   the four-tier instance tree (Sec. III-A, III-E)
+ *   netkv_oracle_build      network cost oracle C[s][p][d] from per-link utilisation
+ *                           snapshots, and the per-instance level bottlenecks UB
+ *   netkv_cache_build       decode caches K_d as open-addressing hash tables
+ *   netkv_prefix_match      block-level prefix hit M[r][d] (Sec. III-B)
+ *   netkv_schedule_streams  the greedy of Algorithm 1 over independent streams
+ *
+ * Conventions for every call:
+ *   - Pointers named d_* are device pointers owned by the caller; the library never
+ *     frees them and keeps no reference after the call returns.  Other pointers are
+ *     host pointers read during the call only.
+ *   - Work is enqueued on `stream` (NULL = the legacy default stream) and runs
+ *     asynchronously; the call returns once the work is enqueued.
+ *   - The return value reports errors found on the host (bad sizes, NULL pointers,
+ *     unaligned buffers, failed CUDA launches) before anything is enqueued, except
+ *     NETKV_ECUDA, which may follow a partial enqueue.
+ *   - Errors found while the kernels run are OR-ed into *d_status (a device int the
+ *     caller zeroes once and reads after synchronising) as NETKV_DEV_* bits.  No kernel
+ *     traps; a flagged kernel still completes, with the affected outputs defined as
+ *     stated per call.
+ *   - No global mutable state: calls on different streams and threads may overlap as
+ *     long as they do not write the same buffers.  A topology handle is immutable
+ *     after creation and may be shared.
+ */
+#ifndef NETKV_H
+#define NETKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* netkv_stream_t; /* identical to cudaStream_t */
+
+typedef enum {
+  NETKV_OK = 0,
+  NETKV_EINVAL = 1, /* argument out of range, NULL where required, misaligned buffer */
+  NETKV_ENOMEM = 2, /* host or device allocation for a topology handle failed */
+  NETKV_ECUDA = 3   /* a CUDA runtime call or kernel launch failed */
+} netkv_status;
+
+/* Bits OR-ed into *d_status by the kernels. */
+#define NETKV_DEV_EDOMAIN 1 /* utilisation outside [0,1) or NaN; zero-length request;
+                               hash value 0 in a chain or key list; M[r][d] > len/16 */
+#define NETKV_DEV_EFULL 2   /* a hash table had no free slot, or a probe ran the whole table */
+#define NETKV_DEV_ERANGE 4  /* a request, prefill rank or snapshot index out of range */
+
+/* ------------------------------------------------------------------ topology
+ * The cluster is a four-level tree (Sec. III-A): fanout[0] instances per node,
+ * fanout[1] nodes per leaf (rack / ToR), fanout[2] leaves per pod, fanout[3] pods
+ * under the spine.  Instances are numbered depth-first, pod-major: instance i sits
+ * in node i/f0, leaf i/(f0 f1), pod i/(f0 f1 f2).  The locality tier tau(p,d) of a
+ * pair is 0 (same node), 1 (same leaf), 2 (same pod) or 3 (Sec. III-A).
+ *
+ * Links (the entries of a utilisation snapshot) are numbered in blocks by level:
+ *   level 0  instance-node links  [0, N)                     link of instance i = i
+ *   level 1  node-leaf links      [N, N + N/f0)              link of node n = N + n
+ *   level 2  leaf-pod links       next N/(f0 f1)             by leaf
+ *   level 3  pod-spine links      next f3                    by pod
+ * The path between p and d uses the links of levels 0..tau(p,d) above p and above d.
+ * A snapshot row holds n_links >= used links floats; entries past the used links are
+ * padding and are never read.
+ *
+ * Prefill ranks number the instances with role 0 in instance order, decode ranks the
+ * instances with role 1; every other argument indexes instances by these ranks.
+ */
+typedef struct netkv_topology* netkv_topology_t;
+
+typedef struct {
+  uint32_t fanout[4];     /* instances/node, nodes/leaf, leaves/pod, pods; each >= 1 */
+  const uint8_t* role;    /* host [N], N = product of fanouts: 0 prefill, 1 decode */
+  double tier_bw_Bps[4];  /* B_k: bandwidth of a level-k link, bytes/s, > 0 (Sec. III-A) */
+  double tier_lat_s[4];   /* L_k: base latency of a tier-k transfer, seconds, >= 0 */
+  uint32_t n_links;       /* utilisation row length (>= used links) */
+} netkv_topology_desc;
+
+/* Validates desc, builds the instance tables and copies them to the current device.
+ * N must be below 2^31 and P, D >= 1.  Synchronous; allocates the handle and its
+ * device mirror (freed by netkv_topology_destroy). */
+netkv_status netkv_topology_create(const netkv_topology_desc* desc, netkv_topology_t* out);
+netkv_status netkv_topology_destroy(netkv_topology_t topo);
+/* Any output pointer may be NULL. */
+netkv_status netkv_topology_query(netkv_topology_t topo, uint32_t* n_instances, uint32_t* P,
+                                  uint32_t* D, uint32_t* used_links);
+
+/* ------------------------------------------------------------------ oracle
+ * Network cost oracle (Sec. III-D, Sec. III-E) with per-link congestion: for snapshot
+ * s, prefill rank p and decode rank d,
+ *     Bbot(s,p,d) = min over links e on the path of  B_level(e) * (1 - u[s][e])
+ *     C[s][p][d]  = kv_bytes / Bbot(s,p,d) + L_tau(p,d)
+ * i.e. Eq. 3 with Eq. 4's residual bandwidth taken at the bottleneck link and the
+ * self-contention count at zero.  fp32 arithmetic; C is correctly-rounded division
+ * of fp32 operands followed by an fp32 add.
+ *
+ *   d_util  [n_snap][n_links] fp32 utilisations in [0,1)
+ *   d_C     [n_snap][P][D] fp32 output, row-major (d fastest), or NULL
+ *   d_UB    [n_snap][N][4] fp32 output, or NULL: the level bottlenecks
+ *           UB[s][i][k] = min over h <= k of B_h * (1 - u[s][link of i at level h]),
+ *           so that Bbot(s,p,d) = min(UB[s][p][tau], UB[s][d][tau]) (instances by index)
+ *   d_status device int, see NETKV_DEV_*.  Utilisations outside [0,1) set EDOMAIN and
+ *           the affected outputs are whatever the formula gives.
+ * At least one of d_C, d_UB must be non-NULL.  kv_bytes > 0.
+ */
+netkv_status netkv_oracle_build(netkv_topology_t topo, const float* d_util, uint32_t n_snap,
+                                double kv_bytes, float* d_C, float* d_UB, int* d_status,
+                                netkv_stream_t stream);
+
+/* ------------------------------------------------------------------ caches
+ * Decode caches K_d (Sec. III-C) as open-addressing tables of uint64 block hashes:
+ * n_tables tables of 2^log2_capacity slots each, contiguous, value 0 = empty slot
+ * (hash 0 is reserved).  Linear probing from a multiplicative hash of the key.
+ *
+ *   d_tables   [n_tables][2^log2_capacity] uint64, cleared then filled by this call
+ *   d_keys     keys of table t are d_keys[d_key_off[t] .. d_key_off[t+1])
+ *   d_key_off  [n_tables+1] uint64, non-decreasing
+ * Duplicate keys are stored once.  A zero key sets EDOMAIN and is skipped; a table
+ * with more distinct keys than slots sets EFULL (the excess keys are dropped).
+ * 1 <= log2_capacity <= 32.
+ */
+netkv_status netkv_cache_build(uint64_t* d_tables, uint64_t n_tables, uint32_t log2_capacity,
+                               const uint64_t* d_keys, const uint64_t* d_key_off,
+                               int* d_status, netkv_stream_t stream);
+
+/* ------------------------------------------------------------------ prefix match
+ * Block-level prefix hit (Sec. III-B): M[r][d] = number of leading blocks of request
+ * r's block-hash chain that are all present in decode d's cache; the cache hit in
+ * tokens is lambda = 16 * M (B_tok = 16).  The scan stops at the first missing block.
+ *
+ *   d_tables     [n_sets][D][2^log2_capacity] tables built by netkv_cache_build
+ *   d_chains     uint64 block hashes; chain r = d_chains[d_chain_off[r] .. d_chain_off[r+1])
+ *   d_chain_off  [R+1] uint64; every chain has at most 65535 blocks
+ *   d_set_off    [n_sets+1] uint32 request offsets: table set g serves requests
+ *                [d_set_off[g], d_set_off[g+1]); may be NULL when n_sets == 1
+ *   d_M          [R][D] uint16 output
+ * A zero hash in a chain sets EDOMAIN and counts as a miss.  A chain longer than 65535
+ * blocks sets EDOMAIN and its M saturates at 65535.
+ */
+netkv_status netkv_prefix_match(const uint64_t* d_tables, uint32_t D, uint32_t log2_capacity,
+                                uint32_t n_sets, const uint64_t* d_chains,
+                                const uint64_t* d_chain_off, uint32_t R,
+                                const uint32_t* d_set_off, uint16_t* d_M, int* d_status,
+                                netkv_stream_t stream);
+
+/* ------------------------------------------------------------------ greedy
+ * Per-stream weights and constants (device memory, one per stream).  Layout is fixed:
+ * 4 floats, then two 8-byte integers (32 bytes).
+ */
+typedef struct {
+  float w_net;             /* weight of the transfer time T_xfer, 1/s */
+  float w_prefix;          /* weight of the missed fraction (l - lambda)/l */
+  float w_load;            /* weight of the load term theta * load[d] */
+  float theta_s_per_token; /* seconds of queueing per active token on a decode */
+  int64_t cap_tokens;      /* capacity: d is feasible iff load[d] + l <= cap (Sec. IV-A) */
+  uint64_t bytes_per_token;/* KV bytes per token per GPU pair (Eq. 1 / TP) */
+} netkv_weights;
+
+/* Algorithm 1 (Sec. V-A) over n_streams independent streams, each a sequence of
+ * events processed in order.  For an arrival of request r (prefill rank p_r, length
+ * l_r tokens, telemetry snapshot k_r), every decode rank d gets
+ *     s_eff  = (l_r - 16 M[r][d]) * bytes_per_token                (Eq. 2, exact integer)
+ *     T_xfer = s_eff / min(UB[k_r][p][tau], UB[k_r][d][tau]) + L_tau  (Eq. 3, Eq. 4)
+ *     miss   = (l_r - 16 M[r][d]) / l_r
+ *     score  = w_net * T_xfer + w_prefix * miss + w_load * (theta * load[d])
+ * over the feasible set load[d] + l_r <= cap (line 1); the request goes to the feasible
+ * d of minimum score, the lowest d among equal scores (line 13), or is rejected (-1)
+ * when nothing is feasible (line 2); then load[d*] += l_r.  A departure event of a
+ * dispatched request subtracts its l from the decode that took it.
+ *
+ *   d_w          [n_streams] netkv_weights
+ *   d_len        [R] request length in tokens (>= 1)
+ *   d_prefill    [R] prefill rank of the request (< P)
+ *   d_snap       [R] snapshot index (< n_snap) into d_UB
+ *   d_M          [R][D] prefix hits from netkv_prefix_match
+ *   d_UB         [n_snap][N][4] level bottlenecks from netkv_oracle_build
+ *   d_events     uint32 codes: bit 31 set = departure, bits 0..30 = request index r;
+ *                stream j's events are d_events[d_event_off[j] .. d_event_off[j+1])
+ *   d_event_off  [n_streams+1] uint64
+ *   d_load_init  [n_streams][D] int64 initial loads, or NULL for zero (resume support)
+ *   d_dec        [R] int32 output: decision of each arrival handled (others untouched)
+ *   d_best       [R] fp32 output: minimum score (+inf when rejected)
+ *   d_second     [R] fp32 output: minimum over the other feasible candidates (+inf if none)
+ *   d_load_final [n_streams][D] int64 output: loads after the last event
+ * Every request index must occur in at most one stream, and its departure after its
+ * arrival.  Out-of-range indices set ERANGE and the event is skipped.
+ */
+netkv_status netkv_schedule_streams(netkv_topology_t topo, uint32_t n_streams,
+                                    const netkv_weights* d_w, uint32_t R, const uint32_t* d_len,
+                                    const uint32_t* d_prefill, const uint32_t* d_snap,
+                                    const uint16_t* d_M, const float* d_UB, uint32_t n_snap,
+                                    const uint32_t* d_events, const uint64_t* d_event_off,
+                                    const int64_t* d_load_init, int32_t* d_dec, float* d_best,
+                                    float* d_second, int64_t* d_load_final, int* d_status,
+                                    netkv_stream_t stream);
+
+/* Library version, for the bindings' load check. */
+uint32_t netkv_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* NETKV_H */

@@ -1,0 +1,179 @@
+"""Thin Python binding of the NetKV C ABI (``include/netkv.h``).
+
+Argument marshalling only: every function forwards to the entry point of the
+same name in ``libnetkv.so``; all computation happens in the CUDA kernels
+behind it.  Device buffers may be given as torch tensors (their ``data_ptr()``
+is passed) or as raw integer device addresses; ``None`` passes NULL.  A
+non-OK status raises :class:`NetKVError`.  There is no CPU fallback: if the
+library is missing, importing this module fails.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+from typing import Optional, Sequence
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libnetkv.so")
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(f"{LIB_PATH} is missing: build it first "
+                      "(python -c 'import __graft_entry__ as g; g.build()')")
+_lib = C.CDLL(LIB_PATH)
+
+NETKV_OK, NETKV_EINVAL, NETKV_ENOMEM, NETKV_ECUDA = 0, 1, 2, 3
+NETKV_DEV_EDOMAIN, NETKV_DEV_EFULL, NETKV_DEV_ERANGE = 1, 2, 4
+_NAMES = {1: "NETKV_EINVAL", 2: "NETKV_ENOMEM", 3: "NETKV_ECUDA"}
+
+EXPORTS = ("netkv_topology_create", "netkv_topology_destroy", "netkv_topology_query",
+           "netkv_oracle_build", "netkv_cache_build", "netkv_prefix_match",
+           "netkv_schedule_streams", "netkv_version")
+
+
+class NetKVError(RuntimeError):
+    def __init__(self, fn: str, code: int):
+        super().__init__(f"{fn} returned {_NAMES.get(code, code)}")
+        self.code = code
+
+
+class _Desc(C.Structure):
+    _fields_ = [("fanout", C.c_uint32 * 4), ("role", C.c_void_p),
+                ("tier_bw_Bps", C.c_double * 4), ("tier_lat_s", C.c_double * 4),
+                ("n_links", C.c_uint32)]
+
+
+# netkv_weights, 32 bytes: 4 x f32, i64, u64
+WEIGHTS_DTYPE = np.dtype([("w_net", "<f4"), ("w_prefix", "<f4"), ("w_load", "<f4"),
+                          ("theta_s_per_token", "<f4"), ("cap_tokens", "<i8"),
+                          ("bytes_per_token", "<u8")])
+assert WEIGHTS_DTYPE.itemsize == 32
+
+_P, _U32, _U64, _F64 = C.c_void_p, C.c_uint32, C.c_uint64, C.c_double
+_lib.netkv_version.restype = C.c_uint32
+_lib.netkv_topology_create.argtypes = [C.POINTER(_Desc), C.POINTER(C.c_void_p)]
+_lib.netkv_topology_destroy.argtypes = [_P]
+_lib.netkv_topology_query.argtypes = [_P, _P, _P, _P, _P]
+_lib.netkv_oracle_build.argtypes = [_P, _P, _U32, _F64, _P, _P, _P, _P]
+_lib.netkv_cache_build.argtypes = [_P, _U64, _U32, _P, _P, _P, _P]
+_lib.netkv_prefix_match.argtypes = [_P, _U32, _U32, _U32, _P, _P, _U32, _P, _P, _P, _P]
+_lib.netkv_schedule_streams.argtypes = [_P, _U32, _P, _U32, _P, _P, _P, _P, _P, _U32, _P, _P,
+                                        _P, _P, _P, _P, _P, _P, _P]
+for _f in EXPORTS:
+    if _f != "netkv_version":
+        getattr(_lib, _f).restype = C.c_int
+
+
+def _ptr(x) -> Optional[int]:
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return int(x.data_ptr())
+
+
+def _stream(s) -> Optional[int]:
+    if s is None:
+        import torch
+        return int(torch.cuda.current_stream().cuda_stream) if torch.cuda.is_initialized() else None
+    if isinstance(s, int):
+        return s
+    return int(s.cuda_stream)
+
+
+def _check(fn: str, code: int) -> None:
+    if code != NETKV_OK:
+        raise NetKVError(fn, code)
+
+
+def netkv_version() -> int:
+    return int(_lib.netkv_version())
+
+
+class Topology:
+    """Owns a netkv_topology_t handle (released by netkv_topology_destroy)."""
+
+    def __init__(self, handle: int):
+        self.handle = handle
+
+    @property
+    def as_parameter(self):
+        return self.handle
+
+    def __del__(self):
+        if getattr(self, "handle", None):
+            try:
+                _lib.netkv_topology_destroy(self.handle)
+            except Exception:
+                pass
+            self.handle = None
+
+
+def netkv_topology_create(fanout: Sequence[int], role: np.ndarray, tier_bw_Bps: Sequence[float],
+                          tier_lat_s: Sequence[float], n_links: int) -> Topology:
+    role = np.ascontiguousarray(role, dtype=np.uint8)
+    d = _Desc()
+    d.fanout[:] = [int(x) for x in fanout]
+    d.role = role.ctypes.data
+    d.tier_bw_Bps[:] = [float(x) for x in tier_bw_Bps]
+    d.tier_lat_s[:] = [float(x) for x in tier_lat_s]
+    d.n_links = int(n_links)
+    h = C.c_void_p()
+    _check("netkv_topology_create", _lib.netkv_topology_create(C.byref(d), C.byref(h)))
+    return Topology(h.value)
+
+
+def netkv_topology_destroy(topo: Topology) -> None:
+    if topo.handle:
+        _check("netkv_topology_destroy", _lib.netkv_topology_destroy(topo.handle))
+        topo.handle = None
+
+
+def netkv_topology_query(topo: Topology):
+    v = [C.c_uint32() for _ in range(4)]
+    _check("netkv_topology_query",
+           _lib.netkv_topology_query(topo.handle, *[C.byref(x) for x in v]))
+    return tuple(int(x.value) for x in v)
+
+
+def netkv_oracle_build(topo: Topology, util, n_snap: int, kv_bytes: float, C_out=None, UB=None,
+                       status=None, stream=None) -> None:
+    _check("netkv_oracle_build", _lib.netkv_oracle_build(
+        topo.handle, _ptr(util), int(n_snap), float(kv_bytes), _ptr(C_out), _ptr(UB),
+        _ptr(status), _stream(stream)))
+
+
+def netkv_cache_build(tables, n_tables: int, log2_capacity: int, keys, key_off, status=None,
+                      stream=None) -> None:
+    _check("netkv_cache_build", _lib.netkv_cache_build(
+        _ptr(tables), int(n_tables), int(log2_capacity), _ptr(keys), _ptr(key_off),
+        _ptr(status), _stream(stream)))
+
+
+def netkv_prefix_match(tables, D: int, log2_capacity: int, n_sets: int, chains, chain_off, R: int,
+                       set_off, M, status=None, stream=None) -> None:
+    _check("netkv_prefix_match", _lib.netkv_prefix_match(
+        _ptr(tables), int(D), int(log2_capacity), int(n_sets), _ptr(chains), _ptr(chain_off),
+        int(R), _ptr(set_off), _ptr(M), _ptr(status), _stream(stream)))
+
+
+def netkv_schedule_streams(topo: Topology, n_streams: int, weights, R: int, length, prefill, snap,
+                           M, UB, n_snap: int, events, event_off, load_init, dec, best, second,
+                           load_final, status=None, stream=None) -> None:
+    _check("netkv_schedule_streams", _lib.netkv_schedule_streams(
+        topo.handle, int(n_streams), _ptr(weights), int(R), _ptr(length), _ptr(prefill),
+        _ptr(snap), _ptr(M), _ptr(UB), int(n_snap), _ptr(events), _ptr(event_off),
+        _ptr(load_init), _ptr(dec), _ptr(best), _ptr(second), _ptr(load_final), _ptr(status),
+        _stream(stream)))
+
+
+def make_weights(w: np.ndarray, theta: float, cap_tokens: int, bytes_per_token: int) -> np.ndarray:
+    """Host array of netkv_weights from an [n_streams, 3] (w_net, w_prefix, w_load) array."""
+    w = np.asarray(w, dtype=np.float32).reshape(-1, 3)
+    out = np.zeros(len(w), WEIGHTS_DTYPE)
+    out["w_net"], out["w_prefix"], out["w_load"] = w[:, 0], w[:, 1], w[:, 2]
+    out["theta_s_per_token"] = np.float32(theta)
+    out["cap_tokens"] = int(cap_tokens)
+    out["bytes_per_token"] = int(bytes_per_token)
+    return out

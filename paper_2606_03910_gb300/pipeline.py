@@ -1,0 +1,142 @@
+"""One step of the NetKV scoring path through the C ABI.
+
+``Scorer`` holds what stays resident between steps (the topology handle and the
+decode caches as hash tables) and runs a step as three library calls on one
+CUDA stream:
+
+1. ``netkv_oracle_build``  -> level bottlenecks UB of every telemetry snapshot
+2. ``netkv_prefix_match``  -> M[r][d] for every request and decode
+3. ``netkv_schedule_streams`` -> decisions, best/second scores, final loads
+
+``step_host`` is the same step from host buffers: it copies the step's inputs
+host->device, runs the step and copies the results back, all on the stream.
+Python here only marshals arguments; PyTorch provides device memory.
+"""
+from __future__ import annotations
+
+import dataclasses
+from typing import Optional
+
+import numpy as np
+import torch
+
+from . import netkv
+
+
+@dataclasses.dataclass
+class StepInputs:
+    util: torch.Tensor        # f32 [n_snap, n_links]
+    chains: torch.Tensor      # i64 (uint64 bits) [total blocks]
+    chain_off: torch.Tensor   # i64 [R+1]
+    set_off: torch.Tensor     # i32 [n_sets+1]
+    length: torch.Tensor      # i32 [R]
+    prefill: torch.Tensor     # i32 [R]
+    snap: torch.Tensor        # i32 [R]
+    events: torch.Tensor      # i32 (uint32 bits) [E]
+    event_off: torch.Tensor   # i64 [n_streams+1]
+    weights: torch.Tensor     # u8 [n_streams * 32] (netkv_weights)
+    load_init: Optional[torch.Tensor] = None
+
+    @property
+    def R(self) -> int:
+        return int(self.length.shape[0])
+
+    @property
+    def n_streams(self) -> int:
+        return int(self.event_off.shape[0] - 1)
+
+    @property
+    def n_snap(self) -> int:
+        return int(self.util.shape[0])
+
+    def nbytes(self) -> int:
+        return sum(int(t.numel() * t.element_size()) for t in dataclasses.astuple(self)
+                   if isinstance(t, torch.Tensor))
+
+
+@dataclasses.dataclass
+class StepOutputs:
+    UB: torch.Tensor          # f32 [n_snap, N, 4]
+    M: torch.Tensor           # i16 (uint16 bits) [R, D]
+    dec: torch.Tensor         # i32 [R]
+    best: torch.Tensor        # f32 [R]
+    second: torch.Tensor      # f32 [R]
+    load_final: torch.Tensor  # i64 [n_streams, D]
+    status: torch.Tensor      # i32 [1]
+
+
+class Scorer:
+    def __init__(self, fanout, role, tier_bw, tier_lat, n_links: int, D_sets: int,
+                 log2_capacity: int, device="cuda"):
+        self.device = torch.device(device)
+        self.topo = netkv.netkv_topology_create(fanout, role, tier_bw, tier_lat, n_links)
+        self.N, self.P, self.D, self.used_links = netkv.netkv_topology_query(self.topo)
+        self.n_links = int(n_links)
+        self.n_sets = int(D_sets)
+        self.log2_capacity = int(log2_capacity)
+        cap = 1 << self.log2_capacity
+        self.tables = torch.empty(self.n_sets * self.D * cap, dtype=torch.int64, device=self.device)
+        self.status = torch.zeros(1, dtype=torch.int32, device=self.device)
+
+    # ---- resident state
+    def load_caches(self, keys: torch.Tensor, key_off: torch.Tensor, set0: int = 0,
+                    n_sets: Optional[int] = None, stream=None) -> None:
+        """Build the tables of table sets [set0, set0 + n_sets) from a key list."""
+        n_sets = self.n_sets - set0 if n_sets is None else n_sets
+        cap = 1 << self.log2_capacity
+        base = self.tables[set0 * self.D * cap:]
+        netkv.netkv_cache_build(base, n_sets * self.D, self.log2_capacity, keys, key_off,
+                                self.status, stream)
+
+    # ---- one step
+    def alloc_outputs(self, n_snap: int, R: int, n_streams: int) -> StepOutputs:
+        dev = self.device
+        return StepOutputs(
+            UB=torch.empty((n_snap, self.N, 4), dtype=torch.float32, device=dev),
+            M=torch.empty((R, self.D), dtype=torch.int16, device=dev),
+            dec=torch.empty(R, dtype=torch.int32, device=dev),
+            best=torch.empty(R, dtype=torch.float32, device=dev),
+            second=torch.empty(R, dtype=torch.float32, device=dev),
+            load_final=torch.empty((n_streams, self.D), dtype=torch.int64, device=dev),
+            status=torch.zeros(1, dtype=torch.int32, device=dev))
+
+    def oracle_build(self, x: StepInputs, out: StepOutputs, stream=None) -> None:
+        netkv.netkv_oracle_build(self.topo, x.util, x.n_snap, 1.0, None, out.UB, out.status, stream)
+
+    def prefix_match(self, x: StepInputs, out: StepOutputs, stream=None) -> None:
+        netkv.netkv_prefix_match(self.tables, self.D, self.log2_capacity, self.n_sets, x.chains,
+                                 x.chain_off, x.R, x.set_off if self.n_sets > 1 else None, out.M,
+                                 out.status, stream)
+
+    def schedule(self, x: StepInputs, out: StepOutputs, stream=None) -> None:
+        netkv.netkv_schedule_streams(self.topo, x.n_streams, x.weights, x.R, x.length, x.prefill,
+                                     x.snap, out.M, out.UB, x.n_snap, x.events, x.event_off,
+                                     x.load_init, out.dec, out.best, out.second, out.load_final,
+                                     out.status, stream)
+
+    def step(self, x: StepInputs, out: StepOutputs, stream=None) -> StepOutputs:
+        self.oracle_build(x, out, stream)
+        self.prefix_match(x, out, stream)
+        self.schedule(x, out, stream)
+        return out
+
+    def step_host(self, xh: StepInputs, xd: StepInputs, out: StepOutputs, res_h: dict,
+                  stream=None) -> StepOutputs:
+        """Host-buffer step: xh holds pinned host tensors, xd same-shaped device tensors,
+        res_h pinned host tensors for dec/best/second/load_final."""
+        s = torch.cuda.current_stream() if stream is None else stream
+        with torch.cuda.stream(s):
+            for f in dataclasses.fields(StepInputs):
+                h = getattr(xh, f.name)
+                if isinstance(h, torch.Tensor):
+                    getattr(xd, f.name).copy_(h, non_blocking=True)
+            self.step(xd, out, s)
+            for k in ("dec", "best", "second", "load_final"):
+                res_h[k].copy_(getattr(out, k), non_blocking=True)
+        return out
+
+
+def weights_tensor(w: np.ndarray, theta: float, cap_tokens: int, bytes_per_token: int,
+                   device="cuda") -> torch.Tensor:
+    host = netkv.make_weights(w, theta, cap_tokens, bytes_per_token)
+    return torch.from_numpy(host.view(np.uint8).copy()).to(device)

@@ -372,6 +372,18 @@ def snapshot_of(arrival_us: np.ndarray) -> np.ndarray:
     return np.where(t >= SNAP_STALE_US, (t - SNAP_STALE_US) // SNAP_PERIOD_US, 0)
 
 
+def draw_rows(seed_per_row: np.ndarray, purpose: int, a: np.ndarray, b=0) -> np.ndarray:
+    """draw(seed_per_row[i], purpose, a[i], b) for every row i (vectorised over seeds)."""
+    seed_per_row = np.asarray(seed_per_row, dtype=np.int64)
+    seeds, inv = np.unique(seed_per_row, return_inverse=True)
+    k = np.array([stream_key(int(x), purpose) for x in seeds], dtype=U64)[inv.reshape(-1)]
+    a = np.asarray(a, dtype=U64)
+    b = np.asarray(b, dtype=U64)
+    with np.errstate(over="ignore"):
+        k2 = _mix(k + (a + U64(1)) * U64(GOLDEN))
+        return _mix(k2 + (b + U64(1)) * U64(GOLDEN))
+
+
 def make_workload(spec: Spec, n_streams: Optional[int] = None,
                   requests_per_stream: Optional[int] = None) -> Workload:
     """Materialise per-request arrays, events and depths; bulk arrays stay lazy."""
@@ -382,40 +394,46 @@ def make_workload(spec: Spec, n_streams: Optional[int] = None,
     ns = spec.n_streams if n_streams is None else n_streams
     rps = spec.requests_per_stream if requests_per_stream is None else requests_per_stream
     seeds = np.arange(spec.seed0, spec.seed0 + ns, dtype=np.int64)
-
-    lens, pref, arr, dep, roots, shared = [], [], [], [], [], []
-    for s in range(ns):
-        sd = int(seeds[s])
-        idx = np.arange(rps, dtype=np.int64)
-        if spec.len_mode == "lognormal":
-            ln = np.rint(lognormal(sd, P_LEN, idx, spec.len_median, spec.len_sigma))
-            ln = np.clip(ln, spec.len_clip[0], spec.len_clip[1]).astype(np.int64)
-        else:
-            ln = np.full(rps, spec.len_fixed, np.int64)
-        out = np.clip(np.rint(lognormal(sd, P_OUT, idx, 256.0, 1.0)), 1, 4096).astype(np.int64)
-        gap = np.rint(-np.log1p(-unit(draw(sd, P_GAP, idx))) / spec.rate_per_s * 1e6).astype(np.int64)
-        t = np.cumsum(gap)
-        p = below(draw(sd, P_PREFILL, idx), P).astype(np.int64)
-        rt = below(draw(sd, P_ROOT, idx), spec.n_roots).astype(np.int64)
-        nb = ln // BLOCK_TOKENS
-        rl = spec.root_len(rt)
-        if spec.share_mode == "frac":
-            f = 0.9 * unit(draw(sd, P_SHARE, idx))
-            sh = np.minimum(np.floor(f * nb).astype(np.int64), rl)
-        else:
-            sh = np.minimum(rl, nb)
-        lens.append(ln); pref.append(p); arr.append(t); dep.append(t + out * TBT_US)
-        roots.append(rt); shared.append(sh)
-
-    cat = (lambda xs, dt: np.concatenate(xs).astype(dt) if xs else np.zeros(0, dt))
-    length = cat(lens, np.uint32)
-    R = int(length.shape[0])
+    R = ns * rps
+    sidx = np.repeat(np.arange(ns, dtype=np.int64), rps)          # stream of each request
+    sd = seeds[sidx]
+    idx = np.tile(np.arange(rps, dtype=np.int64), ns)             # index within the stream
     req_off = np.arange(ns + 1, dtype=np.int64) * rps
-    arrival = cat(arr, np.int64)
-    depart = cat(dep, np.int64)
-    nb = (length.astype(np.int64) // BLOCK_TOKENS).astype(np.uint64)
+
+    def lognorm(purpose, median, sigma):
+        u1 = unit(draw_rows(sd, purpose, idx, 0))
+        u2 = unit(draw_rows(sd, purpose, idx, 1))
+        z = np.sqrt(-2.0 * np.log1p(-u1)) * np.cos(2.0 * np.pi * u2)
+        return median * np.exp(sigma * z)
+
+    if R:
+        if spec.len_mode == "lognormal":
+            ln = np.clip(np.rint(lognorm(P_LEN, spec.len_median, spec.len_sigma)),
+                         spec.len_clip[0], spec.len_clip[1]).astype(np.int64)
+        else:
+            ln = np.full(R, spec.len_fixed, np.int64)
+        out = np.clip(np.rint(lognorm(P_OUT, 256.0, 1.0)), 1, 4096).astype(np.int64)
+        gap = np.rint(-np.log1p(-unit(draw_rows(sd, P_GAP, idx))) / spec.rate_per_s * 1e6).astype(np.int64)
+        csum = np.cumsum(gap)
+        base = np.concatenate([[0], csum[req_off[1:-1] - 1]]) if ns > 1 else np.zeros(1, np.int64)
+        arrival = csum - base[sidx]
+        prefill = below(draw_rows(sd, P_PREFILL, idx), P).astype(np.int64)
+        root = below(draw_rows(sd, P_ROOT, idx), spec.n_roots).astype(np.int64)
+        nb = ln // BLOCK_TOKENS
+        rl = spec.root_len(root)
+        if spec.share_mode == "frac":
+            f = 0.9 * unit(draw_rows(sd, P_SHARE, idx))
+            shared = np.minimum(np.floor(f * nb).astype(np.int64), rl)
+        else:
+            shared = np.minimum(rl, nb)
+        depart = arrival + out * TBT_US
+    else:
+        ln = out = arrival = prefill = root = shared = depart = np.zeros(0, np.int64)
+        nb = np.zeros(0, np.int64)
+
+    length = ln.astype(np.uint32)
     chain_off = np.zeros(R + 1, np.uint64)
-    chain_off[1:] = np.cumsum(nb)
+    chain_off[1:] = np.cumsum(nb.astype(np.uint64))
 
     # telemetry snapshots
     if spec.n_snapshots is not None:
@@ -426,13 +444,12 @@ def make_workload(spec: Spec, n_streams: Optional[int] = None,
     else:
         k = snapshot_of(arrival) if R else np.zeros(0, np.int64)
         if spec.telemetry == "per_stream":
-            counts = [int(k[req_off[s]:req_off[s + 1]].max()) + 1 if rps else 1 for s in range(ns)]
-            base = np.concatenate([[0], np.cumsum(counts)]).astype(np.int64)
-            n_snap = int(base[-1])
-            snap_seed = np.concatenate([np.full(c, seeds[s]) for s, c in enumerate(counts)]).astype(np.int64)
-            snap_local = np.concatenate([np.arange(c) for c in counts]).astype(np.int64)
-            sidx = np.repeat(np.arange(ns), rps)
-            snap = (base[sidx] + k).astype(np.uint32)
+            counts = (np.maximum.reduceat(k, req_off[:-1]) + 1) if R else np.ones(ns, np.int64)
+            sbase = np.concatenate([[0], np.cumsum(counts)]).astype(np.int64)
+            n_snap = int(sbase[-1])
+            snap_seed = np.repeat(seeds, counts).astype(np.int64)
+            snap_local = (np.arange(n_snap, dtype=np.int64) - np.repeat(sbase[:-1], counts))
+            snap = (sbase[sidx] + k).astype(np.uint32)
         else:
             n_snap = int(k.max()) + 1 if R else 1
             snap_seed = np.full(n_snap, spec.seed0, np.int64)
@@ -448,37 +465,34 @@ def make_workload(spec: Spec, n_streams: Optional[int] = None,
         n_sets = 1
         set_off = np.array([0, R], np.uint32)
         set_seed = np.array([spec.seed0], np.int64)
-    depth = np.zeros((n_sets, D, spec.n_roots), np.int64)
-    kk = np.arange(spec.n_roots)
+    kk = np.arange(spec.n_roots, dtype=np.int64)
     rl = spec.root_len(kk)
-    for g in range(n_sets):
-        raw = below(draw(int(set_seed[g]), P_DEPTH, np.arange(D)[:, None], kk[None, :]),
-                    (rl + 1)[None, :].astype(np.uint64)).astype(np.int64)
-        if spec.depth_mode == "scaled":
-            tot = raw.sum(axis=1, keepdims=True)
-            scale = tot > spec.n_keys
-            raw = np.where(scale, (raw * spec.n_keys) // np.maximum(tot, 1), raw)
-        assert (raw.sum(axis=1) <= spec.n_keys).all()
-        depth[g] = raw
+    gg = np.repeat(np.arange(n_sets), D * spec.n_roots)
+    dd = np.tile(np.repeat(np.arange(D), spec.n_roots), n_sets)
+    kx = np.tile(kk, n_sets * D)
+    raw = below(draw_rows(set_seed[gg], P_DEPTH, dd, kx), (rl[kx] + 1).astype(np.uint64))
+    depth = raw.astype(np.int64).reshape(n_sets, D, spec.n_roots)
+    if spec.depth_mode == "scaled":
+        tot = depth.sum(axis=2, keepdims=True)
+        depth = np.where(tot > spec.n_keys, (depth * spec.n_keys) // np.maximum(tot, 1), depth)
+    assert (depth.sum(axis=2) <= spec.n_keys).all()
 
-    # events: sorted by (time, departure before arrival, request index)
-    evs, eoff = [], [0]
-    for s in range(ns):
-        r = np.arange(req_off[s], req_off[s + 1], dtype=np.int64)
-        t = np.concatenate([depart[r], arrival[r]])
-        typ = np.concatenate([np.zeros(len(r), np.int64), np.ones(len(r), np.int64)])
-        rr = np.concatenate([r, r])
-        order = np.lexsort((rr, typ, t))
-        code = rr[order].astype(np.uint64) | ((1 - typ[order]).astype(np.uint64) << U64(31))
-        evs.append(code.astype(np.uint32))
-        eoff.append(eoff[-1] + len(code))
-    events = cat(evs, np.uint32)
-    event_off = np.array(eoff, np.uint64)
+    # events: per stream, sorted by (time, departure before arrival, request index)
+    if R:
+        rr = np.concatenate([np.arange(R), np.arange(R)])
+        t = np.concatenate([depart, arrival])
+        typ = np.concatenate([np.zeros(R, np.int64), np.ones(R, np.int64)])
+        order = np.lexsort((rr, typ, t, sidx[rr]))
+        events = (rr[order].astype(np.uint64) |
+                  ((1 - typ[order]).astype(np.uint64) << U64(31))).astype(np.uint32)
+    else:
+        events = np.zeros(0, np.uint32)
+    event_off = (np.arange(ns + 1, dtype=np.uint64) * np.uint64(2 * rps))
 
     return Workload(spec=spec, role=role, P=P, D=D, L=L, req_off=req_off, stream_seed=seeds,
-                    length=length, prefill=cat(pref, np.uint32), arrival_us=arrival,
-                    depart_us=depart, snap=snap, root=cat(roots, np.uint32),
-                    shared=cat(shared, np.uint32), chain_off=chain_off, n_sets=n_sets,
+                    length=length, prefill=prefill.astype(np.uint32), arrival_us=arrival,
+                    depart_us=depart, snap=snap, root=root.astype(np.uint32),
+                    shared=shared.astype(np.uint32), chain_off=chain_off, n_sets=n_sets,
                     set_off=set_off, set_seed=set_seed, depth=depth, n_snap=n_snap,
                     snap_seed=snap_seed, snap_local=snap_local, events=events,
                     event_off=event_off, weights=stream_weights(spec, ns))

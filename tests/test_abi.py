@@ -1,0 +1,72 @@
+"""The C-ABI library loads and exports every entry point declared in include/netkv.h.
+
+No compute calls: only entry points that fail on host-side validation before
+touching a GPU are called here."""
+import ctypes as C
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "netkv.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2606_03910_gb300 import netkv
+    return netkv
+
+
+def declared():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(netkv_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared()
+    for n in ("netkv_topology_create", "netkv_topology_destroy", "netkv_topology_query",
+              "netkv_oracle_build", "netkv_cache_build", "netkv_prefix_match",
+              "netkv_schedule_streams", "netkv_version"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    so = C.CDLL(lib.LIB_PATH)
+    for name in declared():
+        assert hasattr(so, name), f"{name} not exported"
+    assert set(lib.EXPORTS) <= set(declared())
+
+
+def test_version_and_host_validation(lib):
+    assert lib.netkv_version() >= 1
+    import numpy as np
+    with pytest.raises(lib.NetKVError) as e:
+        lib.netkv_topology_create((2, 0, 2, 2), np.zeros(0, np.uint8), (1, 1, 1, 1), (0, 0, 0, 0), 8)
+    assert e.value.code == lib.NETKV_EINVAL
+    so = lib._lib
+    assert so.netkv_oracle_build(None, None, 1, 1.0, None, None, None, None) == lib.NETKV_EINVAL
+    assert so.netkv_cache_build(None, 1, 4, None, None, None, None) == lib.NETKV_EINVAL
+    assert so.netkv_prefix_match(None, 1, 4, 1, None, None, 1, None, None, None, None) == lib.NETKV_EINVAL
+    assert so.netkv_schedule_streams(None, 1, None, 0, None, None, None, None, None, 0, None, None,
+                                     None, None, None, None, None, None, None) == lib.NETKV_EINVAL
+    assert so.netkv_topology_destroy(None) == lib.NETKV_EINVAL
+
+
+def test_weights_layout(lib):
+    assert lib.WEIGHTS_DTYPE.itemsize == 32
+    assert [lib.WEIGHTS_DTYPE.fields[k][1] for k in lib.WEIGHTS_DTYPE.names] == [0, 4, 8, 12, 16, 24]
+
+
+def test_product_path_does_not_import_the_oracle():
+    """The library package and its binding never reference the oracle."""
+    pkg = os.path.join(ROOT, "paper_2606_03910_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h")):
+                src = open(os.path.join(dirpath, f)).read()
+                assert "import oracle" not in src and "from oracle" not in src, f
+                assert "netkv_oracle.cpp" not in src and "libnetkv_oracle" not in src, f
