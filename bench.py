@@ -55,6 +55,22 @@ def dist_env():
     return rank, world, local
 
 
+def rank_seed0(rank: int, streams: int) -> int:
+    """Weak scaling: rank k runs its own replicas, seeds [k*streams, (k+1)*streams)."""
+    return rank * streams
+
+
+def max_over_ranks(x: float, device=None) -> float:
+    """Maximum of a per-rank value over all ranks (the step time of the slowest rank)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def workload_config(streams, world, extra=None):
     cfg = {"workload": f"{streams} replicas x 64-GPU four-tier tree (8P+8D, TP=4), "
                        "1,000 requests/stream, 2^19-slot caches of 200K blocks",
@@ -195,7 +211,7 @@ def run_netkv(args):
     from paper_2606_03910_gb300.pipeline import Scorer, StepInputs, weights_tensor
 
     spec = synth.config1(args.streams)
-    spec.seed0 = rank * args.streams               # weak scaling: each GPU its own replicas
+    spec.seed0 = rank_seed0(rank, args.streams)
     w = synth.make_workload(spec)
     theta = float(np.float32(synth.THETA_S_PER_TOKEN))
     bpt = synth.BYTES_PER_TOKEN_SHARD
@@ -249,10 +265,7 @@ def run_netkv(args):
     ms = t0.elapsed_time(t1) / args.steps
     per_kernel = {n: sum(ev[k][j][0].elapsed_time(ev[k][j][1]) for k in range(args.steps)) / args.steps
                   for j, n in enumerate(names)}
-    if world > 1:
-        tt = torch.tensor([ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(ms, dev)
     status = int(out.status.item())
     if status != 0:
         raise RuntimeError(f"device status {status} in the timed region")
@@ -309,10 +322,7 @@ def run_netkv(args):
         e1.record(stream)
         torch.cuda.synchronize()
         ems = e0.elapsed_time(e1) / args.steps
-        if world > 1:
-            tt = torch.tensor([ems], device=dev)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            ems = float(tt.item())
+        ems = max_over_ranks(ems, dev)
         e2e = {"value": decisions / (ems / 1e3), "unit": UNIT, "ms_per_step": round(ems, 3),
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
