@@ -271,6 +271,9 @@ def run_netkv(args):
         raise RuntimeError(f"device status {status} in the timed region")
 
     R, D = x.R, sc.D
+    # level bottlenecks 1; prefix match 4 (group insert, group resolve, leaders, members)
+    # with a workspace or 1 without; greedy 1
+    launches_per_step = 1 + (4 if sc.share_prefixes else 1) + 1
     decisions = R * world
     value = decisions / (ms / 1e3)
 
@@ -342,7 +345,7 @@ def run_netkv(args):
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                 "dtype": "f32", "data": "synthetic",
                 "config": workload_config(args.streams, world),
-                "scores_per_s": value * D, "gpu_launches": 3 * args.steps,
+                "scores_per_s": value * D, "gpu_launches": launches_per_step * args.steps,
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk}
         print(json.dumps(line), flush=True)
     if world > 1:

@@ -142,14 +142,23 @@ netkv_status netkv_cache_build(uint64_t* d_tables, uint64_t n_tables, uint32_t l
  *   d_chain_off  [R+1] uint64; every chain has at most 65535 blocks
  *   d_set_off    [n_sets+1] uint32 request offsets: table set g serves requests
  *                [d_set_off[g], d_set_off[g+1]); may be NULL when n_sets == 1
+ *   d_workspace  NULL, or a device buffer of at least
+ *                netkv_prefix_match_workspace_size(R) bytes, 256-byte aligned, owned by
+ *                the caller and overwritten by the call.  With a workspace, requests are
+ *                grouped by (table set, first block hash); each group's longest chain is
+ *                matched in full and the others reuse its answers over their common
+ *                prefix (exactly: the result is identical to the NULL-workspace call).
+ *                Calls that overlap on the GPU need distinct workspaces.
  *   d_M          [R][D] uint16 output
  * A zero hash in a chain sets EDOMAIN and counts as a miss.  A chain longer than 65535
- * blocks sets EDOMAIN and its M saturates at 65535.
+ * blocks sets EDOMAIN and its M saturates at 65535.  R < 2^31.
  */
+size_t netkv_prefix_match_workspace_size(uint32_t R);
 netkv_status netkv_prefix_match(const uint64_t* d_tables, uint32_t D, uint32_t log2_capacity,
                                 uint32_t n_sets, const uint64_t* d_chains,
                                 const uint64_t* d_chain_off, uint32_t R,
-                                const uint32_t* d_set_off, uint16_t* d_M, int* d_status,
+                                const uint32_t* d_set_off, void* d_workspace,
+                                size_t workspace_bytes, uint16_t* d_M, int* d_status,
                                 netkv_stream_t stream);
 
 /* ------------------------------------------------------------------ greedy
@@ -192,7 +201,8 @@ typedef struct {
  *   d_second     [R] fp32 output: minimum over the other feasible candidates (+inf if none)
  *   d_load_final [n_streams][D] int64 output: loads after the last event
  * Every request index must occur in at most one stream, and its departure after its
- * arrival.  Out-of-range indices set ERANGE and the event is skipped.
+ * arrival.  Out-of-range indices set ERANGE and the event is skipped.  The topology
+ * may have at most 4096 decode instances.
  */
 netkv_status netkv_schedule_streams(netkv_topology_t topo, uint32_t n_streams,
                                     const netkv_weights* d_w, uint32_t R, const uint32_t* d_len,

@@ -28,8 +28,8 @@ NETKV_DEV_EDOMAIN, NETKV_DEV_EFULL, NETKV_DEV_ERANGE = 1, 2, 4
 _NAMES = {1: "NETKV_EINVAL", 2: "NETKV_ENOMEM", 3: "NETKV_ECUDA"}
 
 EXPORTS = ("netkv_topology_create", "netkv_topology_destroy", "netkv_topology_query",
-           "netkv_oracle_build", "netkv_cache_build", "netkv_prefix_match",
-           "netkv_schedule_streams", "netkv_version")
+           "netkv_oracle_build", "netkv_cache_build", "netkv_prefix_match_workspace_size",
+           "netkv_prefix_match", "netkv_schedule_streams", "netkv_version")
 
 
 class NetKVError(RuntimeError):
@@ -57,11 +57,14 @@ _lib.netkv_topology_destroy.argtypes = [_P]
 _lib.netkv_topology_query.argtypes = [_P, _P, _P, _P, _P]
 _lib.netkv_oracle_build.argtypes = [_P, _P, _U32, _F64, _P, _P, _P, _P]
 _lib.netkv_cache_build.argtypes = [_P, _U64, _U32, _P, _P, _P, _P]
-_lib.netkv_prefix_match.argtypes = [_P, _U32, _U32, _U32, _P, _P, _U32, _P, _P, _P, _P]
+_lib.netkv_prefix_match_workspace_size.argtypes = [_U32]
+_lib.netkv_prefix_match_workspace_size.restype = C.c_size_t
+_lib.netkv_prefix_match.argtypes = [_P, _U32, _U32, _U32, _P, _P, _U32, _P, _P, C.c_size_t, _P,
+                                    _P, _P]
 _lib.netkv_schedule_streams.argtypes = [_P, _U32, _P, _U32, _P, _P, _P, _P, _P, _U32, _P, _P,
                                         _P, _P, _P, _P, _P, _P, _P]
 for _f in EXPORTS:
-    if _f != "netkv_version":
+    if _f not in ("netkv_version", "netkv_prefix_match_workspace_size"):
         getattr(_lib, _f).restype = C.c_int
 
 
@@ -151,11 +154,16 @@ def netkv_cache_build(tables, n_tables: int, log2_capacity: int, keys, key_off, 
         _ptr(status), _stream(stream)))
 
 
+def netkv_prefix_match_workspace_size(R: int) -> int:
+    return int(_lib.netkv_prefix_match_workspace_size(int(R)))
+
+
 def netkv_prefix_match(tables, D: int, log2_capacity: int, n_sets: int, chains, chain_off, R: int,
-                       set_off, M, status=None, stream=None) -> None:
+                       set_off, M, status=None, stream=None, workspace=None) -> None:
+    ws_bytes = 0 if workspace is None else int(workspace.numel() * workspace.element_size())
     _check("netkv_prefix_match", _lib.netkv_prefix_match(
         _ptr(tables), int(D), int(log2_capacity), int(n_sets), _ptr(chains), _ptr(chain_off),
-        int(R), _ptr(set_off), _ptr(M), _ptr(status), _stream(stream)))
+        int(R), _ptr(set_off), _ptr(workspace), ws_bytes, _ptr(M), _ptr(status), _stream(stream)))
 
 
 def netkv_schedule_streams(topo: Topology, n_streams: int, weights, R: int, length, prefill, snap,

@@ -5,7 +5,8 @@ decode caches as hash tables) and runs a step as three library calls on one
 CUDA stream:
 
 1. ``netkv_oracle_build``  -> level bottlenecks UB of every telemetry snapshot
-2. ``netkv_prefix_match``  -> M[r][d] for every request and decode
+2. ``netkv_prefix_match``  -> M[r][d] for every request and decode (with a
+   workspace, so that requests sharing a prefix share the probing)
 3. ``netkv_schedule_streams`` -> decisions, best/second scores, final loads
 
 ``step_host`` is the same step from host buffers: it copies the step's inputs
@@ -67,7 +68,7 @@ class StepOutputs:
 
 class Scorer:
     def __init__(self, fanout, role, tier_bw, tier_lat, n_links: int, D_sets: int,
-                 log2_capacity: int, device="cuda"):
+                 log2_capacity: int, device="cuda", share_prefixes: bool = True):
         self.device = torch.device(device)
         self.topo = netkv.netkv_topology_create(fanout, role, tier_bw, tier_lat, n_links)
         self.N, self.P, self.D, self.used_links = netkv.netkv_topology_query(self.topo)
@@ -77,6 +78,17 @@ class Scorer:
         cap = 1 << self.log2_capacity
         self.tables = torch.empty(self.n_sets * self.D * cap, dtype=torch.int64, device=self.device)
         self.status = torch.zeros(1, dtype=torch.int32, device=self.device)
+        self.share_prefixes = share_prefixes
+        self.workspace = None
+
+    def _workspace(self, R: int):
+        """Prefix-match workspace for R requests (grown on demand, reused across steps)."""
+        if not self.share_prefixes:
+            return None
+        need = netkv.netkv_prefix_match_workspace_size(R)
+        if self.workspace is None or self.workspace.numel() < need:
+            self.workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=self.device)
+        return self.workspace
 
     # ---- resident state
     def load_caches(self, keys: torch.Tensor, key_off: torch.Tensor, set0: int = 0,
@@ -106,7 +118,7 @@ class Scorer:
     def prefix_match(self, x: StepInputs, out: StepOutputs, stream=None) -> None:
         netkv.netkv_prefix_match(self.tables, self.D, self.log2_capacity, self.n_sets, x.chains,
                                  x.chain_off, x.R, x.set_off if self.n_sets > 1 else None, out.M,
-                                 out.status, stream)
+                                 out.status, stream, workspace=self._workspace(x.R))
 
     def schedule(self, x: StepInputs, out: StepOutputs, stream=None) -> None:
         netkv.netkv_schedule_streams(self.topo, x.n_streams, x.weights, x.R, x.length, x.prefill,

@@ -148,15 +148,26 @@ def _prefix_case(chains_list, caches, D, set_sizes, log2_cap=10):
     tables = torch.empty(n_sets * D << log2_cap, dtype=torch.int64, device="cuda")
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
     dk = torch.from_numpy(keys.view(np.int64)).cuda() if len(keys) else torch.zeros(1, dtype=torch.int64, device="cuda")
+    st_build = torch.zeros(1, dtype=torch.int32, device="cuda")
     netkv.netkv_cache_build(tables, n_sets * D, log2_cap, dk,
-                            torch.from_numpy(key_off.view(np.int64)).cuda(), st)
+                            torch.from_numpy(key_off.view(np.int64)).cuda(), st_build)
     M = torch.full((max(R, 1), D), -1, dtype=torch.int16, device="cuda")
     dch = torch.from_numpy(chains.view(np.int64)).cuda() if len(chains) else torch.zeros(1, dtype=torch.int64, device="cuda")
-    netkv.netkv_prefix_match(tables, D, log2_cap, n_sets, dch,
-                             torch.from_numpy(chain_off.view(np.int64)).cuda(), R,
-                             torch.from_numpy(set_off.view(np.int32)).cuda(), M, st)
+    d_off = torch.from_numpy(chain_off.view(np.int64)).cuda()
+    d_set = torch.from_numpy(set_off.view(np.int32)).cuda()
+    netkv.netkv_prefix_match(tables, D, log2_cap, n_sets, dch, d_off, R, d_set, M, st)
     s = status_of(st)
     Mh = host(M).view(np.uint16)[:R]
+    # the grouped (workspace) form gives the same result and the same status
+    ws = torch.empty(max(netkv.netkv_prefix_match_workspace_size(R), 256), dtype=torch.uint8,
+                     device="cuda")
+    M2 = torch.full((max(R, 1), D), -1, dtype=torch.int16, device="cuda")
+    st2 = torch.zeros(1, dtype=torch.int32, device="cuda")
+    netkv.netkv_prefix_match(tables, D, log2_cap, n_sets, dch, d_off, R, d_set, M2, st2,
+                             workspace=ws)
+    assert status_of(st2) == s
+    np.testing.assert_array_equal(host(M2).view(np.uint16)[:R], Mh)
+    s |= status_of(st_build)
     Mo = oracle.prefix_match(keys, key_off, D, chains, chain_off, set_off) if R else Mh
     return Mh, Mo, s, tables
 
@@ -190,6 +201,69 @@ def test_prefix_match_random_ragged():
     assert s == 0
     np.testing.assert_array_equal(M, Mo)
     assert (Mo > 0).mean() > 0.3
+
+
+def test_prefix_match_shared_prefixes():
+    """Trie-shaped requests: several roots, random-depth root prefixes with random tails,
+    exact duplicates, chains that are prefixes of other chains, the same first block in
+    different table sets, empty chains; caches hold root prefixes with holes."""
+    rng = np.random.default_rng(11)
+    D, set_sizes = 13, [60, 45, 1, 30]
+    roots = [rng.integers(1, 2 ** 63, 700, dtype=np.int64).astype(np.uint64) for _ in range(5)]
+    chains_list = []
+    for g, sz in enumerate(set_sizes):
+        for i in range(sz):
+            kind = rng.integers(0, 6)
+            root = roots[rng.integers(0, 5)]
+            if kind == 0:
+                c = np.zeros(0, np.uint64)
+            elif kind == 1 and chains_list:
+                c = chains_list[int(rng.integers(0, len(chains_list)))].copy()     # duplicate
+            elif kind == 2 and chains_list:
+                c0 = chains_list[int(rng.integers(0, len(chains_list)))]
+                c = c0[:int(rng.integers(0, len(c0) + 1))].copy()                 # a prefix
+            else:
+                k = int(rng.integers(0, 700))
+                tail = rng.integers(1, 2 ** 63, int(rng.integers(0, 80)), dtype=np.int64).astype(np.uint64)
+                c = np.concatenate([root[:k], tail])
+            chains_list.append(c)
+    caches = []
+    for g in range(len(set_sizes)):
+        cg = []
+        for d in range(D):
+            ks = set(int(x) for x in rng.integers(1, 2 ** 63, 30, dtype=np.int64))
+            for root in roots:
+                depth = int(rng.integers(0, 701))
+                keep = root[:depth]
+                if rng.random() < 0.3 and depth > 10:                           # a hole
+                    keep = np.delete(keep, int(rng.integers(0, depth)))
+                ks.update(int(x) for x in keep)
+            cg.append(sorted(ks))
+        caches.append(cg)
+    M, Mo, s, _ = _prefix_case(chains_list, caches, D, set_sizes, log2_cap=13)
+    assert s == 0
+    np.testing.assert_array_equal(M, Mo)
+    assert (Mo > 50).mean() > 0.2
+
+
+def test_prefix_match_workspace_checks():
+    netkv = nk()
+    tables = torch.zeros(4 << 4, dtype=torch.int64, device="cuda")
+    off = torch.tensor([0, 2], dtype=torch.int64, device="cuda")
+    ch = torch.tensor([5, 6], dtype=torch.int64, device="cuda")
+    M = torch.empty((1, 4), dtype=torch.int16, device="cuda")
+    need = netkv.netkv_prefix_match_workspace_size(1)
+    assert need > 0 and netkv.netkv_prefix_match_workspace_size(0) == 0
+    small = torch.empty(need - 1, dtype=torch.uint8, device="cuda")
+    with pytest.raises(netkv.NetKVError):
+        netkv.netkv_prefix_match(tables, 4, 4, 1, ch, off, 1, None, M, None, workspace=small)
+    big = torch.empty(need + 512, dtype=torch.uint8, device="cuda")
+    with pytest.raises(netkv.NetKVError):         # not 256-byte aligned
+        netkv.netkv_prefix_match(tables, 4, 4, 1, ch, off, 1, None, M, None,
+                                 workspace=big[8:])
+    netkv.netkv_prefix_match(tables, 4, 4, 1, ch, off, 1, None, M, None, workspace=big)
+    torch.cuda.synchronize()
+    assert (host(M) == 0).all()
 
 
 def test_prefix_match_holes_and_duplicates():
