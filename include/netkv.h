@@ -47,7 +47,8 @@ typedef enum {
   NETKV_OK = 0,
   NETKV_EINVAL = 1, /* argument out of range, NULL where required, misaligned buffer */
   NETKV_ENOMEM = 2, /* host or device allocation for a topology handle failed */
-  NETKV_ECUDA = 3   /* a CUDA runtime call or kernel launch failed */
+  NETKV_ECUDA = 3,  /* a CUDA runtime call or kernel launch failed */
+  NETKV_ELIMIT = 4  /* request count above the fixed capacity of netkv_prefix_match_static */
 } netkv_status;
 
 /* Bits OR-ed into *d_status by the kernels. */
@@ -160,6 +161,30 @@ netkv_status netkv_prefix_match(const uint64_t* d_tables, uint32_t D, uint32_t l
                                 const uint32_t* d_set_off, void* d_workspace,
                                 size_t workspace_bytes, uint16_t* d_M, int* d_status,
                                 netkv_stream_t stream);
+
+/* Prefix match without allocation.  The paper has no counterpart: this entry point
+ * serves callers that cannot allocate device memory at scoring time, for example a
+ * scheduler plugin that runs inside a serving engine whose memory pool owns the whole
+ * GPU, or code that must not call cudaMalloc on its request path.  It computes exactly
+ * what netkv_prefix_match computes with a workspace, using instead a fixed 24 MiB
+ * device array compiled into the library (every GPU that loads the library keeps it
+ * until the process exits).
+ *   - Arguments are those of netkv_prefix_match without the workspace.
+ *   - R above NETKV_PREFIX_MATCH_STATIC_MAX_R returns NETKV_ELIMIT and enqueues nothing.
+ *   - The first call on a device looks up the array's device address with that device
+ *     current; make that first call before any stream capture.
+ *   - Allocates nothing: no cudaMalloc, no cudaFree, no allocating library routine.
+ *     The array is cleared where it must start at zero on every call.
+ *   - All calls on a device share the one array: calls that overlap on the GPU (on
+ *     different streams, or from several threads) race and must be serialised by the
+ *     caller.
+ */
+#define NETKV_PREFIX_MATCH_STATIC_MAX_R 524288u
+netkv_status netkv_prefix_match_static(const uint64_t* d_tables, uint32_t D,
+                                       uint32_t log2_capacity, uint32_t n_sets,
+                                       const uint64_t* d_chains, const uint64_t* d_chain_off,
+                                       uint32_t R, const uint32_t* d_set_off, uint16_t* d_M,
+                                       int* d_status, netkv_stream_t stream);
 
 /* ------------------------------------------------------------------ greedy
  * Per-stream weights and constants (device memory, one per stream).  Layout is fixed:

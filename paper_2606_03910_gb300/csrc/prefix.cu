@@ -442,3 +442,56 @@ extern "C" netkv_status netkv_prefix_match(const uint64_t* d_tables, uint32_t D,
                                                       d_status);
   return netkv_launch_status();
 }
+
+// ---------------------------------------------------------------------------------
+// netkv_prefix_match_static: the prefix match for callers that cannot allocate device
+// memory (see include/netkv.h).  Its workspace is this fixed device array, shared by
+// every call on a device; the device address is looked up once per device.
+// ---------------------------------------------------------------------------------
+#include <mutex>
+
+namespace {
+
+constexpr size_t kStaticScratchBytes = 24ull << 20;  // 24 MiB per device
+static __device__ __align__(256) unsigned char g_prefix_scratch[kStaticScratchBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mutex;
+void* g_scratch_addr[kMaxDevices] = {};
+
+// Device address of g_prefix_scratch on the current device (looked up on first use).
+netkv_status static_scratch(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return NETKV_ECUDA;
+  std::lock_guard<std::mutex> lock(g_scratch_mutex);
+  if (!g_scratch_addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_prefix_scratch) != cudaSuccess || !p) {
+      cudaGetLastError();
+      return NETKV_ECUDA;
+    }
+    g_scratch_addr[dev] = p;
+  }
+  *out = g_scratch_addr[dev];
+  return NETKV_OK;
+}
+
+}  // namespace
+
+static_assert(NETKV_PREFIX_MATCH_STATIC_MAX_R > 0, "limit must be positive");
+
+extern "C" netkv_status netkv_prefix_match_static(const uint64_t* d_tables, uint32_t D,
+                                                  uint32_t log2_capacity, uint32_t n_sets,
+                                                  const uint64_t* d_chains,
+                                                  const uint64_t* d_chain_off, uint32_t R,
+                                                  const uint32_t* d_set_off, uint16_t* d_M,
+                                                  int* d_status, netkv_stream_t stream) {
+  if (R > NETKV_PREFIX_MATCH_STATIC_MAX_R ||
+      netkv_prefix_match_workspace_size(R) > kStaticScratchBytes)
+    return NETKV_ELIMIT;
+  void* scratch = nullptr;
+  const netkv_status st = static_scratch(&scratch);
+  if (st != NETKV_OK) return st;
+  return netkv_prefix_match(d_tables, D, log2_capacity, n_sets, d_chains, d_chain_off, R,
+                            d_set_off, scratch, kStaticScratchBytes, d_M, d_status, stream);
+}

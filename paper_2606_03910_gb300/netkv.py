@@ -23,13 +23,16 @@ if not os.path.exists(LIB_PATH):
                       "(python -c 'import __graft_entry__ as g; g.build()')")
 _lib = C.CDLL(LIB_PATH)
 
-NETKV_OK, NETKV_EINVAL, NETKV_ENOMEM, NETKV_ECUDA = 0, 1, 2, 3
+NETKV_OK, NETKV_EINVAL, NETKV_ENOMEM, NETKV_ECUDA, NETKV_ELIMIT = 0, 1, 2, 3, 4
+NETKV_PREFIX_MATCH_STATIC_MAX_R = 524288
 NETKV_DEV_EDOMAIN, NETKV_DEV_EFULL, NETKV_DEV_ERANGE = 1, 2, 4
-_NAMES = {1: "NETKV_EINVAL", 2: "NETKV_ENOMEM", 3: "NETKV_ECUDA"}
+_NAMES = {1: "NETKV_EINVAL", 2: "NETKV_ENOMEM", 3: "NETKV_ECUDA",
+          4: "NETKV_ELIMIT (more requests than the fixed scratch of netkv_prefix_match_static holds)"}
 
 EXPORTS = ("netkv_topology_create", "netkv_topology_destroy", "netkv_topology_query",
            "netkv_oracle_build", "netkv_cache_build", "netkv_prefix_match_workspace_size",
-           "netkv_prefix_match", "netkv_schedule_streams", "netkv_version")
+           "netkv_prefix_match", "netkv_prefix_match_static", "netkv_schedule_streams",
+           "netkv_version")
 
 
 class NetKVError(RuntimeError):
@@ -61,6 +64,7 @@ _lib.netkv_prefix_match_workspace_size.argtypes = [_U32]
 _lib.netkv_prefix_match_workspace_size.restype = C.c_size_t
 _lib.netkv_prefix_match.argtypes = [_P, _U32, _U32, _U32, _P, _P, _U32, _P, _P, C.c_size_t, _P,
                                     _P, _P]
+_lib.netkv_prefix_match_static.argtypes = [_P, _U32, _U32, _U32, _P, _P, _U32, _P, _P, _P, _P]
 _lib.netkv_schedule_streams.argtypes = [_P, _U32, _P, _U32, _P, _P, _P, _P, _P, _U32, _P, _P,
                                         _P, _P, _P, _P, _P, _P, _P]
 for _f in EXPORTS:
@@ -164,6 +168,15 @@ def netkv_prefix_match(tables, D: int, log2_capacity: int, n_sets: int, chains, 
     _check("netkv_prefix_match", _lib.netkv_prefix_match(
         _ptr(tables), int(D), int(log2_capacity), int(n_sets), _ptr(chains), _ptr(chain_off),
         int(R), _ptr(set_off), _ptr(workspace), ws_bytes, _ptr(M), _ptr(status), _stream(stream)))
+
+
+def netkv_prefix_match_static(tables, D: int, log2_capacity: int, n_sets: int, chains, chain_off,
+                              R: int, set_off, M, status=None, stream=None) -> None:
+    """Prefix match that allocates nothing (fixed device scratch inside the library);
+    for callers that may not allocate device memory.  Overlapping calls race."""
+    _check("netkv_prefix_match_static", _lib.netkv_prefix_match_static(
+        _ptr(tables), int(D), int(log2_capacity), int(n_sets), _ptr(chains), _ptr(chain_off),
+        int(R), _ptr(set_off), _ptr(M), _ptr(status), _stream(stream)))
 
 
 def netkv_schedule_streams(topo: Topology, n_streams: int, weights, R: int, length, prefill, snap,
