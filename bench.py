@@ -3,7 +3,8 @@
 
 Workload: 4,096 independent replicas of the single-stream 64-GPU cluster
 (8 prefill + 8 decode instances at TP=4, 1,000 requests each, decode caches of
-200K block hashes in 2^19-slot tables), run as 4,096 concurrent streams whose
+200K block hashes, indexed per replica as block hash -> decode mask), run as 4,096
+concurrent streams whose
 score weights cover a 16x16x16 grid.  One step is the whole hot path over all
 streams: level bottlenecks of every telemetry snapshot (netkv_oracle_build),
 prefix hits of every (request, decode) pair (netkv_prefix_match) and the greedy
@@ -73,10 +74,10 @@ def max_over_ranks(x: float, device=None) -> float:
 
 def workload_config(streams, world, extra=None):
     cfg = {"workload": f"{streams} replicas x 64-GPU four-tier tree (8P+8D, TP=4), "
-                       "1,000 requests/stream, 2^19-slot caches of 200K blocks",
+                       "1,000 requests/stream, decode caches of 200K blocks",
            "streams_per_gpu": streams, "requests_per_stream": 1000, "decodes": 8,
            "prefills": 8, "parallelism": f"replicas{world}",
-           "l2": "inputs larger than L2 (tables 128 GiB + chains 27 GB per GPU)"}
+           "l2": "inputs larger than L2 (cache index 64 GiB + chains 27 GB per GPU)"}
     if extra:
         cfg.update(extra)
     return cfg
@@ -217,7 +218,9 @@ def run_netkv(args):
     bpt = synth.BYTES_PER_TOKEN_SHARD
 
     # resident caches, built in batches of table sets
-    sc = Scorer(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, w.L, w.n_sets, spec.log2_cap,
+    from paper_2606_03910_gb300 import netkv
+    log2_index = netkv.index_log2_capacity(synth.distinct_keys_per_group(w))
+    sc = Scorer(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, w.L, w.n_sets, log2_index,
                 device=dev)
     for g0 in range(0, w.n_sets, args.table_batch):
         g1 = min(w.n_sets, g0 + args.table_batch)

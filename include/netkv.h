@@ -118,27 +118,36 @@ netkv_status netkv_oracle_build(netkv_topology_t topo, const float* d_util, uint
                                 netkv_stream_t stream);
 
 /* ------------------------------------------------------------------ caches
- * Decode caches K_d (Sec. III-C) as open-addressing tables of uint64 block hashes:
- * n_tables tables of 2^log2_capacity slots each, contiguous, value 0 = empty slot
- * (hash 0 is reserved).  Linear probing from a multiplicative hash of the key.
+ * Decode caches K_d (Sec. III-C), the sets of block hashes each decode instance holds,
+ * stored as an inverted index.  Decodes are taken in groups of 64 (decode ranks
+ * 64q .. 64q+63 form group q); each (table set, group) has one open-addressing table
+ * of 2^log2_capacity slots of 16 bytes, {uint64 block hash, uint64 mask}, where bit
+ * (d mod 64) of the mask says that decode d caches the hash.  Hash 0 marks an empty slot
+ * (block hash 0 is reserved).  Linear probing from a multiplicative hash of the key.
+ * The index of table set g, group q starts at slot ((g * G + q) << log2_capacity),
+ * G = ceil(D / 64).  One table must hold the distinct hashes of its group's decodes:
+ * keep its load factor below about 0.5.
  *
- *   d_tables   [n_tables][2^log2_capacity] uint64, cleared then filled by this call
- *   d_keys     keys of table t are d_keys[d_key_off[t] .. d_key_off[t+1])
- *   d_key_off  [n_tables+1] uint64, non-decreasing
- * Duplicate keys are stored once.  A zero key sets EDOMAIN and is skipped; a table
- * with more distinct keys than slots sets EFULL (the excess keys are dropped).
+ *   d_index    device buffer of netkv_cache_index_bytes(n_sets, D, log2_capacity) bytes,
+ *              16-byte aligned; cleared, then filled by netkv_cache_build
+ *   d_keys     keys of (set g, decode d), list t = g * D + d, are
+ *              d_keys[d_key_off[t] .. d_key_off[t+1])
+ *   d_key_off  [n_sets * D + 1] uint64, non-decreasing
+ * Duplicate keys are stored once.  A zero key sets EDOMAIN and is skipped; a table with
+ * more distinct keys than slots sets EFULL (the excess keys are dropped).
  * 1 <= log2_capacity <= 32.
  */
-netkv_status netkv_cache_build(uint64_t* d_tables, uint64_t n_tables, uint32_t log2_capacity,
-                               const uint64_t* d_keys, const uint64_t* d_key_off,
-                               int* d_status, netkv_stream_t stream);
+size_t netkv_cache_index_bytes(uint32_t n_sets, uint32_t D, uint32_t log2_capacity);
+netkv_status netkv_cache_build(void* d_index, uint32_t n_sets, uint32_t D,
+                               uint32_t log2_capacity, const uint64_t* d_keys,
+                               const uint64_t* d_key_off, int* d_status, netkv_stream_t stream);
 
 /* ------------------------------------------------------------------ prefix match
  * Block-level prefix hit (Sec. III-B): M[r][d] = number of leading blocks of request
  * r's block-hash chain that are all present in decode d's cache; the cache hit in
  * tokens is lambda = 16 * M (B_tok = 16).  The scan stops at the first missing block.
  *
- *   d_tables     [n_sets][D][2^log2_capacity] tables built by netkv_cache_build
+ *   d_index      cache index built by netkv_cache_build (same n_sets, D, log2_capacity)
  *   d_chains     uint64 block hashes; chain r = d_chains[d_chain_off[r] .. d_chain_off[r+1])
  *   d_chain_off  [R+1] uint64; every chain has at most 65535 blocks
  *   d_set_off    [n_sets+1] uint32 request offsets: table set g serves requests
@@ -155,7 +164,7 @@ netkv_status netkv_cache_build(uint64_t* d_tables, uint64_t n_tables, uint32_t l
  * blocks sets EDOMAIN and its M saturates at 65535.  R < 2^31.
  */
 size_t netkv_prefix_match_workspace_size(uint32_t R);
-netkv_status netkv_prefix_match(const uint64_t* d_tables, uint32_t D, uint32_t log2_capacity,
+netkv_status netkv_prefix_match(const void* d_index, uint32_t D, uint32_t log2_capacity,
                                 uint32_t n_sets, const uint64_t* d_chains,
                                 const uint64_t* d_chain_off, uint32_t R,
                                 const uint32_t* d_set_off, void* d_workspace,
@@ -180,7 +189,7 @@ netkv_status netkv_prefix_match(const uint64_t* d_tables, uint32_t D, uint32_t l
  *     caller.
  */
 #define NETKV_PREFIX_MATCH_STATIC_MAX_R 524288u
-netkv_status netkv_prefix_match_static(const uint64_t* d_tables, uint32_t D,
+netkv_status netkv_prefix_match_static(const void* d_index, uint32_t D,
                                        uint32_t log2_capacity, uint32_t n_sets,
                                        const uint64_t* d_chains, const uint64_t* d_chain_off,
                                        uint32_t R, const uint32_t* d_set_off, uint16_t* d_M,

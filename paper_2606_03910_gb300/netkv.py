@@ -30,7 +30,8 @@ _NAMES = {1: "NETKV_EINVAL", 2: "NETKV_ENOMEM", 3: "NETKV_ECUDA",
           4: "NETKV_ELIMIT (more requests than the fixed scratch of netkv_prefix_match_static holds)"}
 
 EXPORTS = ("netkv_topology_create", "netkv_topology_destroy", "netkv_topology_query",
-           "netkv_oracle_build", "netkv_cache_build", "netkv_prefix_match_workspace_size",
+           "netkv_oracle_build", "netkv_cache_index_bytes", "netkv_cache_build",
+           "netkv_prefix_match_workspace_size",
            "netkv_prefix_match", "netkv_prefix_match_static", "netkv_schedule_streams",
            "netkv_version")
 
@@ -59,7 +60,9 @@ _lib.netkv_topology_create.argtypes = [C.POINTER(_Desc), C.POINTER(C.c_void_p)]
 _lib.netkv_topology_destroy.argtypes = [_P]
 _lib.netkv_topology_query.argtypes = [_P, _P, _P, _P, _P]
 _lib.netkv_oracle_build.argtypes = [_P, _P, _U32, _F64, _P, _P, _P, _P]
-_lib.netkv_cache_build.argtypes = [_P, _U64, _U32, _P, _P, _P, _P]
+_lib.netkv_cache_index_bytes.argtypes = [_U32, _U32, _U32]
+_lib.netkv_cache_index_bytes.restype = C.c_size_t
+_lib.netkv_cache_build.argtypes = [_P, _U32, _U32, _U32, _P, _P, _P, _P]
 _lib.netkv_prefix_match_workspace_size.argtypes = [_U32]
 _lib.netkv_prefix_match_workspace_size.restype = C.c_size_t
 _lib.netkv_prefix_match.argtypes = [_P, _U32, _U32, _U32, _P, _P, _U32, _P, _P, C.c_size_t, _P,
@@ -68,7 +71,7 @@ _lib.netkv_prefix_match_static.argtypes = [_P, _U32, _U32, _U32, _P, _P, _U32, _
 _lib.netkv_schedule_streams.argtypes = [_P, _U32, _P, _U32, _P, _P, _P, _P, _P, _U32, _P, _P,
                                         _P, _P, _P, _P, _P, _P, _P]
 for _f in EXPORTS:
-    if _f not in ("netkv_version", "netkv_prefix_match_workspace_size"):
+    if _f not in ("netkv_version", "netkv_prefix_match_workspace_size", "netkv_cache_index_bytes"):
         getattr(_lib, _f).restype = C.c_int
 
 
@@ -151,10 +154,14 @@ def netkv_oracle_build(topo: Topology, util, n_snap: int, kv_bytes: float, C_out
         _ptr(status), _stream(stream)))
 
 
-def netkv_cache_build(tables, n_tables: int, log2_capacity: int, keys, key_off, status=None,
+def netkv_cache_index_bytes(n_sets: int, D: int, log2_capacity: int) -> int:
+    return int(_lib.netkv_cache_index_bytes(int(n_sets), int(D), int(log2_capacity)))
+
+
+def netkv_cache_build(index, n_sets: int, D: int, log2_capacity: int, keys, key_off, status=None,
                       stream=None) -> None:
     _check("netkv_cache_build", _lib.netkv_cache_build(
-        _ptr(tables), int(n_tables), int(log2_capacity), _ptr(keys), _ptr(key_off),
+        _ptr(index), int(n_sets), int(D), int(log2_capacity), _ptr(keys), _ptr(key_off),
         _ptr(status), _stream(stream)))
 
 
@@ -162,20 +169,20 @@ def netkv_prefix_match_workspace_size(R: int) -> int:
     return int(_lib.netkv_prefix_match_workspace_size(int(R)))
 
 
-def netkv_prefix_match(tables, D: int, log2_capacity: int, n_sets: int, chains, chain_off, R: int,
+def netkv_prefix_match(index, D: int, log2_capacity: int, n_sets: int, chains, chain_off, R: int,
                        set_off, M, status=None, stream=None, workspace=None) -> None:
     ws_bytes = 0 if workspace is None else int(workspace.numel() * workspace.element_size())
     _check("netkv_prefix_match", _lib.netkv_prefix_match(
-        _ptr(tables), int(D), int(log2_capacity), int(n_sets), _ptr(chains), _ptr(chain_off),
+        _ptr(index), int(D), int(log2_capacity), int(n_sets), _ptr(chains), _ptr(chain_off),
         int(R), _ptr(set_off), _ptr(workspace), ws_bytes, _ptr(M), _ptr(status), _stream(stream)))
 
 
-def netkv_prefix_match_static(tables, D: int, log2_capacity: int, n_sets: int, chains, chain_off,
+def netkv_prefix_match_static(index, D: int, log2_capacity: int, n_sets: int, chains, chain_off,
                               R: int, set_off, M, status=None, stream=None) -> None:
     """Prefix match that allocates nothing (fixed device scratch inside the library);
     for callers that may not allocate device memory.  Overlapping calls race."""
     _check("netkv_prefix_match_static", _lib.netkv_prefix_match_static(
-        _ptr(tables), int(D), int(log2_capacity), int(n_sets), _ptr(chains), _ptr(chain_off),
+        _ptr(index), int(D), int(log2_capacity), int(n_sets), _ptr(chains), _ptr(chain_off),
         int(R), _ptr(set_off), _ptr(M), _ptr(status), _stream(stream)))
 
 
@@ -198,3 +205,11 @@ def make_weights(w: np.ndarray, theta: float, cap_tokens: int, bytes_per_token: 
     out["cap_tokens"] = int(cap_tokens)
     out["bytes_per_token"] = int(bytes_per_token)
     return out
+
+
+def index_log2_capacity(max_distinct_keys: int) -> int:
+    """Smallest table size keeping a cache-index table at load factor <= 0.5."""
+    l = 1
+    while (1 << l) < 2 * max(int(max_distinct_keys), 1):
+        l += 1
+    return l

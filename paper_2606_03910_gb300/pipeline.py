@@ -1,7 +1,7 @@
 """One step of the NetKV scoring path through the C ABI.
 
 ``Scorer`` holds what stays resident between steps (the topology handle and the
-decode caches as hash tables) and runs a step as three library calls on one
+decode caches as an inverted hash index) and runs a step as three library calls on one
 CUDA stream:
 
 1. ``netkv_oracle_build``  -> level bottlenecks UB of every telemetry snapshot
@@ -67,16 +67,18 @@ class StepOutputs:
 
 
 class Scorer:
-    def __init__(self, fanout, role, tier_bw, tier_lat, n_links: int, D_sets: int,
+    def __init__(self, fanout, role, tier_bw, tier_lat, n_links: int, n_sets: int,
                  log2_capacity: int, device="cuda", share_prefixes: bool = True):
+        """log2_capacity: slots per cache-index table (one table per table set and group
+        of 64 decodes); see netkv.index_log2_capacity."""
         self.device = torch.device(device)
         self.topo = netkv.netkv_topology_create(fanout, role, tier_bw, tier_lat, n_links)
         self.N, self.P, self.D, self.used_links = netkv.netkv_topology_query(self.topo)
         self.n_links = int(n_links)
-        self.n_sets = int(D_sets)
+        self.n_sets = int(n_sets)
         self.log2_capacity = int(log2_capacity)
-        cap = 1 << self.log2_capacity
-        self.tables = torch.empty(self.n_sets * self.D * cap, dtype=torch.int64, device=self.device)
+        nbytes = netkv.netkv_cache_index_bytes(self.n_sets, self.D, self.log2_capacity)
+        self.index = torch.empty(nbytes // 8, dtype=torch.int64, device=self.device)
         self.status = torch.zeros(1, dtype=torch.int32, device=self.device)
         self.share_prefixes = share_prefixes
         self.workspace = None
@@ -95,10 +97,9 @@ class Scorer:
                     n_sets: Optional[int] = None, stream=None) -> None:
         """Build the tables of table sets [set0, set0 + n_sets) from a key list."""
         n_sets = self.n_sets - set0 if n_sets is None else n_sets
-        cap = 1 << self.log2_capacity
-        base = self.tables[set0 * self.D * cap:]
-        netkv.netkv_cache_build(base, n_sets * self.D, self.log2_capacity, keys, key_off,
-                                self.status, stream)
+        off = netkv.netkv_cache_index_bytes(set0, self.D, self.log2_capacity) // 8
+        netkv.netkv_cache_build(self.index[off:], n_sets, self.D, self.log2_capacity, keys,
+                                key_off, self.status, stream)
 
     # ---- one step
     def alloc_outputs(self, n_snap: int, R: int, n_streams: int) -> StepOutputs:
@@ -116,7 +117,7 @@ class Scorer:
         netkv.netkv_oracle_build(self.topo, x.util, x.n_snap, 1.0, None, out.UB, out.status, stream)
 
     def prefix_match(self, x: StepInputs, out: StepOutputs, stream=None) -> None:
-        netkv.netkv_prefix_match(self.tables, self.D, self.log2_capacity, self.n_sets, x.chains,
+        netkv.netkv_prefix_match(self.index, self.D, self.log2_capacity, self.n_sets, x.chains,
                                  x.chain_off, x.R, x.set_off if self.n_sets > 1 else None, out.M,
                                  out.status, stream, workspace=self._workspace(x.R))
 

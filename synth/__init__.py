@@ -288,6 +288,17 @@ class Workload:
         return utilisation(self, np.arange(s0, s1))
 
 
+def distinct_keys_per_group(w: Workload, group: int = 64) -> int:
+    """Largest number of distinct cached hashes over (table set, group of `group`
+    decodes): the union of the root prefixes plus every decode's filler keys."""
+    best = 0
+    for g in range(w.n_sets):
+        for q0 in range(0, w.D, group):
+            dd = w.depth[g, q0:q0 + group]
+            best = max(best, int(dd.max(axis=0).sum() + (w.spec.n_keys - dd.sum(axis=1)).sum()))
+    return best
+
+
 def request_set(w: Workload) -> np.ndarray:
     out = np.zeros(w.R, np.int64)
     for g in range(w.n_sets):

@@ -20,11 +20,16 @@ def rel_close(a, b, rel=REL):
     return ok
 
 
+def index_log2(w):
+    from paper_2606_03910_gb300 import netkv
+    return netkv.index_log2_capacity(synth.distinct_keys_per_group(w))
+
+
 def make_scorer(w, device="cuda"):
     from paper_2606_03910_gb300.pipeline import Scorer
     spec = w.spec
     return Scorer(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, w.L, w.n_sets,
-                  spec.log2_cap, device=device)
+                  index_log2(w), device=device)
 
 
 def run_gpu(w, sc=None, cap=None, load_init=None):

@@ -134,9 +134,14 @@ def test_oracle_build_edge_cases():
 
 
 # ============================================================== prefix match
-def _prefix_case(chains_list, caches, D, set_sizes, log2_cap=10):
-    """caches[g][d] = list of keys; chains_list[r]; set_sizes = requests per set."""
+def _prefix_case(chains_list, caches, D, set_sizes, log2_cap=None):
+    """caches[g][d] = list of keys; chains_list[r]; set_sizes = requests per set.
+    log2_cap None: sized for load factor <= 0.5 per (set, group of 64 decodes)."""
     netkv = nk()
+    if log2_cap is None:
+        most = max(len(set().union(*[set(int(k) for k in caches[g][d]) for d in range(q, min(q + 64, D))]))
+                   for g in range(len(set_sizes)) for q in range(0, D, 64))
+        log2_cap = netkv.index_log2_capacity(most)
     n_sets = len(set_sizes)
     chains = np.concatenate([np.asarray(c, np.uint64) for c in chains_list]) if chains_list else np.zeros(0, np.uint64)
     chain_off = np.concatenate([[0], np.cumsum([len(c) for c in chains_list])]).astype(np.uint64)
@@ -145,11 +150,12 @@ def _prefix_case(chains_list, caches, D, set_sizes, log2_cap=10):
     keys = np.concatenate(keys_l) if keys_l else np.zeros(0, np.uint64)
     key_off = np.concatenate([[0], np.cumsum([len(k) for k in keys_l])]).astype(np.uint64)
     R = len(chains_list)
-    tables = torch.empty(n_sets * D << log2_cap, dtype=torch.int64, device="cuda")
+    tables = torch.empty(netkv.netkv_cache_index_bytes(n_sets, D, log2_cap) // 8,
+                         dtype=torch.int64, device="cuda")
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
     dk = torch.from_numpy(keys.view(np.int64)).cuda() if len(keys) else torch.zeros(1, dtype=torch.int64, device="cuda")
     st_build = torch.zeros(1, dtype=torch.int32, device="cuda")
-    netkv.netkv_cache_build(tables, n_sets * D, log2_cap, dk,
+    netkv.netkv_cache_build(tables, n_sets, D, log2_cap, dk,
                             torch.from_numpy(key_off.view(np.int64)).cuda(), st_build)
     M = torch.full((max(R, 1), D), -1, dtype=torch.int16, device="cuda")
     dch = torch.from_numpy(chains.view(np.int64)).cuda() if len(chains) else torch.zeros(1, dtype=torch.int64, device="cuda")
@@ -197,7 +203,7 @@ def test_prefix_match_random_ragged():
             cg.append(sorted(ks))
         caches.append(cg)
         r += sz
-    M, Mo, s, _ = _prefix_case(chains_list, caches, D, set_sizes, log2_cap=14)
+    M, Mo, s, _ = _prefix_case(chains_list, caches, D, set_sizes)
     assert s == 0
     np.testing.assert_array_equal(M, Mo)
     assert (Mo > 0).mean() > 0.3
@@ -240,7 +246,7 @@ def test_prefix_match_shared_prefixes():
                 ks.update(int(x) for x in keep)
             cg.append(sorted(ks))
         caches.append(cg)
-    M, Mo, s, _ = _prefix_case(chains_list, caches, D, set_sizes, log2_cap=13)
+    M, Mo, s, _ = _prefix_case(chains_list, caches, D, set_sizes)
     assert s == 0
     np.testing.assert_array_equal(M, Mo)
     assert (Mo > 50).mean() > 0.2
@@ -248,7 +254,8 @@ def test_prefix_match_shared_prefixes():
 
 def test_prefix_match_workspace_checks():
     netkv = nk()
-    tables = torch.zeros(4 << 4, dtype=torch.int64, device="cuda")
+    tables = torch.zeros(netkv.netkv_cache_index_bytes(1, 4, 4) // 8, dtype=torch.int64,
+                         device="cuda")
     off = torch.tensor([0, 2], dtype=torch.int64, device="cuda")
     ch = torch.tensor([5, 6], dtype=torch.int64, device="cuda")
     M = torch.empty((1, 4), dtype=torch.int16, device="cuda")
@@ -300,10 +307,11 @@ def test_prefix_match_long_chain_saturates():
 
 def test_prefix_match_empty_inputs():
     netkv = nk()
-    tables = torch.empty(4 << 4, dtype=torch.int64, device="cuda")
+    tables = torch.empty(netkv.netkv_cache_index_bytes(1, 4, 4) // 8, dtype=torch.int64,
+                         device="cuda")
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
     off = torch.zeros(5, dtype=torch.int64, device="cuda")
-    netkv.netkv_cache_build(tables, 4, 4, None, off, st)       # clear only
+    netkv.netkv_cache_build(tables, 1, 4, 4, None, off, st)    # clear only
     assert (host(tables) == 0).all()
     M = torch.empty((1, 4), dtype=torch.int16, device="cuda")
     netkv.netkv_prefix_match(tables, 4, 4, 1, None, off, 0, None, M, st)   # R = 0

@@ -30,29 +30,30 @@ def _cuda():
 
 def _inputs(w):
     from paper_2606_03910_gb300 import netkv
-    cap = w.spec.log2_cap
-    tables = torch.empty(w.n_sets * w.D << cap, dtype=torch.int64, device="cuda")
+    cap = netkv.index_log2_capacity(synth.distinct_keys_per_group(w))
+    index = torch.empty(netkv.netkv_cache_index_bytes(w.n_sets, w.D, cap) // 8, dtype=torch.int64,
+                        device="cuda")
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
-    netkv.netkv_cache_build(tables, w.n_sets * w.D, cap, stage.keys(w, 0, w.n_sets),
+    netkv.netkv_cache_build(index, w.n_sets, w.D, cap, stage.keys(w, 0, w.n_sets),
                             stage.key_offsets(w, w.n_sets * w.D), st)
     ra = stage.request_arrays(w)
     torch.cuda.synchronize()
     assert int(st.item()) == 0
-    return tables, stage.chains(w), ra["chain_off"], ra["set_off"]
+    return index, cap, stage.chains(w), ra["chain_off"], ra["set_off"]
 
 
 def _compare(w):
     from paper_2606_03910_gb300 import netkv
-    tables, chains, chain_off, set_off = _inputs(w)
+    tables, cap, chains, chain_off, set_off = _inputs(w)
     so = set_off if w.n_sets > 1 else None
     ref = torch.full((w.R, w.D), -1, dtype=torch.int16, device="cuda")
     st_ref = torch.zeros(1, dtype=torch.int32, device="cuda")
     ws = torch.empty(netkv.netkv_prefix_match_workspace_size(w.R), dtype=torch.uint8, device="cuda")
-    netkv.netkv_prefix_match(tables, w.D, w.spec.log2_cap, w.n_sets, chains, chain_off, w.R, so,
+    netkv.netkv_prefix_match(tables, w.D, cap, w.n_sets, chains, chain_off, w.R, so,
                              ref, st_ref, workspace=ws)
     got = torch.full((w.R, w.D), -1, dtype=torch.int16, device="cuda")
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
-    netkv.netkv_prefix_match_static(tables, w.D, w.spec.log2_cap, w.n_sets, chains, chain_off,
+    netkv.netkv_prefix_match_static(tables, w.D, cap, w.n_sets, chains, chain_off,
                                     w.R, so, got, st)
     torch.cuda.synchronize()
     assert int(st.item()) == int(st_ref.item()) == 0
