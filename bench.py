@@ -17,6 +17,7 @@ bounded sample of the same workload.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import os
 import statistics
@@ -46,6 +47,8 @@ def parse():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--table-batch", type=int, default=256)
+    ap.add_argument("--no-share", action="store_true",
+                    help="prefix match without the workspace (no grouping of shared prefixes)")
     return ap.parse_args()
 
 
@@ -195,12 +198,46 @@ def run_reference(args):
     return 0
 
 
-# ------------------------------------------------------------------ GPU arm
-def run_netkv(args):
+def setup_replicas(streams: int, rank: int, dev, table_batch: int = 256):
+    """The benchmark workload on `dev`: generated inputs, the resident cache index and
+    the step's device buffers.  Returns (workload, scorer, step inputs, step outputs)."""
     import torch
     import synth
     import synth.device as sdev
     from synth import stage
+    from paper_2606_03910_gb300 import netkv
+    from paper_2606_03910_gb300.pipeline import Scorer, StepInputs, weights_tensor
+    spec = synth.config1(streams)
+    spec.seed0 = rank_seed0(rank, streams)
+    w = synth.make_workload(spec)
+    theta = float(np.float32(synth.THETA_S_PER_TOKEN))
+    bpt = synth.BYTES_PER_TOKEN_SHARD
+    log2_index = netkv.index_log2_capacity(synth.distinct_keys_per_group(w))
+    sc = Scorer(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, w.L, w.n_sets, log2_index,
+                device=dev)
+    for g0 in range(0, w.n_sets, table_batch):
+        g1 = min(w.n_sets, g0 + table_batch)
+        keys = sdev.keys(w, g0, g1, device=dev)
+        sc.load_caches(keys, stage.key_offsets(w, (g1 - g0) * w.D, device=dev), set0=g0,
+                       n_sets=g1 - g0)
+        del keys
+    torch.cuda.synchronize()
+    if int(sc.status.item()) != 0:
+        raise RuntimeError(f"cache build status {int(sc.status.item())}")
+    ra = stage.request_arrays(w, device=dev)
+    chains, _ = sdev.chains(w, device=dev)
+    x = StepInputs(util=sdev.util(w, device=dev), chains=chains, chain_off=ra["chain_off"],
+                   set_off=ra["set_off"], length=ra["length"], prefill=ra["prefill"],
+                   snap=ra["snap"], events=ra["events"], event_off=ra["event_off"],
+                   weights=weights_tensor(w.weights, theta, spec.cap_tokens, bpt, device=dev))
+    out = sc.alloc_outputs(x.n_snap, x.R, x.n_streams)
+    return w, sc, x, out
+
+
+# ------------------------------------------------------------------ GPU arm
+def run_netkv(args):
+    import torch
+    import synth
     import __graft_entry__
     rank, world, local = dist_env()
     if world > 1:
@@ -209,34 +246,13 @@ def run_netkv(args):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     __graft_entry__.build()
-    from paper_2606_03910_gb300.pipeline import Scorer, StepInputs, weights_tensor
+    from paper_2606_03910_gb300.pipeline import StepInputs
 
-    spec = synth.config1(args.streams)
-    spec.seed0 = rank_seed0(rank, args.streams)
-    w = synth.make_workload(spec)
+    w, sc, x, out = setup_replicas(args.streams, rank, dev, args.table_batch)
+    sc.share_prefixes = not args.no_share
     theta = float(np.float32(synth.THETA_S_PER_TOKEN))
     bpt = synth.BYTES_PER_TOKEN_SHARD
-
-    # resident caches, built in batches of table sets
-    from paper_2606_03910_gb300 import netkv
-    log2_index = netkv.index_log2_capacity(synth.distinct_keys_per_group(w))
-    sc = Scorer(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, w.L, w.n_sets, log2_index,
-                device=dev)
-    for g0 in range(0, w.n_sets, args.table_batch):
-        g1 = min(w.n_sets, g0 + args.table_batch)
-        keys = sdev.keys(w, g0, g1, device=dev)
-        sc.load_caches(keys, stage.key_offsets(w, (g1 - g0) * w.D, device=dev), set0=g0,
-                       n_sets=g1 - g0)
-        del keys
-    torch.cuda.synchronize()
-
-    ra = stage.request_arrays(w, device=dev)
-    chains, _ = sdev.chains(w, device=dev)
-    x = StepInputs(util=sdev.util(w, device=dev), chains=chains, chain_off=ra["chain_off"],
-                   set_off=ra["set_off"], length=ra["length"], prefill=ra["prefill"],
-                   snap=ra["snap"], events=ra["events"], event_off=ra["event_off"],
-                   weights=weights_tensor(w.weights, theta, spec.cap_tokens, bpt, device=dev))
-    out = sc.alloc_outputs(x.n_snap, x.R, x.n_streams)
+    spec = w.spec
     stream = torch.cuda.current_stream(dev)
     for _ in range(args.warmup):
         sc.step(x, out, stream)
@@ -277,6 +293,8 @@ def run_netkv(args):
     # level bottlenecks 1; prefix match 4 (group insert, group resolve, leaders, members)
     # with a workspace or 1 without; greedy 1
     launches_per_step = 1 + (4 if sc.share_prefixes else 1) + 1
+    n_input_tensors = sum(1 for f in dataclasses.fields(StepInputs)
+                          if isinstance(getattr(x, f.name), torch.Tensor))
     decisions = R * world
     value = decisions / (ms / 1e3)
 
@@ -308,7 +326,6 @@ def run_netkv(args):
     # ---- end to end through the public API with pinned host buffers
     e2e = None
     if not args.no_e2e:
-        import dataclasses
         xh = StepInputs(**{f.name: (getattr(x, f.name).cpu().pin_memory()
                                     if isinstance(getattr(x, f.name), torch.Tensor) else None)
                            for f in dataclasses.fields(StepInputs)})
@@ -330,7 +347,8 @@ def run_netkv(args):
         ems = e0.elapsed_time(e1) / args.steps
         ems = max_over_ranks(ems, dev)
         e2e = {"value": decisions / (ems / 1e3), "unit": UNIT, "ms_per_step": round(ems, 3),
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+               "gpu_launches_per_step": launches_per_step + n_input_tensors + 4}
 
     # ---- CPU oracle baseline, rank 0 at N=1 only
     cpu = None

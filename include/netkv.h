@@ -54,7 +54,8 @@ typedef enum {
 /* Bits OR-ed into *d_status by the kernels. */
 #define NETKV_DEV_EDOMAIN 1 /* utilisation outside [0,1) or NaN; zero-length request;
                                hash value 0 in a chain or key list; M[r][d] > len/16 */
-#define NETKV_DEV_EFULL 2   /* a hash table had no free slot, or a probe ran the whole table */
+#define NETKV_DEV_EFULL 2   /* a hash table had no free slot, a probe ran the whole table,
+                               or a cache index is inconsistent */
 #define NETKV_DEV_ERANGE 4  /* a request, prefill rank or snapshot index out of range */
 
 /* ------------------------------------------------------------------ topology
@@ -118,24 +119,28 @@ netkv_status netkv_oracle_build(netkv_topology_t topo, const float* d_util, uint
                                 netkv_stream_t stream);
 
 /* ------------------------------------------------------------------ caches
- * Decode caches K_d (Sec. III-C), the sets of block hashes each decode instance holds,
- * stored as an inverted index.  Decodes are taken in groups of 64 (decode ranks
- * 64q .. 64q+63 form group q); each (table set, group) has one open-addressing table
- * of 2^log2_capacity slots of 16 bytes, {uint64 block hash, uint64 mask}, where bit
- * (d mod 64) of the mask says that decode d caches the hash.  Hash 0 marks an empty slot
- * (block hash 0 is reserved).  Linear probing from a multiplicative hash of the key.
- * The index of table set g, group q starts at slot ((g * G + q) << log2_capacity),
- * G = ceil(D / 64).  One table must hold the distinct hashes of its group's decodes:
- * keep its load factor below about 0.5.
+ * Decode caches K_d (Sec. III-C), the sets of block hashes each decode instance holds.
+ * Decodes are taken in groups of 64 (decode ranks 64q .. 64q+63 form group q); each
+ * (table set g, group q) has one index of 2^log2_capacity hash slots followed by
+ * 2^log2_capacity run entries, index number g * G + q with G = ceil(D / 64):
+ *   run entries  {uint64 hash, uint64 mask}: the group's distinct cached hashes in list
+ *                order (decode by decode, first appearance); bit (d mod 64) of the mask
+ *                says that decode d caches the hash;
+ *   hash slots   {uint64 hash, uint64 run position}, open addressing with linear probing
+ *                from a multiplicative hash; hash 0 marks an empty slot (block hash 0 is
+ *                reserved).
+ * Lists that give each cached prefix in chain order (as caches are filled) let the match
+ * follow runs instead of probing block by block; any order gives the same results.
+ * Keep the group's distinct hashes below about half of 2^log2_capacity.
  *
  *   d_index    device buffer of netkv_cache_index_bytes(n_sets, D, log2_capacity) bytes,
  *              16-byte aligned; cleared, then filled by netkv_cache_build
  *   d_keys     keys of (set g, decode d), list t = g * D + d, are
  *              d_keys[d_key_off[t] .. d_key_off[t+1])
  *   d_key_off  [n_sets * D + 1] uint64, non-decreasing
- * Duplicate keys are stored once.  A zero key sets EDOMAIN and is skipped; a table with
+ * Duplicate keys are stored once.  A zero key sets EDOMAIN and is skipped; an index with
  * more distinct keys than slots sets EFULL (the excess keys are dropped).
- * 1 <= log2_capacity <= 32.
+ * 1 <= log2_capacity <= 31.
  */
 size_t netkv_cache_index_bytes(uint32_t n_sets, uint32_t D, uint32_t log2_capacity);
 netkv_status netkv_cache_build(void* d_index, uint32_t n_sets, uint32_t D,
@@ -234,18 +239,35 @@ typedef struct {
  *   d_best       [R] fp32 output: minimum score (+inf when rejected)
  *   d_second     [R] fp32 output: minimum over the other feasible candidates (+inf if none)
  *   d_load_final [n_streams][D] int64 output: loads after the last event
+ *   d_workspace  NULL, or a device buffer of at least netkv_schedule_workspace_size(R, D)
+ *                bytes, 256-byte aligned, owned by the caller and overwritten by the call.
+ *                With a workspace the decision-independent part of every arrival's scores
+ *                (w_net * T_xfer + w_prefix * miss) is computed first for all arrivals in
+ *                parallel and the sequential walk only adds the load term; without one
+ *                the walk computes every term itself.  Overlapping calls need distinct
+ *                workspaces.
  * Every request index must occur in at most one stream, and its departure after its
  * arrival.  Out-of-range indices set ERANGE and the event is skipped.  The topology
  * may have at most 4096 decode instances.
  */
+size_t netkv_schedule_workspace_size(uint32_t R, uint32_t D);
 netkv_status netkv_schedule_streams(netkv_topology_t topo, uint32_t n_streams,
                                     const netkv_weights* d_w, uint32_t R, const uint32_t* d_len,
                                     const uint32_t* d_prefill, const uint32_t* d_snap,
                                     const uint16_t* d_M, const float* d_UB, uint32_t n_snap,
                                     const uint32_t* d_events, const uint64_t* d_event_off,
                                     const int64_t* d_load_init, int32_t* d_dec, float* d_best,
-                                    float* d_second, int64_t* d_load_final, int* d_status,
-                                    netkv_stream_t stream);
+                                    float* d_second, int64_t* d_load_final, void* d_workspace,
+                                    size_t workspace_bytes, int* d_status, netkv_stream_t stream);
+
+/* ------------------------------------------------------------------ transfers
+ * Asynchronous copy of `bytes` bytes by a kernel (SM loads and stores).  Either side may
+ * be device memory or pinned host memory reachable through unified addressing (memory
+ * from cudaHostAlloc / cudaMallocHost); on NVLink-C2C systems this moves a step's inputs
+ * host->device faster than the copy engines.  Both pointers 16-byte aligned; the
+ * regions must not overlap.  Used by the host-buffer step; not part of the paper's path.
+ */
+netkv_status netkv_copy_async(void* dst, const void* src, size_t bytes, netkv_stream_t stream);
 
 /* Library version, for the bindings' load check. */
 uint32_t netkv_version(void);

@@ -2,20 +2,27 @@
 // M[r][d] = |LCP_block(h_r, K_d)|, the number of leading blocks of request r's hash chain
 // that are all cached on decode d.
 //
-// Cache index.  The caches of a table set are stored as an inverted index: one
-// open-addressing table per group of up to 64 decodes, whose 16-byte slots hold a block
-// hash and a 64-bit mask of the group's decodes that cache it.  One probe therefore
-// answers the membership question for every decode of the group at once; the decodes
-// of a set mostly cache the same shared prefixes, so this also keeps the index small.
-//   cache_insert_kernel: one block per (set, decode) key list; linear probing from a
-//   Fibonacci-hashed home slot, atomicCAS to claim the slot, atomicOr to add the decode.
+// Cache index.  The caches of a table set are indexed per group of up to 64 decodes:
+//   run array   the group's distinct cached hashes in the order the key lists give them
+//               (decode by decode, first appearance), each with a 64-bit mask of the
+//               group's decodes that cache it;
+//   hash table  open addressing, 16-byte slots {hash, position in the run array}.
+// Caches are filled with whole prefixes of chains, so a cached prefix sits in the run
+// array as a contiguous run in chain order.
+//   cache_build_kernel: one CTA per index; it walks the lists in order in chunks of 1024
+//   keys, claims new hashes with atomicCAS, numbers them with a block-wide scan and
+//   appends them to the run array, and ORs each decode's bit into the hashes it lists.
 //
-// Match.  One warp per (request, decode group).  The warp first probes the block at the
-// starting position (one probe serves the whole group), then walks the chain in chunks of
-// 32 consecutive blocks: a 256-byte coalesced chain load, one index probe per lane, and one
-// ballot per live decode to find its first missing block; a decode leaves once its first
-// miss is known and the warp stops when every decode of the group has missed.  Probes are
-// bounded by the table size.
+// Match.  One warp per (request, decode group).  The warp looks up the block at the
+// current position in the hash table (one random access), then compares the chain with
+// the run array from that position on, 32 blocks per step (a 256-byte chain load and a
+// 512-byte run load, both coalesced): every block that equals the next run entry is
+// cached exactly on the decodes of that entry's mask, and one ballot per live decode
+// finds its first missing block.  Where chain and run part, the next block is looked up
+// in the hash table again; a block absent from the table is missing on every decode.
+// The answer never depends on the run order (any key order is exact); the order only
+// decides how many random lookups a chain needs.  A decode leaves once its first miss is
+// known and the warp stops when every decode of the group has missed.
 //
 // Prefix sharing.  Requests that share leading blocks have the same membership answers
 // on those blocks, so with a workspace the match runs in three steps:
@@ -27,73 +34,134 @@
 //   match_kernel<kMembers>: a member r with leader L compares chains to get
 //     lcp = |common prefix of h_r and h_L| (capped at max_d M_L[d] + 1).  For a decode
 //     with M_L[d] < lcp the first missing block of L lies inside the common prefix, so
-//     M_r[d] = M_L[d] exactly; otherwise blocks [0, lcp) are all cached and the probe
-//     resumes at block lcp.  The result equals the full match whatever the grouping;
-//     grouping only decides how much probing is saved.
+//     M_r[d] = M_L[d] exactly; otherwise blocks [0, lcp) are all cached and the walk
+//     resumes at block lcp.  The result equals the full match whatever the grouping.
 #include "netkv_internal.cuh"
 
 namespace {
 
-constexpr int kInsertBlock = 256;
+constexpr int kBuildBlock = 1024;
 constexpr int kMatchBlock = 256;
-constexpr uint32_t kGroup = 64;  // decodes per index table (bits of the mask)
+constexpr uint32_t kGroup = 64;  // decodes per index (bits of the mask)
+constexpr unsigned long long kNotFound = ~0ull;
 
 struct __align__(16) IndexSlot {
   unsigned long long key;
-  unsigned long long mask;
+  unsigned long long pos;  // position of the key in the run array
 };
 
-__global__ void __launch_bounds__(kInsertBlock) cache_insert_kernel(
-    IndexSlot* __restrict__ index, uint32_t n_sets, uint32_t D, uint32_t log2_cap,
+struct __align__(16) RunEntry {
+  unsigned long long key;
+  unsigned long long mask;  // decodes of the group that cache the key
+};
+
+// Hash table and run array of index (set g, decode group q): 2^L slots then 2^L entries.
+__device__ __forceinline__ IndexSlot* index_hash(void* index, uint64_t idx, uint32_t L) {
+  return reinterpret_cast<IndexSlot*>(index) + (idx << (L + 1));
+}
+__device__ __forceinline__ const IndexSlot* index_hash(const void* index, uint64_t idx,
+                                                       uint32_t L) {
+  return reinterpret_cast<const IndexSlot*>(index) + (idx << (L + 1));
+}
+
+// Exclusive scan of one flag per thread over a 1024-thread block; returns the prefix and
+// writes the block total to *total (shared).
+__device__ __forceinline__ uint32_t block_scan(uint32_t flag, uint32_t* warp_sums,
+                                               uint32_t* total) {
+  const uint32_t lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const uint32_t b = __ballot_sync(0xffffffffu, flag);
+  const uint32_t in_warp = __popc(b & ((1u << lane) - 1));
+  if (lane == 0) warp_sums[wid] = __popc(b);
+  __syncthreads();
+  if (wid == 0) {
+    const uint32_t v = warp_sums[lane];
+    uint32_t x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= (uint32_t)o) x += y;
+    }
+    warp_sums[lane] = x - v;  // exclusive
+    if (lane == 31) *total = x;
+  }
+  __syncthreads();
+  return warp_sums[wid] + in_warp;
+}
+
+__global__ void __launch_bounds__(kBuildBlock) cache_build_kernel(
+    void* __restrict__ index, uint32_t n_sets, uint32_t D, uint32_t log2_cap,
     const uint64_t* __restrict__ keys, const uint64_t* __restrict__ key_off, int* status) {
+  __shared__ uint32_t warp_sums[32];
+  __shared__ uint32_t chunk_new;
   const uint64_t cap = 1ull << log2_cap, mask = cap - 1;
   const uint32_t n_dgroups = (D + kGroup - 1) / kGroup;
-  const uint64_t n_lists = (uint64_t)n_sets * D;
-  for (uint64_t t = blockIdx.x; t < n_lists; t += gridDim.x) {
-    const uint64_t beg = __ldg(key_off + t), end = __ldg(key_off + t + 1);
-    if (end < beg) {
-      if (threadIdx.x == 0) flag_status(status, NETKV_DEV_ERANGE);
-      continue;
-    }
-    const uint64_t g = t / D;
-    const uint32_t d = (uint32_t)(t - g * D);
-    IndexSlot* tab = index + ((g * n_dgroups + d / kGroup) << log2_cap);
-    const unsigned long long bit = 1ull << (d % kGroup);
-    for (uint64_t j = beg + threadIdx.x; j < end; j += blockDim.x) {
-      const unsigned long long key = __ldg(keys + j);
-      if (key == 0ull) {
-        flag_status(status, NETKV_DEV_EDOMAIN);
+  const uint64_t n_index = (uint64_t)n_sets * n_dgroups;
+  for (uint64_t idx = blockIdx.x; idx < n_index; idx += gridDim.x) {
+    const uint64_t g = idx / n_dgroups;
+    const uint32_t q = (uint32_t)(idx - g * n_dgroups);
+    IndexSlot* hash = index_hash(index, idx, log2_cap);
+    RunEntry* run = reinterpret_cast<RunEntry*>(hash + cap);
+    uint32_t run_len = 0;  // same value in every thread
+    for (uint32_t d = q * kGroup; d < min(D, (q + 1) * kGroup); ++d) {
+      const uint64_t t = g * D + d;
+      const uint64_t beg = __ldg(key_off + t), end = __ldg(key_off + t + 1);
+      if (end < beg) {
+        if (threadIdx.x == 0) flag_status(status, NETKV_DEV_ERANGE);
         continue;
       }
-      uint64_t slot = home_slot(key, log2_cap);
-      uint64_t step = 0;
-      for (; step < cap; ++step) {
-        const unsigned long long prev = atomicCAS(&tab[slot].key, 0ull, key);
-        if (prev == 0ull || prev == key) {
-          atomicOr(&tab[slot].mask, bit);
-          break;
+      const unsigned long long bit = 1ull << (d % kGroup);
+      for (uint64_t c = beg; c < end; c += kBuildBlock) {
+        const uint64_t j = c + threadIdx.x;
+        unsigned long long key = j < end ? __ldg(keys + j) : 0ull;
+        if (j < end && key == 0ull) flag_status(status, NETKV_DEV_EDOMAIN);
+        bool is_new = false;
+        uint64_t slot = 0;
+        bool placed = false;
+        if (key != 0ull) {
+          slot = home_slot(key, log2_cap);
+          for (uint64_t step = 0; step < cap; ++step) {
+            const unsigned long long prev = atomicCAS(&hash[slot].key, 0ull, key);
+            if (prev == 0ull || prev == key) {
+              is_new = prev == 0ull;
+              placed = true;
+              break;
+            }
+            slot = (slot + 1) & mask;
+          }
+          if (!placed) flag_status(status, NETKV_DEV_EFULL);
         }
-        slot = (slot + 1) & mask;
+        const uint32_t pos = run_len + block_scan(is_new ? 1u : 0u, warp_sums, &chunk_new);
+        if (is_new) {
+          hash[slot].pos = pos;
+          run[pos].key = key;
+          run[pos].mask = bit;
+        }
+        __syncthreads();
+        if (placed && !is_new) {
+          const uint64_t p = *((volatile unsigned long long*)&hash[slot].pos);
+          atomicOr(&run[p].mask, bit);
+        }
+        run_len += chunk_new;
+        __syncthreads();
       }
-      if (step == cap) flag_status(status, NETKV_DEV_EFULL);
     }
   }
 }
 
-// Decodes of the group that cache `key` (non-zero); 0 when absent.
-__device__ __forceinline__ unsigned long long lookup(const IndexSlot* __restrict__ tab,
+// Run position of `key` (non-zero) in one index, or kNotFound.
+__device__ __forceinline__ unsigned long long lookup(const IndexSlot* __restrict__ hash,
                                                      uint64_t key, uint32_t log2_cap,
                                                      int* status) {
   const uint64_t mask = (1ull << log2_cap) - 1;
   uint64_t slot = home_slot(key, log2_cap);
   for (uint64_t seen = 0; seen <= mask; ++seen) {
-    const ulonglong2 s = __ldg(reinterpret_cast<const ulonglong2*>(tab + slot));
+    const ulonglong2 s = __ldg(reinterpret_cast<const ulonglong2*>(hash + slot));
     if (s.x == key) return s.y;
-    if (s.x == 0ull) return 0ull;
+    if (s.x == 0ull) return kNotFound;
     slot = (slot + 1) & mask;
   }
   flag_status(status, NETKV_DEV_EFULL);
-  return 0ull;
+  return kNotFound;
 }
 
 __device__ __forceinline__ int32_t find_set(const uint32_t* __restrict__ set_off, uint32_t n_sets,
@@ -118,48 +186,74 @@ __device__ __forceinline__ void set_hit(GroupHits& h, uint32_t lane, uint32_t j,
   if (j == lane + 32) h.hi = v;
 }
 
+// Every decode in `alive` misses at position v.
+__device__ __forceinline__ void miss_all(GroupHits& h, uint32_t lane, unsigned long long alive,
+                                         uint32_t v) {
+  if ((alive >> lane) & 1ull) h.lo = v;
+  if ((alive >> (lane + 32)) & 1ull) h.hi = v;
+}
+
 // First-miss scan of blocks [start, n) of one chain for the `alive` decodes of a group.
 // Decodes found missing at position p get p; decodes never missing keep their value.
-__device__ __forceinline__ void scan_chain(const IndexSlot* __restrict__ tab, uint32_t log2_cap,
+__device__ __forceinline__ void scan_chain(const IndexSlot* __restrict__ hash, uint32_t log2_cap,
                                            const uint64_t* __restrict__ chain, uint64_t start,
                                            uint64_t n, unsigned long long alive, GroupHits& h,
                                            uint32_t lane, int* status) {
-  if (!alive || start >= n) return;
-  {  // the first block: one probe for the whole group
-    const uint64_t key = __ldg(chain + start);
-    unsigned long long mk = 0ull;
-    if (key == 0ull) {
-      if (lane == 0) flag_status(status, NETKV_DEV_EDOMAIN);
-    } else if (lane == 0) {
-      mk = lookup(tab, key, log2_cap, status);
+  const uint64_t cap = 1ull << log2_cap;
+  const RunEntry* __restrict__ run = reinterpret_cast<const RunEntry*>(hash + cap);
+  uint64_t p = start;
+  uint64_t seg_run = 0, seg_p = 0;  // run position matched with chain position seg_p
+  bool in_run = false;
+  while (p < n && alive) {
+    const bool looked_up = !in_run;
+    if (!in_run) {  // locate block p in the hash table
+      const uint64_t key = __ldg(chain + p);
+      unsigned long long pos = kNotFound;
+      if (lane == 0) {
+        if (key == 0ull) flag_status(status, NETKV_DEV_EDOMAIN);
+        else pos = lookup(hash, key, log2_cap, status);
+      }
+      pos = __shfl_sync(0xffffffffu, pos, 0);
+      if (pos == kNotFound) {  // absent from every cache of the group
+        miss_all(h, lane, alive, (uint32_t)p);
+        return;
+      }
+      seg_run = pos;
+      seg_p = p;
+      in_run = true;
     }
-    mk = __shfl_sync(0xffffffffu, mk, 0);
-    unsigned long long miss = alive & ~mk;
-    while (miss) {
-      const uint32_t j = __ffsll((long long)miss) - 1;
-      miss &= miss - 1;
-      set_hit(h, lane, j, (uint32_t)start);
-    }
-    alive &= mk;
-    ++start;
-  }
-  for (uint64_t base = start; base < n && alive; base += 32) {
-    const uint64_t i = base + lane;
+    // blocks p .. p+31 against the run from seg_run
+    const uint64_t i = p + lane;
+    const uint64_t rp = seg_run + (i - seg_p);
     const bool in = i < n;
-    const uint64_t key = in ? __ldcs(chain + i) : 0ull;
-    if (in && key == 0ull) flag_status(status, NETKV_DEV_EDOMAIN);
-    const unsigned long long mk = (in && key != 0ull) ? lookup(tab, key, log2_cap, status) : 0ull;
-    const uint32_t valid = __ballot_sync(0xffffffffu, in);
-    unsigned long long a = alive;
+    const uint64_t ck = in ? __ldcs(chain + i) : 0ull;
+    ulonglong2 re = make_ulonglong2(0ull, 0ull);
+    if (in && rp < cap) re = __ldg(reinterpret_cast<const ulonglong2*>(run + rp));
+    const bool same = in && ck != 0ull && re.x == ck;
+    const uint32_t run_ok = __ballot_sync(0xffffffffu, same);
+    const uint32_t lead = (~run_ok) ? (uint32_t)(__ffs(~run_ok) - 1) : 32u;  // leading matches
+    const bool counted = lane < lead;
+    // decodes missing at some counted position of this step (usually none)
+    const unsigned long long nm = counted ? (alive & ~re.y) : 0ull;
+    unsigned long long a = ((unsigned long long)__reduce_or_sync(0xffffffffu, (uint32_t)(nm >> 32))
+                            << 32) |
+                           __reduce_or_sync(0xffffffffu, (uint32_t)nm);
     while (a) {
       const uint32_t j = __ffsll((long long)a) - 1;
       a &= a - 1;
-      const uint32_t miss = valid & ~__ballot_sync(0xffffffffu, (mk >> j) & 1ull);
-      if (miss) {
-        set_hit(h, lane, j, (uint32_t)base + (uint32_t)(__ffs(miss) - 1));
-        alive &= ~(1ull << j);
-      }
+      const uint32_t miss = __ballot_sync(0xffffffffu, (nm >> j) & 1ull);
+      set_hit(h, lane, j, (uint32_t)(p + (uint64_t)(__ffs(miss) - 1)));
+      alive &= ~(1ull << j);
     }
+    if (lead == 0 && looked_up) {
+      // the run entry the table points to does not hold the key: a corrupted index.
+      // Report it and count the block as missing, so the walk always advances.
+      if (lane == 0) flag_status(status, NETKV_DEV_EFULL);
+      miss_all(h, lane, alive, (uint32_t)p);
+      return;
+    }
+    p += lead;
+    if (lead < 32) in_run = false;  // the run parts here: look the next block up
   }
 }
 
@@ -214,7 +308,7 @@ __global__ void group_resolve_kernel(const GroupSlot* __restrict__ tab, uint32_t
                                      const uint64_t* __restrict__ chains,
                                      const uint64_t* __restrict__ chain_off, uint32_t R,
                                      const uint32_t* __restrict__ set_off, uint32_t n_sets,
-                                     uint32_t* __restrict__ leader_of,
+                                     uint32_t* __restrict__ leader_of, int32_t* __restrict__ set_of,
                                      uint32_t* __restrict__ leaders, MatchCounters* counters) {
   const uint64_t mask = (1ull << log2_slots) - 1;
   for (uint32_t r = blockIdx.x * blockDim.x + threadIdx.x; r < R; r += gridDim.x * blockDim.x) {
@@ -237,6 +331,7 @@ __global__ void group_resolve_kernel(const GroupSlot* __restrict__ tab, uint32_t
       }
     }
     leader_of[r] = lead;
+    set_of[r] = set;
     if (lead == r) leaders[atomicAdd(&counters->n_leaders, 1ull)] = r;
   }
 }
@@ -244,10 +339,10 @@ __global__ void group_resolve_kernel(const GroupSlot* __restrict__ tab, uint32_t
 // Chain r's extent clamped to 65535 blocks; false on a bad request (flagged).
 __device__ __forceinline__ bool chain_extent(const uint64_t* __restrict__ chain_off,
                                              const uint32_t* __restrict__ set_off,
-                                             uint32_t n_sets, uint32_t r, uint32_t lane,
-                                             int* status, int32_t& set, uint64_t& c0,
-                                             uint64_t& n) {
-  set = find_set(set_off, n_sets, r);
+                                             uint32_t n_sets, const int32_t* __restrict__ set_of,
+                                             uint32_t r, uint32_t lane, int* status,
+                                             int32_t& set, uint64_t& c0, uint64_t& n) {
+  set = set_of ? __ldg(set_of + r) : find_set(set_off, n_sets, r);
   c0 = __ldg(chain_off + r);
   const uint64_t c1 = __ldg(chain_off + r + 1);
   if (set < 0 || c1 < c0) {
@@ -271,10 +366,11 @@ __device__ __forceinline__ void store_hits(uint16_t* __restrict__ M, uint64_t ro
 // Leader pass: one task per (leader, decode group), taken in order from a global counter
 // by whole warps, so long and short chains balance across the GPU.
 __global__ void __launch_bounds__(kMatchBlock) match_leaders_kernel(
-    const IndexSlot* __restrict__ index, uint32_t D, uint32_t log2_cap, uint32_t n_sets,
+    const void* __restrict__ index, uint32_t D, uint32_t log2_cap, uint32_t n_sets,
     const uint64_t* __restrict__ chains, const uint64_t* __restrict__ chain_off,
-    const uint32_t* __restrict__ set_off, const uint32_t* __restrict__ leaders,
-    MatchCounters* counters, uint16_t* __restrict__ M, int* status) {
+    const uint32_t* __restrict__ set_off, const int32_t* __restrict__ set_of,
+    const uint32_t* __restrict__ leaders, MatchCounters* counters, uint16_t* __restrict__ M,
+    int* status) {
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t n_dgroups = (D + kGroup - 1) / kGroup;
   const unsigned long long total =
@@ -284,16 +380,17 @@ __global__ void __launch_bounds__(kMatchBlock) match_leaders_kernel(
     if (lane == 0) t = atomicAdd(&counters->next_task, 1ull);
     t = __shfl_sync(0xffffffffu, t, 0);
     if (t >= total) break;
-    const uint32_t r = __ldg(leaders + t / n_dgroups);
-    const uint32_t q = (uint32_t)(t % n_dgroups);
+    const uint64_t li = n_dgroups == 1 ? t : t / n_dgroups;
+    const uint32_t r = __ldg(leaders + li);
+    const uint32_t q = (uint32_t)(t - li * n_dgroups);
     const uint32_t q0 = q * kGroup, ng = min(kGroup, D - q0);
     GroupHits h = {0u, 0u};
     int32_t set;
     uint64_t c0, n;
-    if (chain_extent(chain_off, set_off, n_sets, r, lane, status, set, c0, n)) {
+    if (chain_extent(chain_off, set_off, n_sets, set_of, r, lane, status, set, c0, n)) {
       h.lo = h.hi = (uint32_t)n;
       const unsigned long long alive = ng >= 64 ? ~0ull : ((1ull << ng) - 1);
-      const IndexSlot* tab = index + (((uint64_t)set * n_dgroups + q) << log2_cap);
+      const IndexSlot* tab = index_hash(index, (uint64_t)set * n_dgroups + q, log2_cap);
       scan_chain(tab, log2_cap, chains + c0, 0, n, alive, h, lane, status);
     }
     store_hits(M, (uint64_t)r * D, q0, ng, lane, h);
@@ -302,10 +399,10 @@ __global__ void __launch_bounds__(kMatchBlock) match_leaders_kernel(
 
 template <int kMode>
 __global__ void __launch_bounds__(kMatchBlock) match_kernel(
-    const IndexSlot* __restrict__ index, uint32_t D, uint32_t log2_cap, uint32_t n_sets,
+    const void* __restrict__ index, uint32_t D, uint32_t log2_cap, uint32_t n_sets,
     const uint64_t* __restrict__ chains, const uint64_t* __restrict__ chain_off, uint32_t R,
     const uint32_t* __restrict__ set_off, const uint32_t* __restrict__ leader_of,
-    uint16_t* __restrict__ M, int* status) {
+    const int32_t* __restrict__ set_of, uint16_t* __restrict__ M, int* status) {
   const uint32_t lane = threadIdx.x & 31;
   const uint64_t warp = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const uint64_t n_warps = ((uint64_t)gridDim.x * blockDim.x) >> 5;
@@ -313,7 +410,7 @@ __global__ void __launch_bounds__(kMatchBlock) match_kernel(
   const uint64_t total = (uint64_t)R * n_dgroups;
 
   for (uint64_t task = warp; task < total; task += n_warps) {
-    const uint32_t r = (uint32_t)(task / n_dgroups);
+    const uint32_t r = (uint32_t)(n_dgroups == 1 ? task : task / n_dgroups);
     uint32_t lead = r;
     if (kMode == kMembers) {
       lead = __ldg(leader_of + r);
@@ -324,7 +421,7 @@ __global__ void __launch_bounds__(kMatchBlock) match_kernel(
     GroupHits h = {0u, 0u};
     int32_t set;
     uint64_t c0, n;
-    if (!chain_extent(chain_off, set_off, n_sets, r, lane, status, set, c0, n)) {
+    if (!chain_extent(chain_off, set_off, n_sets, set_of, r, lane, status, set, c0, n)) {
       store_hits(M, (uint64_t)r * D, q0, ng, lane, h);
       continue;
     }
@@ -370,7 +467,7 @@ __global__ void __launch_bounds__(kMatchBlock) match_kernel(
       alive &= ~copy;
       start = lcp;
     }
-    const IndexSlot* tab = index + (((uint64_t)set * n_dgroups + q) << log2_cap);
+    const IndexSlot* tab = index_hash(index, (uint64_t)set * n_dgroups + q, log2_cap);
     scan_chain(tab, log2_cap, chains + c0, start, n, alive, h, lane, status);
     store_hits(M, (uint64_t)r * D, q0, ng, lane, h);
   }
@@ -384,16 +481,17 @@ uint32_t group_log2_slots(uint32_t R) {
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-// Workspace: group table | leader_of [R] | leader list [R] | counters.
+// Workspace: group table | leader_of [R] | set_of [R] | leader list [R] | counters.
 struct WorkspaceLayout {
-  size_t table, leader_of, leaders, counters, total;
+  size_t table, leader_of, set_of, leaders, counters, total;
 };
 
 WorkspaceLayout workspace_layout(uint32_t R) {
   WorkspaceLayout w;
   w.table = 0;
   w.leader_of = align_up(sizeof(GroupSlot) << group_log2_slots(R), 256);
-  w.leaders = w.leader_of + align_up(sizeof(uint32_t) * (size_t)R, 256);
+  w.set_of = w.leader_of + align_up(sizeof(uint32_t) * (size_t)R, 256);
+  w.leaders = w.set_of + align_up(sizeof(int32_t) * (size_t)R, 256);
   w.counters = w.leaders + align_up(sizeof(uint32_t) * (size_t)R, 256);
   w.total = w.counters + align_up(sizeof(MatchCounters), 256);
   return w;
@@ -410,15 +508,16 @@ int leader_grid() {
 }  // namespace
 
 extern "C" size_t netkv_cache_index_bytes(uint32_t n_sets, uint32_t D, uint32_t log2_capacity) {
-  if (log2_capacity < 1 || log2_capacity > 32) return 0;
-  return (size_t)n_sets * ((D + kGroup - 1) / kGroup) * (sizeof(IndexSlot) << log2_capacity);
+  if (log2_capacity < 1 || log2_capacity > 31) return 0;
+  return (size_t)n_sets * ((D + kGroup - 1) / kGroup) *
+         ((sizeof(IndexSlot) + sizeof(RunEntry)) << log2_capacity);
 }
 
 extern "C" netkv_status netkv_cache_build(void* d_index, uint32_t n_sets, uint32_t D,
                                           uint32_t log2_capacity, const uint64_t* d_keys,
                                           const uint64_t* d_key_off, int* d_status,
                                           netkv_stream_t stream) {
-  if (!d_index || !d_key_off || D == 0 || log2_capacity < 1 || log2_capacity > 32)
+  if (!d_index || !d_key_off || D == 0 || log2_capacity < 1 || log2_capacity > 31)
     return NETKV_EINVAL;
   if (!aligned_to(d_index, 16) || !aligned_to(d_key_off, 8) || (d_keys && !aligned_to(d_keys, 8)))
     return NETKV_EINVAL;
@@ -426,10 +525,10 @@ extern "C" netkv_status netkv_cache_build(void* d_index, uint32_t n_sets, uint32
   cudaStream_t s = (cudaStream_t)stream;
   NETKV_CUDA_TRY(cudaMemsetAsync(d_index, 0, netkv_cache_index_bytes(n_sets, D, log2_capacity), s));
   if (!d_keys) return NETKV_OK;
-  const uint64_t lists = (uint64_t)n_sets * D;
-  const unsigned grid = (unsigned)(lists < (1u << 20) ? lists : (1u << 20));
-  cache_insert_kernel<<<grid, kInsertBlock, 0, s>>>(reinterpret_cast<IndexSlot*>(d_index), n_sets,
-                                                    D, log2_capacity, d_keys, d_key_off, d_status);
+  const uint64_t n_index = (uint64_t)n_sets * ((D + kGroup - 1) / kGroup);
+  const unsigned grid = (unsigned)(n_index < (1u << 20) ? n_index : (1u << 20));
+  cache_build_kernel<<<grid, kBuildBlock, 0, s>>>(d_index, n_sets, D, log2_capacity, d_keys,
+                                                  d_key_off, d_status);
   return netkv_launch_status();
 }
 
@@ -445,7 +544,7 @@ extern "C" netkv_status netkv_prefix_match(const void* d_index, uint32_t D,
                                            void* d_workspace, size_t workspace_bytes,
                                            uint16_t* d_M, int* d_status, netkv_stream_t stream) {
   if (!d_index || !d_chain_off || !d_M || D == 0 || n_sets == 0) return NETKV_EINVAL;
-  if (log2_capacity < 1 || log2_capacity > 32) return NETKV_EINVAL;
+  if (log2_capacity < 1 || log2_capacity > 31) return NETKV_EINVAL;
   if (n_sets > 1 && !d_set_off) return NETKV_EINVAL;
   if (!aligned_to(d_index, 16) || !aligned_to(d_chain_off, 8) || !aligned_to(d_M, 2) ||
       (d_chains && !aligned_to(d_chains, 8)) || (d_set_off && !aligned_to(d_set_off, 4)) ||
@@ -455,15 +554,15 @@ extern "C" netkv_status netkv_prefix_match(const void* d_index, uint32_t D,
   if (!d_chains || R > 0x7fffffffu) return NETKV_EINVAL;
   if (d_workspace && workspace_bytes < netkv_prefix_match_workspace_size(R)) return NETKV_EINVAL;
   cudaStream_t s = (cudaStream_t)stream;
-  const IndexSlot* index = reinterpret_cast<const IndexSlot*>(d_index);
+  const void* index = d_index;
   const uint64_t tasks = (uint64_t)R * ((D + kGroup - 1) / kGroup);
   const uint64_t warps_per_block = kMatchBlock / 32;
   const uint64_t blocks = (tasks + warps_per_block - 1) / warps_per_block;
   const unsigned grid = (unsigned)(blocks < (1u << 24) ? blocks : (1u << 24));
   if (!d_workspace) {
     match_kernel<kAll><<<grid, kMatchBlock, 0, s>>>(index, D, log2_capacity, n_sets, d_chains,
-                                                    d_chain_off, R, d_set_off, nullptr, d_M,
-                                                    d_status);
+                                                    d_chain_off, R, d_set_off, nullptr, nullptr,
+                                                    d_M, d_status);
     return netkv_launch_status();
   }
   const uint32_t lg = group_log2_slots(R);
@@ -471,6 +570,7 @@ extern "C" netkv_status netkv_prefix_match(const void* d_index, uint32_t D,
   char* ws = reinterpret_cast<char*>(d_workspace);
   GroupSlot* tab = reinterpret_cast<GroupSlot*>(ws + L.table);
   uint32_t* leader_of = reinterpret_cast<uint32_t*>(ws + L.leader_of);
+  int32_t* set_of = reinterpret_cast<int32_t*>(ws + L.set_of);
   uint32_t* leaders = reinterpret_cast<uint32_t*>(ws + L.leaders);
   MatchCounters* counters = reinterpret_cast<MatchCounters*>(ws + L.counters);
   NETKV_CUDA_TRY(cudaMemsetAsync(tab, 0, sizeof(GroupSlot) << lg, s));
@@ -478,13 +578,13 @@ extern "C" netkv_status netkv_prefix_match(const void* d_index, uint32_t D,
   const unsigned rgrid = (unsigned)((R + 255) / 256 < 65535u * 16 ? (R + 255) / 256 : 65535u * 16);
   group_insert_kernel<<<rgrid, 256, 0, s>>>(tab, lg, d_chains, d_chain_off, R, d_set_off, n_sets);
   group_resolve_kernel<<<rgrid, 256, 0, s>>>(tab, lg, d_chains, d_chain_off, R, d_set_off, n_sets,
-                                             leader_of, leaders, counters);
+                                             leader_of, set_of, leaders, counters);
   match_leaders_kernel<<<leader_grid(), kMatchBlock, 0, s>>>(
-      index, D, log2_capacity, n_sets, d_chains, d_chain_off, d_set_off, leaders, counters, d_M,
-      d_status);
+      index, D, log2_capacity, n_sets, d_chains, d_chain_off, d_set_off, set_of, leaders, counters,
+      d_M, d_status);
   match_kernel<kMembers><<<grid, kMatchBlock, 0, s>>>(index, D, log2_capacity, n_sets, d_chains,
-                                                      d_chain_off, R, d_set_off, leader_of, d_M,
-                                                      d_status);
+                                                      d_chain_off, R, d_set_off, leader_of, set_of,
+                                                      d_M, d_status);
   return netkv_launch_status();
 }
 

@@ -10,8 +10,13 @@
 // over the per-warp partials (double-buffered so one barrier per arrival suffices).
 // Ties go to the lowest decode rank (line 13).  The decision is written by lane 0 of
 // every warp, so a later departure event is resolved by the same lanes that wrote it.
-// No scratch memory: network, prefix and load terms are combined on the fly from the
-// level bottlenecks UB and the prefix hits M.
+// Events are software-pipelined (up to five events ahead) so that no global load sits
+// on the per-event critical path (see the loop below).
+// Without a workspace the network, prefix and load terms are combined on the fly from
+// the level bottlenecks UB and the prefix hits M.  With a workspace, base_kernel first
+// computes the decision-independent network + prefix term of every (arrival, decode)
+// in parallel, and the greedy only adds the load term: the sequential part of a step
+// shrinks to a load, a capacity test, one multiply-add and the argmin per candidate.
 #include <math.h>
 
 #include "netkv_internal.cuh"
@@ -32,30 +37,100 @@ __device__ __forceinline__ void combine(float& b, uint32_t& i, float& s, float b
   }
 }
 
-__device__ __forceinline__ void warp_argmin(float& b, uint32_t& i, float& s) {
+// (score, index, second) argmin over the lanes of one segment of LPS lanes.
+template <int LPS>
+__device__ __forceinline__ void seg_argmin(float& b, uint32_t& i, float& s, uint32_t mask) {
 #pragma unroll
-  for (int o = 16; o; o >>= 1) {
-    const float b2 = __shfl_xor_sync(0xffffffffu, b, o);
-    const uint32_t i2 = __shfl_xor_sync(0xffffffffu, i, o);
-    const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
+  for (int o = LPS / 2; o; o >>= 1) {
+    const float b2 = __shfl_xor_sync(mask, b, o, LPS);
+    const uint32_t i2 = __shfl_xor_sync(mask, i, o, LPS);
+    const float s2 = __shfl_xor_sync(mask, s, o, LPS);
     combine(b, i, s, b2, i2, s2);
   }
 }
 
-template <int NPT, int BLOCK>
+// Decision-independent part of a candidate's score (Algorithm 1 lines 5-8, Eq. 2, Eq. 3):
+// w_net * (s_eff / min(UB_p[tau], UB_d[tau]) + L_tau) + w_prefix * (l - 16 M) / l.
+__device__ __forceinline__ float base_score(const netkv_weights& w, uint32_t l, uint32_t m,
+                                            float ub_p, float ub_d, float lat_tau, int* status) {
+  uint32_t lam = 16u * m;
+  if (m > l / 16u) {
+    flag_status(status, NETKV_DEV_EDOMAIN);
+    lam = lam < l ? lam : l;
+  }
+  const uint32_t miss_tok = l - lam;
+  const float bb = fminf(ub_p, ub_d);
+  const float s_eff = (float)((int64_t)miss_tok * (int64_t)w.bytes_per_token);
+  const float T = s_eff / bb + lat_tau;
+  const float miss = (float)miss_tok / (float)l;
+  return w.w_net * T + w.w_prefix * miss;
+}
+
+// Base scores of every arrival: base[r][d] = base_score(...) for the stream's weights.
+// No dependence between events, so the arrivals of a stream are spread over the
+// segments (LPS lanes each) of grid.y blocks; each segment strides over one row's
+// decodes.  Departures and invalid events are skipped (the greedy reports them).
+template <int LPS>
+__global__ void __launch_bounds__(256) base_kernel(
+    TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
+    const uint32_t* __restrict__ len, const uint32_t* __restrict__ prefill,
+    const uint32_t* __restrict__ snap, const uint16_t* __restrict__ M,
+    const float* __restrict__ UB, uint32_t n_snap, const uint32_t* __restrict__ events,
+    const uint64_t* __restrict__ event_off, float* __restrict__ base, int* status) {
+  constexpr uint32_t kSegs = 256 / LPS;
+  const uint32_t seg = threadIdx.x / LPS, sl = threadIdx.x % LPS;
+  const uint32_t D = t.D, N = t.N;
+  const float4 lat = make_float4(t.lat[0], t.lat[1], t.lat[2], t.lat[3]);
+  for (uint32_t stream = blockIdx.x; stream < n_streams; stream += gridDim.x) {
+    const netkv_weights w = W[stream];
+    const uint64_t e0 = event_off[stream], e1 = event_off[stream + 1];
+    for (uint64_t e = e0 + (uint64_t)blockIdx.y * kSegs + seg; e < e1;
+         e += (uint64_t)gridDim.y * kSegs) {
+      const uint32_t code = __ldg(events + e);
+      const uint32_t r = code & 0x7fffffffu;
+      if ((code >> 31) || r >= R) continue;
+      const uint32_t l = __ldg(len + r), pr = __ldg(prefill + r), k = __ldg(snap + r);
+      if (pr >= t.P || k >= n_snap || l == 0) continue;
+      const uint32_t pinst = __ldg(t.pre + pr);
+      const uint4 lp = __ldg(t.links + pinst);
+      const float4 ubp = __ldg(reinterpret_cast<const float4*>(UB) + (uint64_t)k * N + pinst);
+      const float* ub_row = UB + (uint64_t)k * N * 4;
+      for (uint32_t d = sl; d < D; d += LPS) {
+        const uint4 ld = __ldg(t.links + __ldg(t.dec + d));
+        const int tau = tier_of(lp, ld);
+        const float ubd = __ldg(ub_row + (uint64_t)ld.x * 4 + tau);
+        const uint32_t m = __ldg(M + (uint64_t)r * D + d);
+        base[(uint64_t)r * D + d] = base_score(w, l, m, pick4(ubp, tau), ubd, pick4(lat, tau), status);
+      }
+    }
+  }
+}
+
+// LPS = lanes per stream.  LPS == 32: one stream per CTA of BLOCK threads.  LPS < 32
+// (BLOCK == 32, NPT == 1, D <= LPS): a warp runs 32 / LPS streams side by side, one per
+// segment of LPS lanes, so that small decode pools still use every lane.
+template <int NPT, int BLOCK, int LPS, bool kBase>
 __global__ void __launch_bounds__(BLOCK) schedule_kernel(
-    TopoArgs t, const netkv_weights* __restrict__ W, uint32_t R, const uint32_t* __restrict__ len,
+    TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
+    const float* __restrict__ base, const uint32_t* __restrict__ len,
     const uint32_t* __restrict__ prefill, const uint32_t* __restrict__ snap,
     const uint16_t* __restrict__ M, const float* __restrict__ UB, uint32_t n_snap,
     const uint32_t* __restrict__ events, const uint64_t* __restrict__ event_off,
     const int64_t* __restrict__ load_init, int32_t* dec, float* __restrict__ best,
     float* __restrict__ second, int64_t* __restrict__ load_final, int* status) {
+  static_assert(LPS == 32 || (BLOCK == 32 && NPT == 1), "packed streams use one warp");
   constexpr int NW = BLOCK / 32;
   __shared__ float s_b[2][NW];
   __shared__ uint32_t s_i[2][NW];
   __shared__ float s_s[2][NW];
-  const uint32_t stream = blockIdx.x;
-  const uint32_t tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  const uint32_t lane_w = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const uint32_t seg = LPS == 32 ? 0u : lane_w / LPS;
+  const uint32_t stream = LPS == 32 ? blockIdx.x : blockIdx.x * (32 / LPS) + seg;
+  if (stream >= n_streams) return;  // whole segments only: never inside a CTA of LPS == 32
+  const uint32_t smask = LPS == 32 ? 0xffffffffu : (((1u << LPS) - 1u) << (seg * LPS));
+  const uint32_t tid = LPS == 32 ? threadIdx.x : lane_w % LPS;  // thread within the stream
+  const uint32_t lane = LPS == 32 ? lane_w : tid;                // lane within the segment
+  const bool lead_thread = tid == 0;
   const uint32_t D = t.D, N = t.N;
   const netkv_weights w = W[stream];
   const float4 lat = make_float4(t.lat[0], t.lat[1], t.lat[2], t.lat[3]);
@@ -76,18 +151,145 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
 
   const uint64_t e0 = event_off[stream], e1 = event_off[stream + 1];
   uint32_t parity = 0;
+
+  // Software pipeline over events.  When event e is processed, its operands were
+  // requested PD iterations earlier: event e+PD+1 gets its level bottlenecks (and, for a
+  // departure, its decision) requested, event e+FD+1 its request fields and prefix hits,
+  // event e+CD+1 its code; every global load is consumed at least one iteration after
+  // it is issued, PD iterations for the level-bottleneck rows that come from DRAM.  The
+  // topology tables read on the way (prefill instance and links) are L1-resident.  A
+  // prefetched decision is superseded when the request's arrival was processed after
+  // the prefetch was issued (the last PD+1 arrivals are kept in registers).
+  constexpr int PD = 1;
+  constexpr int FD = PD + 1;
+  constexpr int CD = PD + 2;
+  const uint32_t kBad = 0xffffffffu;
+  uint32_t cq[CD + 1];                        // event codes, index i = event e+i
+  uint32_t lq[FD + 1], pq[FD + 1], kq[FD + 1], mq[FD + 1][NPT];
+  float4 ubpq[PD + 1];
+  float ubdq[PD + 1][NPT];
+  int tauq[PD + 1][NPT];
+  int32_t decq[PD + 1];
+  uint32_t arr_r[PD + 1];                     // last arrivals processed, newest first
+  int32_t arr_d[PD + 1];
+#pragma unroll
+  for (int i = 0; i <= PD; ++i) {
+    arr_r[i] = kBad;
+    arr_d[i] = -1;
+  }
+
+  // fields of an event (len, prefill, snap, prefix hits); kBad code or bad r gives zeros
+  auto fields = [&](uint32_t code, uint32_t& l, uint32_t& pr, uint32_t& k, uint32_t* m) {
+    l = pr = k = 0;
+#pragma unroll
+    for (int j = 0; j < NPT; ++j) m[j] = 0;
+    if (code == kBad) return;
+    const uint32_t r = code & 0x7fffffffu;
+    if (r >= R) return;
+    l = __ldg(len + r);
+    if (code >> 31) return;
+    pr = __ldg(prefill + r);
+    k = __ldg(snap + r);
+    if (kBase) {  // precomputed network + prefix terms, carried as raw bits
+      const float* b_row = base + (uint64_t)r * D;
+#pragma unroll
+      for (int j = 0; j < NPT; ++j) {
+        const uint32_t d = tid * NPT + j;
+        if (d < D) m[j] = __float_as_uint(__ldg(b_row + d));
+      }
+    } else {
+      const uint16_t* m_row = M + (uint64_t)r * D;
+#pragma unroll
+      for (int j = 0; j < NPT; ++j) {
+        const uint32_t d = tid * NPT + j;
+        if (d < D) m[j] = __ldg(m_row + d);
+      }
+    }
+  };
+  // level bottlenecks (arrival) or decision (departure) of an event whose fields are known
+  auto operands = [&](uint32_t code, uint32_t pr, uint32_t k, float4& ubp, float* ubd, int* tau,
+                      int32_t& dec_pref) {
+    dec_pref = -1;
+    ubp = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int j = 0; j < NPT; ++j) {
+      ubd[j] = 0.0f;
+      tau[j] = 0;
+    }
+    if (code == kBad) return;
+    const uint32_t r = code & 0x7fffffffu;
+    if (r >= R) return;
+    if (code >> 31) {
+      if (lane == 0) dec_pref = *((volatile int32_t*)(dec + r));
+      return;
+    }
+    if (kBase || pr >= t.P || k >= n_snap) return;
+    const uint32_t pinst = __ldg(t.pre + pr);
+    const uint4 lp = __ldg(t.links + pinst);
+    ubp = __ldg(reinterpret_cast<const float4*>(UB) + (uint64_t)k * N + pinst);
+    const float* ub_row = UB + (uint64_t)k * N * 4;
+#pragma unroll
+    for (int j = 0; j < NPT; ++j) {
+      tau[j] = tier_of(lp, ld[j]);
+      if (tid * NPT + j < D) ubd[j] = __ldg(ub_row + (uint64_t)ld[j].x * 4 + tau[j]);
+    }
+  };
+
+#pragma unroll
+  for (int i = 0; i <= CD; ++i) cq[i] = (e0 + i < e1) ? __ldg(events + e0 + i) : kBad;
+#pragma unroll
+  for (int i = 0; i <= FD; ++i) fields(cq[i], lq[i], pq[i], kq[i], mq[i]);
+#pragma unroll
+  for (int i = 0; i <= PD; ++i) operands(cq[i], pq[i], kq[i], ubpq[i], ubdq[i], tauq[i], decq[i]);
+
   for (uint64_t e = e0; e < e1; ++e) {
-    const uint32_t code = __ldg(events + e);
+    // take event e's operands, then advance the pipeline by one event
+    const uint32_t code = cq[0], l = lq[0], pr = pq[0], k = kq[0];
+    const float4 ubp = ubpq[0];
+    float ubd[NPT];
+    int tau[NPT];
+    uint32_t m[NPT];
+#pragma unroll
+    for (int j = 0; j < NPT; ++j) {
+      ubd[j] = ubdq[0][j];
+      tau[j] = tauq[0][j];
+      m[j] = mq[0][j];
+    }
+    const int32_t dec_pref = decq[0];
+#pragma unroll
+    for (int i = 0; i < CD; ++i) cq[i] = cq[i + 1];
+#pragma unroll
+    for (int i = 0; i < FD; ++i) {
+      lq[i] = lq[i + 1];
+      pq[i] = pq[i + 1];
+      kq[i] = kq[i + 1];
+#pragma unroll
+      for (int j = 0; j < NPT; ++j) mq[i][j] = mq[i + 1][j];
+    }
+#pragma unroll
+    for (int i = 0; i < PD; ++i) {
+      ubpq[i] = ubpq[i + 1];
+      decq[i] = decq[i + 1];
+#pragma unroll
+      for (int j = 0; j < NPT; ++j) {
+        ubdq[i][j] = ubdq[i + 1][j];
+        tauq[i][j] = tauq[i + 1][j];
+      }
+    }
+    cq[CD] = (e + 1 + CD < e1) ? __ldg(events + e + 1 + CD) : kBad;
+    fields(cq[FD], lq[FD], pq[FD], kq[FD], mq[FD]);
+    operands(cq[PD], pq[PD], kq[PD], ubpq[PD], ubdq[PD], tauq[PD], decq[PD]);
+
     const uint32_t r = code & 0x7fffffffu;
     if (r >= R) {
-      if (tid == 0) flag_status(status, NETKV_DEV_ERANGE);
+      if (lead_thread) flag_status(status, NETKV_DEV_ERANGE);
       continue;
     }
-    const uint32_t l = __ldg(len + r);
     if (code >> 31) {  // departure: release the tokens of a dispatched request
-      int32_t dd = 0;
-      if (lane == 0) dd = *((volatile int32_t*)(dec + r));
-      dd = __shfl_sync(0xffffffffu, dd, 0);
+      int32_t dd = __shfl_sync(smask, dec_pref, 0, LPS);
+#pragma unroll
+      for (int i = PD; i >= 0; --i)  // decided after the prefetch was issued
+        if (r == arr_r[i]) dd = arr_d[i];
       if (dd >= 0 && (uint32_t)dd < D) {
 #pragma unroll
         for (int j = 0; j < NPT; ++j)
@@ -95,21 +297,22 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
       }
       continue;
     }
-    const uint32_t pr = __ldg(prefill + r), k = __ldg(snap + r);
     if (pr >= t.P || k >= n_snap || l == 0) {
-      if (tid == 0) {
+      if (lead_thread) {
         flag_status(status, l == 0 ? NETKV_DEV_EDOMAIN : NETKV_DEV_ERANGE);
         best[r] = inf;
         second[r] = inf;
       }
-      if (lane == 0) dec[r] = -1;
+      if (lane == 0) *((volatile int32_t*)(dec + r)) = -1;
+#pragma unroll
+      for (int i = PD; i > 0; --i) {
+        arr_r[i] = arr_r[i - 1];
+        arr_d[i] = arr_d[i - 1];
+      }
+      arr_r[0] = r;
+      arr_d[0] = -1;
       continue;
     }
-    const uint32_t pinst = __ldg(t.pre + pr);
-    const uint4 lp = __ldg(t.links + pinst);
-    const float4 ubp = __ldg(reinterpret_cast<const float4*>(UB) + (uint64_t)k * N + pinst);
-    const float* ub_row = UB + (uint64_t)k * N * 4;
-    const uint16_t* m_row = M + (uint64_t)r * D;
 
     float b = inf, s2 = inf;
     uint32_t bi = kNone;
@@ -117,20 +320,15 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
     for (int j = 0; j < NPT; ++j) {
       const uint32_t d = tid * NPT + j;
       if (d < D) {
-        const uint32_t m = __ldg(m_row + d);
-        uint32_t lam = 16u * m;
-        if (m > l / 16u) {
-          flag_status(status, NETKV_DEV_EDOMAIN);
-          lam = lam < l ? lam : l;
-        }
-        const uint32_t miss_tok = l - lam;
         const bool feasible = load[j] + (int64_t)l <= w.cap_tokens;
-        const int tau = tier_of(lp, ld[j]);
-        const float bb = fminf(pick4(ubp, tau), __ldg(ub_row + (uint64_t)ld[j].x * 4 + tau));
-        const float s_eff = (float)((int64_t)miss_tok * (int64_t)w.bytes_per_token);
-        const float T = s_eff / bb + pick4(lat, tau);
-        const float miss = (float)miss_tok / (float)l;
-        const float sc = w.w_net * T + w.w_prefix * miss + w.w_load * (w.theta_s_per_token * (float)load[j]);
+        float sc;
+        if (kBase) {
+          sc = __uint_as_float(m[j]) + w.w_load * (w.theta_s_per_token * (float)load[j]);
+        } else {
+          const float net_prefix = base_score(w, l, m[j], pick4(ubp, tau[j]), ubd[j],
+                                              pick4(lat, tau[j]), status);
+          sc = net_prefix + w.w_load * (w.theta_s_per_token * (float)load[j]);
+        }
         if (feasible) {
           if (bi == kNone || sc < b) {
             s2 = b;
@@ -142,7 +340,7 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
         }
       }
     }
-    warp_argmin(b, bi, s2);
+    seg_argmin<LPS>(b, bi, s2, smask);
     if (NW > 1) {
       if (lane == 0) {
         s_b[parity][wid] = b;
@@ -158,7 +356,7 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
         bi = s_i[parity][lane];
         s2 = s_s[parity][lane];
       }
-      warp_argmin(b, bi, s2);
+      seg_argmin<32>(b, bi, s2, 0xffffffffu);
       parity ^= 1u;
     }
     const int32_t dstar = bi == kNone ? -1 : (int32_t)bi;
@@ -168,10 +366,17 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
         if (tid * NPT + j == (uint32_t)dstar) load[j] += l;
     }
     if (lane == 0) *((volatile int32_t*)(dec + r)) = dstar;
-    if (tid == 0) {
+    if (lead_thread) {
       best[r] = b;
       second[r] = s2;
     }
+#pragma unroll
+    for (int i = PD; i > 0; --i) {
+      arr_r[i] = arr_r[i - 1];
+      arr_d[i] = arr_d[i - 1];
+    }
+    arr_r[0] = r;
+    arr_d[0] = dstar;
   }
 #pragma unroll
   for (int j = 0; j < NPT; ++j) {
@@ -180,27 +385,54 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
   }
 }
 
-template <int NPT, int BLOCK>
+template <int NPT, int BLOCK, int LPS>
 netkv_status launch(const TopoArgs& t, uint32_t n_streams, const netkv_weights* d_w, uint32_t R,
                     const uint32_t* d_len, const uint32_t* d_prefill, const uint32_t* d_snap,
                     const uint16_t* d_M, const float* d_UB, uint32_t n_snap,
                     const uint32_t* d_events, const uint64_t* d_event_off,
                     const int64_t* d_load_init, int32_t* d_dec, float* d_best, float* d_second,
-                    int64_t* d_load_final, int* d_status, cudaStream_t s) {
-  schedule_kernel<NPT, BLOCK><<<n_streams, BLOCK, 0, s>>>(
-      t, d_w, R, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events, d_event_off, d_load_init,
-      d_dec, d_best, d_second, d_load_final, d_status);
+                    int64_t* d_load_final, float* d_base, int* d_status, cudaStream_t s) {
+  const uint32_t per_cta = LPS == 32 ? 1u : 32u / LPS;
+  const unsigned grid = (n_streams + per_cta - 1) / per_cta;
+  if (d_base) {
+    const uint32_t D = t.D;
+    const unsigned gy = n_streams >= 1024u ? 1u : (1024u + n_streams - 1) / n_streams;
+    const dim3 bgrid(n_streams < (1u << 20) ? n_streams : (1u << 20), gy);
+    if (D <= 8)
+      base_kernel<8><<<bgrid, 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,
+                                           d_UB, n_snap, d_events, d_event_off, d_base, d_status);
+    else if (D <= 16)
+      base_kernel<16><<<bgrid, 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,
+                                            d_UB, n_snap, d_events, d_event_off, d_base, d_status);
+    else
+      base_kernel<32><<<bgrid, 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,
+                                            d_UB, n_snap, d_events, d_event_off, d_base, d_status);
+    if (netkv_launch_status() != NETKV_OK) return NETKV_ECUDA;
+    schedule_kernel<NPT, BLOCK, LPS, true><<<grid, BLOCK, 0, s>>>(
+        t, n_streams, d_w, R, d_base, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events,
+        d_event_off, d_load_init, d_dec, d_best, d_second, d_load_final, d_status);
+  } else {
+    schedule_kernel<NPT, BLOCK, LPS, false><<<grid, BLOCK, 0, s>>>(
+        t, n_streams, d_w, R, nullptr, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events,
+        d_event_off, d_load_init, d_dec, d_best, d_second, d_load_final, d_status);
+  }
   return netkv_launch_status();
 }
 
 }  // namespace
+
+extern "C" size_t netkv_schedule_workspace_size(uint32_t R, uint32_t D) {
+  const size_t b = (size_t)R * D * sizeof(float);
+  return (b + 255) / 256 * 256;
+}
 
 extern "C" netkv_status netkv_schedule_streams(
     netkv_topology_t topo, uint32_t n_streams, const netkv_weights* d_w, uint32_t R,
     const uint32_t* d_len, const uint32_t* d_prefill, const uint32_t* d_snap, const uint16_t* d_M,
     const float* d_UB, uint32_t n_snap, const uint32_t* d_events, const uint64_t* d_event_off,
     const int64_t* d_load_init, int32_t* d_dec, float* d_best, float* d_second,
-    int64_t* d_load_final, int* d_status, netkv_stream_t stream) {
+    int64_t* d_load_final, void* d_workspace, size_t workspace_bytes, int* d_status,
+    netkv_stream_t stream) {
   if (!topo || !d_w || !d_event_off || !d_load_final) return NETKV_EINVAL;
   if (n_streams == 0) return NETKV_OK;
   if (n_streams > 0x7fffffffu) return NETKV_EINVAL;
@@ -213,14 +445,20 @@ extern "C" netkv_status netkv_schedule_streams(
   const TopoArgs t = topo_args(topo);
   const uint32_t D = t.D;
   cudaStream_t s = (cudaStream_t)stream;
-#define NETKV_SCHED(NPT, BLOCK)                                                                  \
-  return launch<NPT, BLOCK>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, \
+  if (d_workspace && (!aligned_to(d_workspace, 256) ||
+                      workspace_bytes < netkv_schedule_workspace_size(R, D)))
+    return NETKV_EINVAL;
+  float* d_base = (d_workspace && R > 0) ? reinterpret_cast<float*>(d_workspace) : nullptr;
+#define NETKV_SCHED(NPT, BLOCK, LPS)                                                             \
+  return launch<NPT, BLOCK, LPS>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, \
                             d_events, d_event_off, d_load_init, d_dec, d_best, d_second,       \
-                            d_load_final, d_status, s)
-  if (D <= 32) NETKV_SCHED(1, 32);
-  if (D <= 256) NETKV_SCHED(1, 256);
-  if (D <= 1024) NETKV_SCHED(4, 256);
-  if (D <= 4096) NETKV_SCHED(4, 1024);
+                            d_load_final, d_base, d_status, s)
+  if (D <= 8) NETKV_SCHED(1, 32, 8);
+  if (D <= 16) NETKV_SCHED(1, 32, 16);
+  if (D <= 32) NETKV_SCHED(1, 32, 32);
+  if (D <= 256) NETKV_SCHED(1, 256, 32);
+  if (D <= 1024) NETKV_SCHED(4, 256, 32);
+  if (D <= 4096) NETKV_SCHED(4, 1024, 32);
 #undef NETKV_SCHED
   return NETKV_EINVAL;
 }

@@ -32,8 +32,9 @@ _NAMES = {1: "NETKV_EINVAL", 2: "NETKV_ENOMEM", 3: "NETKV_ECUDA",
 EXPORTS = ("netkv_topology_create", "netkv_topology_destroy", "netkv_topology_query",
            "netkv_oracle_build", "netkv_cache_index_bytes", "netkv_cache_build",
            "netkv_prefix_match_workspace_size",
-           "netkv_prefix_match", "netkv_prefix_match_static", "netkv_schedule_streams",
-           "netkv_version")
+           "netkv_prefix_match", "netkv_prefix_match_static", "netkv_schedule_workspace_size",
+           "netkv_schedule_streams",
+           "netkv_copy_async", "netkv_version")
 
 
 class NetKVError(RuntimeError):
@@ -68,10 +69,14 @@ _lib.netkv_prefix_match_workspace_size.restype = C.c_size_t
 _lib.netkv_prefix_match.argtypes = [_P, _U32, _U32, _U32, _P, _P, _U32, _P, _P, C.c_size_t, _P,
                                     _P, _P]
 _lib.netkv_prefix_match_static.argtypes = [_P, _U32, _U32, _U32, _P, _P, _U32, _P, _P, _P, _P]
+_lib.netkv_schedule_workspace_size.argtypes = [_U32, _U32]
+_lib.netkv_schedule_workspace_size.restype = C.c_size_t
 _lib.netkv_schedule_streams.argtypes = [_P, _U32, _P, _U32, _P, _P, _P, _P, _P, _U32, _P, _P,
-                                        _P, _P, _P, _P, _P, _P, _P]
+                                        _P, _P, _P, _P, _P, _P, C.c_size_t, _P, _P]
+_lib.netkv_copy_async.argtypes = [_P, _P, C.c_size_t, _P]
 for _f in EXPORTS:
-    if _f not in ("netkv_version", "netkv_prefix_match_workspace_size", "netkv_cache_index_bytes"):
+    if _f not in ("netkv_version", "netkv_prefix_match_workspace_size", "netkv_cache_index_bytes",
+                  "netkv_schedule_workspace_size"):
         getattr(_lib, _f).restype = C.c_int
 
 
@@ -186,14 +191,25 @@ def netkv_prefix_match_static(index, D: int, log2_capacity: int, n_sets: int, ch
         int(R), _ptr(set_off), _ptr(M), _ptr(status), _stream(stream)))
 
 
+def netkv_schedule_workspace_size(R: int, D: int) -> int:
+    return int(_lib.netkv_schedule_workspace_size(int(R), int(D)))
+
+
 def netkv_schedule_streams(topo: Topology, n_streams: int, weights, R: int, length, prefill, snap,
                            M, UB, n_snap: int, events, event_off, load_init, dec, best, second,
-                           load_final, status=None, stream=None) -> None:
+                           load_final, status=None, stream=None, workspace=None) -> None:
+    ws_bytes = 0 if workspace is None else int(workspace.numel() * workspace.element_size())
     _check("netkv_schedule_streams", _lib.netkv_schedule_streams(
         topo.handle, int(n_streams), _ptr(weights), int(R), _ptr(length), _ptr(prefill),
         _ptr(snap), _ptr(M), _ptr(UB), int(n_snap), _ptr(events), _ptr(event_off),
-        _ptr(load_init), _ptr(dec), _ptr(best), _ptr(second), _ptr(load_final), _ptr(status),
-        _stream(stream)))
+        _ptr(load_init), _ptr(dec), _ptr(best), _ptr(second), _ptr(load_final), _ptr(workspace),
+        ws_bytes, _ptr(status), _stream(stream)))
+
+
+def netkv_copy_async(dst, src, nbytes: int, stream=None) -> None:
+    """Kernel copy between device and/or pinned host buffers (torch tensors or addresses)."""
+    _check("netkv_copy_async", _lib.netkv_copy_async(_ptr(dst), _ptr(src), int(nbytes),
+                                                     _stream(stream)))
 
 
 def make_weights(w: np.ndarray, theta: float, cap_tokens: int, bytes_per_token: int) -> np.ndarray:

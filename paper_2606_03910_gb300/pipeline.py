@@ -10,7 +10,8 @@ CUDA stream:
 3. ``netkv_schedule_streams`` -> decisions, best/second scores, final loads
 
 ``step_host`` is the same step from host buffers: it copies the step's inputs
-host->device, runs the step and copies the results back, all on the stream.
+host->device (``netkv_copy_async``: SM-driven reads of pinned host memory), runs
+the step and copies the results back, all on the stream.
 Python here only marshals arguments; PyTorch provides device memory.
 """
 from __future__ import annotations
@@ -82,6 +83,18 @@ class Scorer:
         self.status = torch.zeros(1, dtype=torch.int32, device=self.device)
         self.share_prefixes = share_prefixes
         self.workspace = None
+        self.precompute_scores = True
+        self.sched_workspace = None
+
+    def _sched_workspace(self, R: int):
+        """Greedy workspace (base scores of every arrival), grown on demand."""
+        if not self.precompute_scores:
+            return None
+        need = netkv.netkv_schedule_workspace_size(R, self.D)
+        if self.sched_workspace is None or self.sched_workspace.numel() < need:
+            self.sched_workspace = torch.empty(max(need, 256), dtype=torch.uint8,
+                                               device=self.device)
+        return self.sched_workspace
 
     def _workspace(self, R: int):
         """Prefix-match workspace for R requests (grown on demand, reused across steps)."""
@@ -125,7 +138,7 @@ class Scorer:
         netkv.netkv_schedule_streams(self.topo, x.n_streams, x.weights, x.R, x.length, x.prefill,
                                      x.snap, out.M, out.UB, x.n_snap, x.events, x.event_off,
                                      x.load_init, out.dec, out.best, out.second, out.load_final,
-                                     out.status, stream)
+                                     out.status, stream, workspace=self._sched_workspace(x.R))
 
     def step(self, x: StepInputs, out: StepOutputs, stream=None) -> StepOutputs:
         self.oracle_build(x, out, stream)
@@ -138,14 +151,15 @@ class Scorer:
         """Host-buffer step: xh holds pinned host tensors, xd same-shaped device tensors,
         res_h pinned host tensors for dec/best/second/load_final."""
         s = torch.cuda.current_stream() if stream is None else stream
-        with torch.cuda.stream(s):
-            for f in dataclasses.fields(StepInputs):
-                h = getattr(xh, f.name)
-                if isinstance(h, torch.Tensor):
-                    getattr(xd, f.name).copy_(h, non_blocking=True)
-            self.step(xd, out, s)
-            for k in ("dec", "best", "second", "load_final"):
-                res_h[k].copy_(getattr(out, k), non_blocking=True)
+        for f in dataclasses.fields(StepInputs):
+            h = getattr(xh, f.name)
+            if isinstance(h, torch.Tensor):
+                d = getattr(xd, f.name)
+                netkv.netkv_copy_async(d, h, h.numel() * h.element_size(), s)
+        self.step(xd, out, s)
+        for k in ("dec", "best", "second", "load_final"):
+            d = getattr(out, k)
+            netkv.netkv_copy_async(res_h[k], d, d.numel() * d.element_size(), s)
         return out
 
 

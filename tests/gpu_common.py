@@ -61,12 +61,13 @@ def check_stream(w, s, out, cap=None, M_gpu=None):
     Returns the oracle result."""
     from oracle.workload import run_stream
     cap = w.spec.cap_tokens if cap is None else cap
+    import torch
     r0, r1 = int(w.req_off[s]), int(w.req_off[s + 1])
-    dec = host(out.dec)[r0:r1]
+    dec = host(out.dec[r0:r1])
     res = run_stream(w, s, THETA, cap, synth.BYTES_PER_TOKEN_SHARD, hint=dec)
     # prefix hits: bit-exact
     if M_gpu is None:
-        M_gpu = host(out.M).view(np.uint16)[r0:r1]
+        M_gpu = host(out.M[r0:r1]).view(np.uint16)
     np.testing.assert_array_equal(M_gpu, res.M)
     # decisions: exact except near-ties (counted), no unexplained mismatch
     assert res.mismatches == 0, f"stream {s}: {res.mismatches} unexplained decision mismatches"
@@ -74,12 +75,12 @@ def check_stream(w, s, out, cap=None, M_gpu=None):
     # scores of every arrival within 1e-5 relative
     arrivals = w.events[w.event_off[s]:w.event_off[s + 1]]
     arr = (arrivals[(arrivals >> 31) == 0] & 0x7FFFFFFF).astype(np.int64) - r0
-    gb = host(out.best)[r0:r1][arr]
-    gs = host(out.second)[r0:r1][arr]
+    gb = host(out.best[r0:r1])[arr]
+    gs = host(out.second[r0:r1])[arr]
     assert rel_close(gb, res.best[arr]).all(), "best scores differ"
     assert rel_close(gs, res.second[arr]).all(), "second-best scores differ"
-    np.testing.assert_array_equal(host(out.load_final)[s], res.load)
+    np.testing.assert_array_equal(host(out.load_final[s]), res.load)
     # level bottlenecks of the snapshots this stream read
-    UB = host(out.UB)[res.snaps]
+    UB = host(out.UB[torch.from_numpy(res.snaps).to(out.UB.device)])
     assert rel_close(UB, res.UB).all(), "level bottlenecks differ"
     return res

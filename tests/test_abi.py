@@ -50,11 +50,13 @@ def test_version_and_host_validation(lib):
     so = lib._lib
     assert so.netkv_oracle_build(None, None, 1, 1.0, None, None, None, None) == lib.NETKV_EINVAL
     assert so.netkv_cache_build(None, 1, 1, 4, None, None, None, None) == lib.NETKV_EINVAL
-    assert so.netkv_cache_index_bytes(2, 65, 4) == 2 * 2 * 16 * 16
+    assert so.netkv_cache_index_bytes(2, 65, 4) == 2 * 2 * (16 + 16) * 16
     assert so.netkv_prefix_match(None, 1, 4, 1, None, None, 1, None, None, 0, None, None, None) == lib.NETKV_EINVAL
     assert so.netkv_prefix_match_workspace_size(0) == 0
     assert so.netkv_schedule_streams(None, 1, None, 0, None, None, None, None, None, 0, None, None,
-                                     None, None, None, None, None, None, None) == lib.NETKV_EINVAL
+                                     None, None, None, None, None, None, 0, None,
+                                     None) == lib.NETKV_EINVAL
+    assert so.netkv_schedule_workspace_size(10, 8) == 512
     assert so.netkv_topology_destroy(None) == lib.NETKV_EINVAL
 
 

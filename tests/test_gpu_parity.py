@@ -452,3 +452,66 @@ def test_schedule_edge_cases():
         netkv.netkv_schedule_streams(sc.topo, 1, None, x.R, x.length, x.prefill, x.snap, out.M,
                                      out.UB, x.n_snap, x.events, x.event_off, None, out.dec,
                                      out.best, out.second, lf, st)
+
+
+def test_copy_async_host_and_device():
+    """Kernel copies between pinned host and device memory, including ragged tails."""
+    netkv = nk()
+    gen = torch.Generator().manual_seed(3)
+    for nbytes in (16, 17, 4096 + 5, 3 * 2 ** 20 + 15):
+        h = torch.randint(0, 255, (nbytes,), dtype=torch.uint8, generator=gen).pin_memory()
+        d = torch.zeros(nbytes, dtype=torch.uint8, device="cuda")
+        netkv.netkv_copy_async(d, h, nbytes)
+        d2 = torch.zeros_like(d)
+        netkv.netkv_copy_async(d2, d, nbytes)
+        h2 = torch.zeros(nbytes, dtype=torch.uint8).pin_memory()
+        netkv.netkv_copy_async(h2, d2, nbytes)
+        torch.cuda.synchronize()
+        assert torch.equal(d.cpu(), h) and torch.equal(h2, h)
+    netkv.netkv_copy_async(d, h, 0)                      # nothing to do
+    with pytest.raises(netkv.NetKVError):
+        netkv.netkv_copy_async(d[1:], h, 16)             # misaligned destination
+
+
+def test_index_key_order_does_not_change_results():
+    """The same caches listed in chain order (long runs) and shuffled (no runs) give the
+    same prefix hits; chain order is only faster."""
+    from synth import stage
+    netkv = nk()
+    w = synth.make_workload(synth.config0())
+    from tests.gpu_common import index_log2
+    L = index_log2(w)
+    keys = stage.keys(w, 0, w.n_sets)
+    key_off = stage.key_offsets(w, w.n_sets * w.D)
+    ra = stage.request_arrays(w)
+    chains = stage.chains(w)
+    Ms = []
+    for shuffle in (False, True):
+        k = keys.clone()
+        if shuffle:
+            ko = key_off.cpu().numpy()
+            for t in range(w.D):
+                seg = k[ko[t]:ko[t + 1]]
+                k[ko[t]:ko[t + 1]] = seg[torch.randperm(seg.numel(), device=seg.device)]
+        index = torch.empty(netkv.netkv_cache_index_bytes(1, w.D, L) // 8, dtype=torch.int64,
+                            device="cuda")
+        st = torch.zeros(1, dtype=torch.int32, device="cuda")
+        netkv.netkv_cache_build(index, 1, w.D, L, k, key_off, st)
+        M = torch.empty((w.R, w.D), dtype=torch.int16, device="cuda")
+        netkv.netkv_prefix_match(index, w.D, L, 1, chains, ra["chain_off"], w.R, None, M, st)
+        assert status_of(st) == 0
+        Ms.append(M)
+    assert torch.equal(Ms[0], Ms[1])
+    assert (host(Ms[0]).view(np.uint16) > 100).any()
+
+
+@pytest.mark.parametrize("make_spec", [synth.tiny_spec, synth.config0])
+def test_greedy_without_workspace(make_spec):
+    """The fused greedy (no base-score workspace) against the oracle."""
+    w = synth.make_workload(make_spec())
+    sc = make_scorer(w)
+    sc.precompute_scores = False
+    _, x, out = run_gpu(w, sc=sc)
+    assert status_of(out.status) == 0
+    for s in range(w.n_streams):
+        check_stream(w, s, out)
