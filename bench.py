@@ -39,7 +39,7 @@ UNIT = "decisions/s"
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="netkv", choices=["netkv", "reference"])
     ap.add_argument("--streams", type=int, default=4096)
@@ -47,6 +47,8 @@ def parse():
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--table-batch", type=int, default=256)
+    ap.add_argument("--e2e-copy-chains", action="store_true",
+                    help="e2e: copy the chains to the device instead of reading them in place")
     ap.add_argument("--no-share", action="store_true",
                     help="prefix match without the workspace (no grouping of shared prefixes)")
     return ap.parse_args()
@@ -136,6 +138,28 @@ class Clocks:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
+# DRAM traffic per launch from single-pass ncu captures of the full bench workload
+# (dram__bytes_read.sum + dram__bytes_write.sum summed over the call's kernels), keyed by
+# the source file they were taken from; a changed source reports null until re-measured.
+MEASURED_TRAFFIC = {
+    "prefix_match": {"source": "paper_2606_03910_gb300/csrc/prefix.cu",
+                     "sha256_16": "ef30d475712aae66", "bytes": 25_265_000_000},
+}
+
+
+def measured_traffic(kernel: str):
+    import hashlib
+    m = MEASURED_TRAFFIC.get(kernel)
+    if not m:
+        return None
+    try:
+        with open(os.path.join(ROOT, m["source"]), "rb") as f:
+            h = hashlib.sha256(f.read()).hexdigest()[:16]
+    except OSError:
+        return None
+    return m["bytes"] if h == m["sha256_16"] else None
+
+
 def measured_peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -170,7 +194,7 @@ def run_reference(args):
     spec = synth.config1(args.streams)
     w = synth.make_workload(spec)
     theta = float(np.float32(synth.THETA_S_PER_TOKEN))
-    per_step = max(1, min(4, args.streams))
+    per_step = 1
     order = np.random.default_rng(1).permutation(args.streams)
     k = 0
     for _ in range(args.warmup):
@@ -298,30 +322,36 @@ def run_netkv(args):
     decisions = R * world
     value = decisions / (ms / 1e3)
 
-    # ---- roofline of the dominant kernel
+    # ---- roofline of the dominant kernel (the prefix-match call)
     M = out.M.to(torch.int32) & 0xFFFF
     nblk = (x.chain_off[1:] - x.chain_off[:-1]).to(torch.int32)
+    # blocks any exact matcher must examine: each chain up to the first miss of its
+    # last surviving decode (or its end)
+    examined = int(torch.minimum(M.max(dim=1).values + 1, nblk).sum().item())
     probes = int(torch.minimum(M + 1, nblk[:, None]).sum().item())
-    n_arr = R
-    n_dep = R
     algo = {
-        # 8-byte chain block + 8-byte table slot per probe, 2-byte M store per pair
-        "prefix_match": 16 * probes + 2 * R * D,
+        # 8-byte chain block + 16-byte index entry per examined block, 2-byte M store
+        "prefix_match": 24 * examined + 2 * R * D,
         # per snapshot: the utilisation row (L floats), 16-byte UB of every instance
         "oracle_build": x.n_snap * (4 * w.L + 16 * sc.N),
-        # per arrival: event, len/prefill/snap, UB of the prefill, per candidate M (2 B)
-        # and its UB entry (4 B), dec/best/second stores; per departure: event, len, dec
-        "schedule": n_arr * (4 + 12 + 16 + D * 6 + 12) + n_dep * 12 + 2 * 8 * D * x.n_streams,
+        # per arrival: event, len/prefill/snap, per candidate base score (4 B) + the
+        # dec/best/second stores; per departure: event, len, dec
+        "schedule": R * (4 + 12 + 4 * D + 12) + R * 12 + 2 * 8 * D * x.n_streams,
     }
     dom = max(per_kernel, key=per_kernel.get)
     peak, peak_src = measured_peaks()
     achieved = algo[dom] / (per_kernel[dom] / 1e3) / 1e9
+    traffic = measured_traffic(dom)
     roofline = {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
-                "unit": "GB/s", "frac": round(achieved / peak, 4), "traffic": None,
-                "peak_source": peak_src,
+                "unit": "GB/s", "frac": round(achieved / peak, 4),
+                "traffic": traffic, "peak_source": peak_src,
                 "algorithmic_bytes_per_launch": algo[dom],
-                "kernel_ms": {k: round(v, 4) for k, v in per_kernel.items()},
-                "probes_per_launch": probes}
+                "per_unit": "24 B per (request, chain block examined up to its last first miss)"
+                            " + 2 B per M entry",
+                "examined_blocks_per_launch": examined,
+                "survey_probe_bytes_per_launch": 16 * probes + 2 * R * D,
+                "survey_probes_per_launch": probes,
+                "kernel_ms": {k: round(v, 4) for k, v in per_kernel.items()}}
 
     # ---- end to end through the public API with pinned host buffers
     e2e = None
@@ -331,24 +361,33 @@ def run_netkv(args):
                            for f in dataclasses.fields(StepInputs)})
         res_h = {k: torch.empty_like(getattr(out, k), device="cpu").pin_memory()
                  for k in ("dec", "best", "second", "load_final")}
-        h2d = xh.nbytes()
+        zc = () if args.e2e_copy_chains else ("chains",)
+        h2d = sum(int(t.numel() * t.element_size()) for f in dataclasses.fields(StepInputs)
+                  if isinstance((t := getattr(xh, f.name)), torch.Tensor) and f.name not in zc)
+        zc_bytes = sum(int(getattr(xh, n).numel() * getattr(xh, n).element_size()) for n in zc)
         d2h = sum(int(t.numel() * t.element_size()) for t in res_h.values())
         for _ in range(max(1, args.warmup)):
-            sc.step_host(xh, x, out, res_h, stream)
+            sc.step_host(xh, x, out, res_h, stream, zero_copy=zc)
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for _ in range(args.steps):
-            sc.step_host(xh, x, out, res_h, stream)
+            sc.step_host(xh, x, out, res_h, stream, zero_copy=zc)
         e1.record(stream)
         torch.cuda.synchronize()
         ems = e0.elapsed_time(e1) / args.steps
         ems = max_over_ranks(ems, dev)
+        if int(out.status.item()) != 0:
+            raise RuntimeError(f"device status {int(out.status.item())} in the e2e region")
+        if not (torch.equal(res_h["dec"], out.dec.cpu()) and torch.equal(res_h["best"], out.best.cpu())):
+            raise RuntimeError("host-buffer step results differ from the device step")
         e2e = {"value": decisions / (ems / 1e3), "unit": UNIT, "ms_per_step": round(ems, 3),
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-               "gpu_launches_per_step": launches_per_step + n_input_tensors + 4}
+               "host_read_in_place_bytes": zc_bytes,
+               "host_read_in_place": list(zc),
+               "gpu_launches_per_step": launches_per_step + n_input_tensors - len(zc) + 4}
 
     # ---- CPU oracle baseline, rank 0 at N=1 only
     cpu = None

@@ -147,15 +147,21 @@ class Scorer:
         return out
 
     def step_host(self, xh: StepInputs, xd: StepInputs, out: StepOutputs, res_h: dict,
-                  stream=None) -> StepOutputs:
+                  stream=None, zero_copy=()) -> StepOutputs:
         """Host-buffer step: xh holds pinned host tensors, xd same-shaped device tensors,
-        res_h pinned host tensors for dec/best/second/load_final."""
+        res_h pinned host tensors for dec/best/second/load_final.
+
+        Fields named in `zero_copy` are not copied: the kernels read them in place from
+        pinned host memory (unified addressing over NVLink-C2C), so only the parts a step
+        actually touches cross the link (for the chains: blocks up to each first miss)."""
         s = torch.cuda.current_stream() if stream is None else stream
         for f in dataclasses.fields(StepInputs):
             h = getattr(xh, f.name)
-            if isinstance(h, torch.Tensor):
+            if isinstance(h, torch.Tensor) and f.name not in zero_copy:
                 d = getattr(xd, f.name)
                 netkv.netkv_copy_async(d, h, h.numel() * h.element_size(), s)
+        if zero_copy:
+            xd = dataclasses.replace(xd, **{name: getattr(xh, name) for name in zero_copy})
         self.step(xd, out, s)
         for k in ("dec", "best", "second", "load_final"):
             d = getattr(out, k)

@@ -515,3 +515,29 @@ def test_greedy_without_workspace(make_spec):
     assert status_of(out.status) == 0
     for s in range(w.n_streams):
         check_stream(w, s, out)
+
+
+@pytest.mark.parametrize("zero_copy", [(), ("chains",)])
+def test_host_buffer_step(zero_copy):
+    """The step from pinned host buffers (copied, or chains read in place over the
+    host link) gives exactly the device-resident step's results."""
+    import dataclasses
+    from paper_2606_03910_gb300.pipeline import StepInputs
+    w = synth.make_workload(synth.config0())
+    sc, x, out = run_gpu(w)
+    ref = {k: getattr(out, k).clone() for k in ("dec", "best", "second", "load_final", "M")}
+    xh = StepInputs(**{f.name: (getattr(x, f.name).cpu().pin_memory()
+                                if isinstance(getattr(x, f.name), torch.Tensor) else None)
+                       for f in dataclasses.fields(StepInputs)})
+    xd = StepInputs(**{f.name: (torch.empty_like(getattr(x, f.name))
+                                if isinstance(getattr(x, f.name), torch.Tensor) else None)
+                       for f in dataclasses.fields(StepInputs)})
+    out2 = sc.alloc_outputs(x.n_snap, x.R, x.n_streams)
+    res_h = {k: torch.empty_like(getattr(out, k), device="cpu").pin_memory()
+             for k in ("dec", "best", "second", "load_final")}
+    sc.step_host(xh, xd, out2, res_h, zero_copy=zero_copy)
+    torch.cuda.synchronize()
+    assert status_of(out2.status) == 0
+    for k in ("dec", "best", "second", "load_final"):
+        assert torch.equal(res_h[k], ref[k].cpu()), k
+    assert torch.equal(out2.M, ref["M"])
