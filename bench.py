@@ -315,8 +315,8 @@ def run_netkv(args):
 
     R, D = x.R, sc.D
     # level bottlenecks 1; prefix match 4 (group insert, group resolve, leaders, members)
-    # with a workspace or 1 without; greedy 1
-    launches_per_step = 1 + (4 if sc.share_prefixes else 1) + 1
+    # with a workspace or 1 without; greedy 2 (base scores + walk) with a workspace or 1
+    launches_per_step = 1 + (4 if sc.share_prefixes else 1) + (2 if sc.precompute_scores else 1)
     n_input_tensors = sum(1 for f in dataclasses.fields(StepInputs)
                           if isinstance(getattr(x, f.name), torch.Tensor))
     decisions = R * world
