@@ -42,6 +42,10 @@ def parse():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="netkv", choices=["netkv", "reference"])
+    ap.add_argument("--workload", default="replicas", choices=["replicas", "sweep"],
+                    help="replicas: the 4,096-stream scoring step (default); sweep: the "
+                         "oracle-build sweep (1,000 snapshots x 2,048 x 8,192 pairs)")
+    ap.add_argument("--snapshots", type=int, default=1000)
     ap.add_argument("--streams", type=int, default=4096)
     ap.add_argument("--cpu-streams", type=int, default=24)
     ap.add_argument("--no-cpu", action="store_true")
@@ -144,7 +148,16 @@ class Clocks:
 MEASURED_TRAFFIC = {
     "prefix_match": {"source": "paper_2606_03910_gb300/csrc/prefix.cu",
                      "sha256_16": "ef30d475712aae66", "bytes": 25_265_000_000},
+    # the 1,000-snapshot oracle-build sweep (scaled by snapshots for other sizes)
+    "oracle_build": {"source": "paper_2606_03910_gb300/csrc/oracle_build.cu",
+                     "sha256_16": "01d454368c851284", "bytes": 67_156_540_000},
 }
+
+
+def sweep_traffic(n_snap: int):
+    """oracle_build's traffic is one pass over the output, so it scales with the snapshots."""
+    b = measured_traffic("oracle_build")
+    return None if b is None else round(b * n_snap / 1000)
 
 
 def measured_traffic(kernel: str):
@@ -181,6 +194,16 @@ def cpu_oracle_sample(w, streams, theta, cap, bpt):
     return dec, time.perf_counter() - t0
 
 
+def cpu_sweep_sample(spec, w, util, n_snap):
+    """Time the CPU oracle building the full cost matrix of n_snap snapshots; returns
+    (pair costs, seconds)."""
+    import oracle
+    t0 = time.perf_counter()
+    C = oracle.cost_matrix(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, util[:n_snap],
+                           spec.kv_bytes)
+    return C.size, time.perf_counter() - t0
+
+
 def cpu_cores():
     return int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
 
@@ -190,6 +213,8 @@ def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
         return 0
+    if args.workload == "sweep":
+        return run_reference_sweep(args, world)
     import synth
     spec = synth.config1(args.streams)
     w = synth.make_workload(spec)
@@ -217,6 +242,33 @@ def run_reference(args):
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_reference_sweep(args, world):
+    import synth
+    spec = synth.config3(args.snapshots)
+    w = synth.make_workload(spec)
+    util = w.util()
+    for _ in range(args.warmup):
+        cpu_sweep_sample(spec, w, util, 1)
+    pairs, secs = 0, 0.0
+    for _ in range(args.steps):
+        n, t = cpu_sweep_sample(spec, w, util, 1)
+        pairs += n
+        secs += t
+    value = pairs / secs
+    line = {"impl": "reference", "metric": SWEEP_METRIC, "value": value, "unit": SWEEP_UNIT,
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * secs / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": sweep_config(args.snapshots, spec, w),
+            "cpu_baseline": {"value": value, "unit": SWEEP_UNIT, "cores": cpu_cores(),
+                             "kind": "oracle",
+                             "sample": "one snapshot's full cost matrix per step"},
+            "e2e": {"value": value, "unit": SWEEP_UNIT, "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     return 0
@@ -413,10 +465,116 @@ def run_netkv(args):
     return 0
 
 
+SWEEP_METRIC = "pair-costs/sec"
+SWEEP_UNIT = "pair-costs/s"
+
+
+def sweep_config(S, spec, w):
+    P = int((w.role == 0).sum())
+    D = int((w.role == 1).sum())
+    return {"workload": f"oracle-build sweep: {S} snapshots x {P} x {D} pairs, "
+                        f"{w.L}-link rows, Beta(2,5) + 5% hot links, KV {spec.kv_bytes / 1e9:g} GB",
+            "l2": f"output {4 * S * P * D / 1e9:.1f} GB per step, larger than L2"}
+
+
+def run_sweep(args):
+    """Oracle-build sweep: the full fp32 C[s][p][d] rebuilt for every telemetry snapshot."""
+    import torch
+    import synth
+    import __graft_entry__
+    from paper_2606_03910_gb300 import netkv
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    __graft_entry__.build()
+    spec = synth.config3(args.snapshots)
+    spec.seed0 = rank
+    w = synth.make_workload(spec)
+    util_h = w.util()
+    util = torch.from_numpy(util_h).to(dev)
+    topo = netkv.netkv_topology_create(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, w.L)
+    _, P, D, _ = netkv.netkv_topology_query(topo)
+    S = args.snapshots
+    C = torch.empty((S, P, D), dtype=torch.float32, device=dev)
+    st = torch.zeros(1, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    for _ in range(args.warmup):
+        netkv.netkv_oracle_build(topo, util, S, spec.kv_bytes, C, None, st, stream)
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = Clocks(local)
+    clocks.start()
+    t0.record(stream)
+    for _ in range(args.steps):
+        netkv.netkv_oracle_build(topo, util, S, spec.kv_bytes, C, None, st, stream)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, dev)
+    if int(st.item()) != 0:
+        raise RuntimeError(f"device status {int(st.item())}")
+    pairs = S * P * D
+    peak, src = measured_peaks()
+    algo = 4 * pairs + S * w.L * 4
+    achieved = algo / (ms / 1e3) / 1e9
+    e2e = None
+    if not args.no_e2e:
+        # each step takes the snapshots' utilisation rows from pinned host memory, rebuilds
+        # C on the device (where the greedy reads it) and reads the status word back
+        util_p = torch.from_numpy(util_h).pin_memory()
+        st_p = torch.zeros(1, dtype=torch.int32).pin_memory()
+        ub = util_p.numel() * 4
+        for _ in range(args.warmup):
+            netkv.netkv_copy_async(util, util_p, ub, stream)
+            netkv.netkv_oracle_build(topo, util, S, spec.kv_bytes, C, None, st, stream)
+            netkv.netkv_copy_async(st_p, st, 4, stream)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            netkv.netkv_copy_async(util, util_p, ub, stream)
+            netkv.netkv_oracle_build(topo, util, S, spec.kv_bytes, C, None, st, stream)
+            netkv.netkv_copy_async(st_p, st, 4, stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if int(st_p.item()) != 0:
+            raise RuntimeError(f"device status {int(st_p.item())}")
+        ems = max_over_ranks(e0.elapsed_time(e1) / args.steps, dev)
+        e2e = {"value": pairs * world / (ems / 1e3), "unit": SWEEP_UNIT,
+               "ms_per_step": round(ems, 3), "h2d_bytes_per_step": ub, "d2h_bytes_per_step": 4}
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        n, t = cpu_sweep_sample(spec, w, util_h, 8)
+        cpu = {"value": n / t, "unit": SWEEP_UNIT, "cores": cpu_cores(), "kind": "oracle",
+               "sample": "the full cost matrix of the first 8 snapshots"}
+    line = {"metric": SWEEP_METRIC, "value": pairs * world / (ms / 1e3), "unit": SWEEP_UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(ms, 4), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": sweep_config(S, spec, w),
+            "gpu_launches": args.steps, "e2e": e2e,
+            "roofline": {"kernel": "oracle_build", "bound": "hbm", "achieved": round(achieved, 1),
+                         "peak": peak, "unit": "GB/s", "frac": round(achieved / peak, 4),
+                         "traffic": sweep_traffic(S), "peak_source": src,
+                         "algorithmic_bytes_per_launch": algo,
+                         "per_unit": "4 B per pair written + the utilisation rows read"},
+            "cpu_baseline": cpu, "clocks": clk}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
+    if args.workload == "sweep":
+        return run_sweep(args)
     return run_netkv(args)
 
 
