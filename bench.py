@@ -42,7 +42,7 @@ def parse():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="netkv", choices=["netkv", "reference"])
-    ap.add_argument("--workload", default="replicas", choices=["replicas", "sweep"],
+    ap.add_argument("--workload", default="replicas", choices=["replicas", "sweep", "longctx", "cluster"],
                     help="replicas: the 4,096-stream scoring step (default); sweep: the "
                          "oracle-build sweep (1,000 snapshots x 2,048 x 8,192 pairs)")
     ap.add_argument("--snapshots", type=int, default=1000)
@@ -81,12 +81,27 @@ def max_over_ranks(x: float, device=None) -> float:
     return float(t.item())
 
 
-def workload_config(streams, world, extra=None):
-    cfg = {"workload": f"{streams} replicas x 64-GPU four-tier tree (8P+8D, TP=4), "
-                       "1,000 requests/stream, decode caches of 200K blocks",
-           "streams_per_gpu": streams, "requests_per_stream": 1000, "decodes": 8,
-           "prefills": 8, "parallelism": f"replicas{world}",
-           "l2": "inputs larger than L2 (cache index 64 GiB + chains 27 GB per GPU)"}
+def workload_config(streams, world, extra=None, kind="replicas"):
+    if kind == "longctx":
+        cfg = {"workload": "prefix-heavy long context: 1,280-instance 8-ary tree (256P+1,024D), "
+                           "64 streams x 256 requests of 131,072 tokens (8,192-block chains) "
+                           "over 8 shared roots, decode caches of 2^20 blocks, full R x D match",
+               "streams_per_gpu": 64, "requests_per_stream": 256, "decodes": 1024,
+               "prefills": 256, "parallelism": f"replicas{world}",
+               "l2": "inputs larger than L2 (cache index 64 GiB + chains 1 GiB per GPU)"}
+    elif kind == "cluster":
+        cfg = {"workload": "large cluster: 5,120-instance 8-ary tree (1,024P+4,096D), "
+                           "16 streams x 100,000 requests sharing caches of 200K blocks and "
+                           "telemetry",
+               "streams_per_gpu": 16, "requests_per_stream": 100_000, "decodes": 4096,
+               "prefills": 1024, "parallelism": f"replicas{world}",
+               "l2": "inputs larger than L2 (cache index 64 GiB, M 13 GB per GPU)"}
+    else:
+        cfg = {"workload": f"{streams} replicas x 64-GPU four-tier tree (8P+8D, TP=4), "
+                           "1,000 requests/stream, decode caches of 200K blocks",
+               "streams_per_gpu": streams, "requests_per_stream": 1000, "decodes": 8,
+               "prefills": 8, "parallelism": f"replicas{world}",
+               "l2": "inputs larger than L2 (cache index 64 GiB + chains 27 GB per GPU)"}
     if extra:
         cfg.update(extra)
     return cfg
@@ -194,6 +209,45 @@ def cpu_oracle_sample(w, streams, theta, cap, bpt):
     return dec, time.perf_counter() - t0
 
 
+def cpu_oracle_sample_large(w, s, n_req, n_dec, theta, cap, bpt):
+    """Oracle time per decision on a workload whose caches are too large for the oracle's
+    whole-stream sets: its matcher over the first n_req requests of stream s against
+    n_dec evenly spaced decodes (time scaled by D / n_dec), plus its greedy over those
+    requests' events given the generator's constructed hits.  Key and chain generation
+    stay outside the timed parts.  Returns (decisions, seconds)."""
+    import oracle
+    import synth
+    spec = w.spec
+    r0 = int(w.req_off[s])
+    r1 = min(int(w.req_off[s + 1]), r0 + n_req)
+    g = int(synth.request_set(w)[r0])
+    chains = w.chains(r0, r1)
+    chain_off = (w.chain_off[r0:r1 + 1] - w.chain_off[r0]).astype(np.uint64)
+    t_match = 0.0
+    decs = np.unique(np.linspace(0, w.D - 1, n_dec).astype(np.int64))
+    for d in decs:
+        keys = w.keys(g, int(d))
+        t0 = time.perf_counter()
+        oracle.prefix_match_one(keys, chains, chain_off)
+        t_match += time.perf_counter() - t0
+    t_match *= w.D / len(decs)
+    ev = w.events[int(w.event_off[s]):int(w.event_off[s + 1])].astype(np.uint64)
+    rr = (ev & np.uint64(0x7FFFFFFF)).astype(np.int64)
+    keep = rr < r1
+    ev_local = ((rr[keep] - r0).astype(np.uint64) |
+                (ev[keep] & np.uint64(1 << 31))).astype(np.uint32)
+    snaps, snap_local = np.unique(w.snap[r0:r1].astype(np.int64), return_inverse=True)
+    util = np.stack([w.util(int(k), int(k) + 1)[0] for k in snaps])
+    M = synth.constructed_hits(w, r0, r1)
+    wn, wp, wl = (float(v) for v in w.weights[s])
+    t0 = time.perf_counter()
+    oracle.schedule_stream(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, util,
+                           w.length[r0:r1], w.prefill[r0:r1], snap_local.astype(np.uint32), M,
+                           ev_local, wn, wp, wl, theta, cap, bpt)
+    t_greedy = time.perf_counter() - t0
+    return r1 - r0, t_match + t_greedy
+
+
 def cpu_sweep_sample(spec, w, util, n_snap):
     """Time the CPU oracle building the full cost matrix of n_snap snapshots; returns
     (pair costs, seconds)."""
@@ -274,17 +328,32 @@ def run_reference_sweep(args, world):
     return 0
 
 
-def setup_replicas(streams: int, rank: int, dev, table_batch: int = 256):
-    """The benchmark workload on `dev`: generated inputs, the resident cache index and
-    the step's device buffers.  Returns (workload, scorer, step inputs, step outputs)."""
+def workload_spec(kind: str, streams: int, rank: int):
+    """Generator spec of a bench workload; rank k takes its own seeds (weak scaling)."""
+    import synth
+    if kind == "replicas":
+        spec = synth.config1(streams)
+        spec.seed0 = rank_seed0(rank, streams)
+    elif kind == "longctx":
+        spec = synth.config4()
+        spec.seed0 = rank_seed0(rank, spec.n_streams)
+    elif kind == "cluster":
+        spec = synth.config2()
+        spec.seed0 = rank_seed0(rank, spec.n_streams)
+    else:
+        raise ValueError(f"unknown workload {kind!r}")
+    return spec
+
+
+def setup_workload(spec, dev, table_batch: int = 256):
+    """A generated workload on `dev`: its inputs, the resident cache index and the step's
+    device buffers.  Returns (workload, scorer, step inputs, step outputs)."""
     import torch
     import synth
     import synth.device as sdev
     from synth import stage
     from paper_2606_03910_gb300 import netkv
     from paper_2606_03910_gb300.pipeline import Scorer, StepInputs, weights_tensor
-    spec = synth.config1(streams)
-    spec.seed0 = rank_seed0(rank, streams)
     w = synth.make_workload(spec)
     theta = float(np.float32(synth.THETA_S_PER_TOKEN))
     bpt = synth.BYTES_PER_TOKEN_SHARD
@@ -310,6 +379,26 @@ def setup_replicas(streams: int, rank: int, dev, table_batch: int = 256):
     return w, sc, x, out
 
 
+def setup_replicas(streams: int, rank: int, dev, table_batch: int = 256):
+    """The 4,096-replica workload (or `streams` replicas) of rank `rank` on `dev`."""
+    return setup_workload(workload_spec("replicas", streams, rank), dev, table_batch)
+
+
+def match_extent(M, chain_off, rows: int = 1 << 16):
+    """(examined, probes) of a prefix-match result, in row chunks: blocks any exact matcher
+    must examine (each chain up to the first miss of its last surviving decode, or its end)
+    and per-(request, decode) probes up to each first miss."""
+    import torch
+    nblk_all = (chain_off[1:] - chain_off[:-1]).to(torch.int64)
+    examined = probes = 0
+    for r0 in range(0, M.shape[0], rows):
+        m = M[r0:r0 + rows].to(torch.int32) & 0xFFFF
+        nb = nblk_all[r0:r0 + rows]
+        examined += int(torch.minimum(m.max(dim=1).values.to(torch.int64) + 1, nb).sum().item())
+        probes += int(torch.minimum(m.to(torch.int64) + 1, nb[:, None]).sum().item())
+    return examined, probes
+
+
 # ------------------------------------------------------------------ GPU arm
 def run_netkv(args):
     import torch
@@ -324,7 +413,8 @@ def run_netkv(args):
     __graft_entry__.build()
     from paper_2606_03910_gb300.pipeline import StepInputs
 
-    w, sc, x, out = setup_replicas(args.streams, rank, dev, args.table_batch)
+    w, sc, x, out = setup_workload(workload_spec(args.workload, args.streams, rank), dev,
+                                   args.table_batch)
     sc.share_prefixes = not args.no_share
     theta = float(np.float32(synth.THETA_S_PER_TOKEN))
     bpt = synth.BYTES_PER_TOKEN_SHARD
@@ -375,12 +465,7 @@ def run_netkv(args):
     value = decisions / (ms / 1e3)
 
     # ---- roofline of the dominant kernel (the prefix-match call)
-    M = out.M.to(torch.int32) & 0xFFFF
-    nblk = (x.chain_off[1:] - x.chain_off[:-1]).to(torch.int32)
-    # blocks any exact matcher must examine: each chain up to the first miss of its
-    # last surviving decode (or its end)
-    examined = int(torch.minimum(M.max(dim=1).values + 1, nblk).sum().item())
-    probes = int(torch.minimum(M + 1, nblk[:, None]).sum().item())
+    examined, probes = match_extent(out.M, x.chain_off)
     algo = {
         # 8-byte chain block + 16-byte index entry per examined block, 2-byte M store
         "prefix_match": 24 * examined + 2 * R * D,
@@ -393,13 +478,16 @@ def run_netkv(args):
     dom = max(per_kernel, key=per_kernel.get)
     peak, peak_src = measured_peaks()
     achieved = algo[dom] / (per_kernel[dom] / 1e3) / 1e9
-    traffic = measured_traffic(dom)
+    traffic = measured_traffic(dom) if args.workload == "replicas" else None
     roofline = {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
                 "unit": "GB/s", "frac": round(achieved / peak, 4),
                 "traffic": traffic, "peak_source": peak_src,
                 "algorithmic_bytes_per_launch": algo[dom],
-                "per_unit": "24 B per (request, chain block examined up to its last first miss)"
-                            " + 2 B per M entry",
+                "per_unit": {"prefix_match": "24 B per (request, chain block examined up to its "
+                                             "last first miss) + 2 B per M entry",
+                             "oracle_build": "per snapshot: the utilisation row + 16 B per instance",
+                             "schedule": "per arrival: event, request fields, 4 B base score per "
+                                         "candidate, dec/best/second; per departure: event, len, dec"}[dom],
                 "examined_blocks_per_launch": examined,
                 "survey_probe_bytes_per_launch": 16 * probes + 2 * R * D,
                 "survey_probes_per_launch": probes,
@@ -443,20 +531,27 @@ def run_netkv(args):
 
     # ---- CPU oracle baseline, rank 0 at N=1 only
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu:
+    if rank == 0 and world == 1 and not args.no_cpu and args.workload == "replicas":
         sample = np.random.default_rng(0).choice(args.streams, size=min(args.cpu_streams, args.streams),
                                                  replace=False)
         d, secs = cpu_oracle_sample(w, sample, theta, spec.cap_tokens, bpt)
         cpu = {"value": d / secs, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                "sample": f"{len(sample)} of {args.streams} streams, whole streams "
                          f"({d} decisions in {secs:.1f} s)"}
+    elif rank == 0 and world == 1 and not args.no_cpu:
+        n_req, n_dec = (256, 16) if args.workload == "longctx" else (2000, 32)
+        d, secs = cpu_oracle_sample_large(w, 0, n_req, n_dec, theta, spec.cap_tokens, bpt)
+        cpu = {"value": d / secs, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+               "sample": f"first {d} requests of stream 0: the oracle's matcher on {n_dec} "
+                         f"of {w.D} decodes scaled to all, plus its greedy given the "
+                         f"constructed hits ({secs:.1f} s)"}
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
                 "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                 "dtype": "f32", "data": "synthetic",
-                "config": workload_config(args.streams, world),
+                "config": workload_config(args.streams, world, kind=args.workload),
                 "scores_per_s": value * D, "gpu_launches": launches_per_step * args.steps,
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk}
         print(json.dumps(line), flush=True)

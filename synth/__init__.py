@@ -306,6 +306,18 @@ def request_set(w: Workload) -> np.ndarray:
     return out
 
 
+def constructed_hits(w: Workload, r0: int = 0, r1: Optional[int] = None) -> np.ndarray:
+    """[r1 - r0, D] uint16: the leading run of cached blocks each (request, decode) has by
+    construction.  A chain is the first `shared` blocks of its root followed by blocks no
+    cache lists, and decode d of table set g lists the first depth[g, d, k] blocks of every
+    root k, so the run is min(shared_r, depth[g, d, root_r]) (barring a 64-bit collision
+    between independently drawn hashes)."""
+    r1 = w.R if r1 is None else r1
+    g = request_set(w)[r0:r1, None]
+    dep = w.depth.astype(np.uint16)[g, np.arange(w.D)[None, :], w.root[r0:r1, None].astype(np.int64)]
+    return np.minimum(w.shared[r0:r1, None].astype(np.uint16), dep)
+
+
 def chain_of(w: Workload, r: int, n: int, g: int) -> np.ndarray:
     s = int(np.searchsorted(w.req_off, r, side="right") - 1)
     local = r - int(w.req_off[s])

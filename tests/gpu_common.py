@@ -56,15 +56,16 @@ def host(t):
     return t.detach().cpu().numpy()
 
 
-def check_stream(w, s, out, cap=None, M_gpu=None):
+def check_stream(w, s, out, cap=None, M_gpu=None, M_expect=None):
     """Oracle on stream s with the GPU decisions as near-tie hints; asserts parity.
-    Returns the oracle result."""
+    M_expect: the stream's prefix hits for the oracle's greedy where its own per-stream
+    cache sets would not fit (the generator's constructed hits).  Returns the oracle result."""
     from oracle.workload import run_stream
     cap = w.spec.cap_tokens if cap is None else cap
     import torch
     r0, r1 = int(w.req_off[s]), int(w.req_off[s + 1])
     dec = host(out.dec[r0:r1])
-    res = run_stream(w, s, THETA, cap, synth.BYTES_PER_TOKEN_SHARD, hint=dec)
+    res = run_stream(w, s, THETA, cap, synth.BYTES_PER_TOKEN_SHARD, hint=dec, M=M_expect)
     # prefix hits: bit-exact
     if M_gpu is None:
         M_gpu = host(out.M[r0:r1]).view(np.uint16)

@@ -230,6 +230,9 @@ def test_prefix_closed_form_under_generator():
     expect = np.minimum(w.shared[:, None].astype(np.int64),
                         w.depth[set_of, :, :][np.arange(w.R), :, w.root.astype(np.int64)])
     np.testing.assert_array_equal(M.astype(np.int64), expect)
+    # the generator's own statement of it, used where the oracle's sets do not fit
+    np.testing.assert_array_equal(synth.constructed_hits(w), M)
+    np.testing.assert_array_equal(synth.constructed_hits(w, 7, 29), M[7:29])
     assert (M > 0).any() and (M.astype(np.int64) < (w.chain_off[1:] - w.chain_off[:-1])[:, None]).any()
 
 
