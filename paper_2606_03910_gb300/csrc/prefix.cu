@@ -36,6 +36,10 @@
 //     with M_L[d] < lcp the first missing block of L lies inside the common prefix, so
 //     M_r[d] = M_L[d] exactly; otherwise blocks [0, lcp) are all cached and the walk
 //     resumes at block lcp.  The result equals the full match whatever the grouping.
+//   match_members_wide_kernel: the same for pools of more than one decode group, one
+//     warp per member: the common prefix is read once, the member's row is
+//     min(M_L, lcp) elementwise, and block lcp is probed only in the groups where a
+//     leader hit reaches lcp, up to 32 groups at a time.
 #include "netkv_internal.cuh"
 
 namespace {
@@ -195,17 +199,25 @@ __device__ __forceinline__ void miss_all(GroupHits& h, uint32_t lane, unsigned l
 
 // First-miss scan of blocks [start, n) of one chain for the `alive` decodes of a group.
 // Decodes found missing at position p get p; decodes never missing keep their value.
+// start_pos: the run position of block `start` when the caller has already looked it up.
 __device__ __forceinline__ void scan_chain(const IndexSlot* __restrict__ hash, uint32_t log2_cap,
                                            const uint64_t* __restrict__ chain, uint64_t start,
                                            uint64_t n, unsigned long long alive, GroupHits& h,
-                                           uint32_t lane, int* status) {
+                                           uint32_t lane, int* status,
+                                           unsigned long long start_pos = kNotFound) {
   const uint64_t cap = 1ull << log2_cap;
   const RunEntry* __restrict__ run = reinterpret_cast<const RunEntry*>(hash + cap);
   uint64_t p = start;
   uint64_t seg_run = 0, seg_p = 0;  // run position matched with chain position seg_p
-  bool in_run = false;
+  bool in_run = false, fresh = false;
+  if (start_pos != kNotFound) {
+    seg_run = start_pos;
+    seg_p = start;
+    in_run = fresh = true;
+  }
   while (p < n && alive) {
-    const bool looked_up = !in_run;
+    const bool looked_up = !in_run || fresh;
+    fresh = false;
     if (!in_run) {  // locate block p in the hash table
       const uint64_t key = __ldg(chain + p);
       unsigned long long pos = kNotFound;
@@ -473,6 +485,160 @@ __global__ void __launch_bounds__(kMatchBlock) match_kernel(
   }
 }
 
+// Member pass for pools of several decode groups: one warp per member.  With
+// lcp = |common prefix of h_r and h_L| capped at min(n_r, n_L, max_d M_L[d] + 1), every
+// decode has M_r[d] = min(M_L[d], lcp) unless M_L[d] >= lcp and block lcp of h_r is
+// cached on d.  So the member's row is one elementwise pass over the leader's row (16
+// bytes a lane when the rows are 16-byte aligned), and block lcp is then probed in the
+// groups where some leader hit reaches lcp, up to 32 groups at once with one lane per
+// group; a group whose probe finds the block is walked again by the whole warp.
+__global__ void __launch_bounds__(kMatchBlock) match_members_wide_kernel(
+    const void* __restrict__ index, uint32_t D, uint32_t log2_cap, uint32_t n_sets,
+    const uint64_t* __restrict__ chains, const uint64_t* __restrict__ chain_off, uint32_t R,
+    const uint32_t* __restrict__ set_off, const uint32_t* __restrict__ leader_of,
+    const int32_t* __restrict__ set_of, uint16_t* __restrict__ M, int* status) {
+  const uint32_t lane = threadIdx.x & 31;
+  const uint64_t warp = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const uint64_t n_warps = ((uint64_t)gridDim.x * blockDim.x) >> 5;
+  const uint32_t n_dgroups = (D + kGroup - 1) / kGroup;
+  const bool vec = (D % 8u == 0) && ((reinterpret_cast<uintptr_t>(M) & 15u) == 0);
+  const uint32_t n8 = D / 8u;  // 16-byte chunks of a row (vector form)
+
+  for (uint64_t rr = warp; rr < R; rr += n_warps) {
+    const uint32_t r = (uint32_t)rr;
+    const uint32_t lead = __ldg(leader_of + r);
+    if (lead == r) continue;  // leaders were matched by the leader pass
+    const uint64_t row = (uint64_t)r * D;
+    int32_t set;
+    uint64_t c0, n;
+    if (!chain_extent(chain_off, set_off, n_sets, set_of, r, lane, status, set, c0, n)) {
+      const GroupHits z = {0u, 0u};
+      for (uint32_t q = 0; q < n_dgroups; ++q)
+        store_hits(M, row, q * kGroup, min(kGroup, D - q * kGroup), lane, z);
+      continue;
+    }
+    const uint64_t l0 = __ldg(chain_off + lead);
+    const uint64_t nl = min(__ldg(chain_off + lead + 1) - l0, (uint64_t)65535);
+    const uint64_t* __restrict__ own = chains + c0;
+    const uint64_t* __restrict__ lch = chains + l0;
+    const uint16_t* __restrict__ ml = M + (uint64_t)lead * D;
+    uint16_t* __restrict__ mr = M + row;
+
+    // the leader's largest hit
+    uint32_t mmax = 0;
+    if (vec) {
+      for (uint32_t c = lane; c < n8; c += 32) {
+        const uint4 v = __ldg(reinterpret_cast<const uint4*>(ml) + c);
+        const uint32_t m2 = __vmaxu2(__vmaxu2(v.x, v.y), __vmaxu2(v.z, v.w));
+        mmax = max(mmax, max(m2 & 0xffffu, m2 >> 16));
+      }
+    } else {
+      for (uint32_t d = lane; d < D; d += 32) mmax = max(mmax, (uint32_t)__ldg(ml + d));
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1) mmax = max(mmax, __shfl_xor_sync(0xffffffffu, mmax, o));
+
+    // common prefix with the leader, capped, 128 blocks a step
+    const uint64_t cap = min(n, min(nl, (uint64_t)mmax + 1));
+    uint64_t lcp = cap;
+    for (uint64_t base = 0; base < cap; base += 128) {
+      uint64_t a[4], b[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint64_t i = base + 32 * k + lane;
+        a[k] = i < cap ? __ldg(own + i) : 0ull;
+        b[k] = i < cap ? __ldg(lch + i) : 0ull;
+      }
+      uint64_t found = cap;
+#pragma unroll
+      for (int k = 3; k >= 0; --k) {
+        const uint32_t diff = __ballot_sync(0xffffffffu, a[k] != b[k]);
+        if (diff) found = base + 32 * k + (uint64_t)(__ffs(diff) - 1);
+      }
+      if (found < cap) {
+        lcp = found;
+        break;
+      }
+    }
+    const bool probe = lcp < n;  // decodes with M_L >= lcp may hit block lcp
+
+    uint32_t pend_q = 0;  // lane j: the j-th group waiting for its probe of block lcp
+    uint32_t n_pend = 0;
+    auto flush = [&]() {
+      __syncwarp();
+      unsigned long long pos = kNotFound;
+      if (lane < n_pend) {
+        const uint64_t key = __ldg(own + lcp);
+        if (key == 0ull) flag_status(status, NETKV_DEV_EDOMAIN);
+        else pos = lookup(index_hash(index, (uint64_t)set * n_dgroups + pend_q, log2_cap), key,
+                          log2_cap, status);
+      }
+      uint32_t hit = __ballot_sync(0xffffffffu, lane < n_pend && pos != kNotFound);
+      while (hit) {
+        const uint32_t j = __ffs(hit) - 1;
+        hit &= hit - 1;
+        const uint32_t q = __shfl_sync(0xffffffffu, pend_q, j);
+        const unsigned long long pj = __shfl_sync(0xffffffffu, pos, j);
+        const uint32_t q0 = q * kGroup, ng = min(kGroup, D - q0);
+        const uint32_t mlo = lane < ng ? (uint32_t)__ldg(ml + q0 + lane) : 0u;
+        const uint32_t mhi = lane + 32 < ng ? (uint32_t)__ldg(ml + q0 + lane + 32) : 0u;
+        GroupHits h;
+        h.lo = (uint64_t)mlo < lcp ? mlo : (uint32_t)n;
+        h.hi = (uint64_t)mhi < lcp ? mhi : (uint32_t)n;
+        const uint32_t alo = __ballot_sync(0xffffffffu, lane < ng && (uint64_t)mlo >= lcp);
+        const uint32_t ahi = __ballot_sync(0xffffffffu, lane + 32 < ng && (uint64_t)mhi >= lcp);
+        const unsigned long long alive = (unsigned long long)alo | ((unsigned long long)ahi << 32);
+        scan_chain(index_hash(index, (uint64_t)set * n_dgroups + q, log2_cap), log2_cap, own, lcp,
+                   n, alive, h, lane, status, pj);
+        store_hits(M, row, q0, ng, lane, h);
+      }
+      n_pend = 0;
+    };
+    auto pend = [&](uint32_t q) {
+      if (lane == n_pend) pend_q = q;
+      if (++n_pend == 32) flush();
+    };
+
+    // M_r = min(M_L, lcp); note the groups where a leader hit reaches lcp
+    const uint32_t lcp_u = (uint32_t)lcp;
+    if (vec) {
+      const uint32_t lcp2 = lcp_u | (lcp_u << 16);
+      for (uint32_t c0v = 0; c0v < n8; c0v += 32) {
+        const uint32_t c = c0v + lane;
+        bool reach = false;
+        if (c < n8) {
+          uint4 v = __ldg(reinterpret_cast<const uint4*>(ml) + c);
+          const uint32_t m2 = __vmaxu2(__vmaxu2(v.x, v.y), __vmaxu2(v.z, v.w));
+          reach = max(m2 & 0xffffu, m2 >> 16) >= lcp_u;
+          v.x = __vminu2(v.x, lcp2);
+          v.y = __vminu2(v.y, lcp2);
+          v.z = __vminu2(v.z, lcp2);
+          v.w = __vminu2(v.w, lcp2);
+          reinterpret_cast<uint4*>(mr)[c] = v;
+        }
+        // 8 chunks per group: lanes 8k .. 8k+7 hold group c0v / 8 + k
+        const uint32_t fb = __ballot_sync(0xffffffffu, probe && reach);
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          if ((fb >> (8 * k)) & 0xffu) pend(c0v / 8u + (uint32_t)k);
+      }
+    } else {
+      for (uint32_t q = 0; q < n_dgroups; ++q) {
+        const uint32_t q0 = q * kGroup, ng = min(kGroup, D - q0);
+        const uint32_t mlo = lane < ng ? (uint32_t)__ldg(ml + q0 + lane) : 0u;
+        const uint32_t mhi = lane + 32 < ng ? (uint32_t)__ldg(ml + q0 + lane + 32) : 0u;
+        GroupHits h;
+        h.lo = min(mlo, lcp_u);
+        h.hi = min(mhi, lcp_u);
+        store_hits(M, row, q0, ng, lane, h);
+        const bool reach = (lane < ng && mlo >= lcp_u) || (lane + 32 < ng && mhi >= lcp_u);
+        if (__any_sync(0xffffffffu, probe && reach)) pend(q);
+      }
+    }
+    if (n_pend) flush();
+  }
+}
+
 uint32_t group_log2_slots(uint32_t R) {
   uint32_t l = 1;
   while ((1ull << l) < 2ull * R) ++l;
@@ -582,9 +748,17 @@ extern "C" netkv_status netkv_prefix_match(const void* d_index, uint32_t D,
   match_leaders_kernel<<<leader_grid(), kMatchBlock, 0, s>>>(
       index, D, log2_capacity, n_sets, d_chains, d_chain_off, d_set_off, set_of, leaders, counters,
       d_M, d_status);
-  match_kernel<kMembers><<<grid, kMatchBlock, 0, s>>>(index, D, log2_capacity, n_sets, d_chains,
-                                                      d_chain_off, R, d_set_off, leader_of, set_of,
-                                                      d_M, d_status);
+  if (D <= kGroup) {
+    match_kernel<kMembers><<<grid, kMatchBlock, 0, s>>>(index, D, log2_capacity, n_sets, d_chains,
+                                                        d_chain_off, R, d_set_off, leader_of,
+                                                        set_of, d_M, d_status);
+  } else {
+    const uint64_t mblocks = ((uint64_t)R + warps_per_block - 1) / warps_per_block;
+    const unsigned mgrid = (unsigned)(mblocks < (1u << 24) ? mblocks : (1u << 24));
+    match_members_wide_kernel<<<mgrid, kMatchBlock, 0, s>>>(index, D, log2_capacity, n_sets,
+                                                            d_chains, d_chain_off, R, d_set_off,
+                                                            leader_of, set_of, d_M, d_status);
+  }
   return netkv_launch_status();
 }
 

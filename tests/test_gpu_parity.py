@@ -252,6 +252,58 @@ def test_prefix_match_shared_prefixes():
     assert (Mo > 50).mean() > 0.2
 
 
+@pytest.mark.parametrize("D", [65, 200, 2112, 2113])
+def test_prefix_match_shared_prefixes_wide(D):
+    """Pools of several 64-decode groups (ragged last group; 33 and 34 groups at D = 2112
+    and 2113, more than one warp of pending probes, in the 16-byte row form and the
+    scalar one): trie-shaped requests with duplicates and prefixes
+    of other chains; caches hold root prefixes with holes and, on some decodes, the first
+    blocks of request chains, so members resume past the leader and find blocks there."""
+    rng = np.random.default_rng(D)
+    set_sizes = [40, 1, 25]
+    roots = [rng.integers(1, 2 ** 63, 300, dtype=np.int64).astype(np.uint64) for _ in range(3)]
+    chains_list = []
+    for g, sz in enumerate(set_sizes):
+        for i in range(sz):
+            kind = rng.integers(0, 6)
+            root = roots[rng.integers(0, 3)]
+            if kind == 0:
+                c = np.zeros(0, np.uint64)
+            elif kind == 1 and chains_list:
+                c = chains_list[int(rng.integers(0, len(chains_list)))].copy()
+            elif kind == 2 and chains_list:
+                c0 = chains_list[int(rng.integers(0, len(chains_list)))]
+                c = c0[:int(rng.integers(0, len(c0) + 1))].copy()
+            else:
+                k = int(rng.integers(0, 301))
+                tail = rng.integers(1, 2 ** 63, int(rng.integers(0, 40)), dtype=np.int64).astype(np.uint64)
+                c = np.concatenate([root[:k], tail])
+            chains_list.append(c)
+    caches = []
+    r0 = 0
+    for g, sz in enumerate(set_sizes):
+        members = chains_list[r0:r0 + sz]
+        r0 += sz
+        cg = []
+        for d in range(D):
+            ks = set(int(x) for x in rng.integers(1, 2 ** 63, 8, dtype=np.int64))
+            for root in roots:
+                depth = int(rng.integers(0, 301))
+                keep = root[:depth]
+                if rng.random() < 0.3 and depth > 10:
+                    keep = np.delete(keep, int(rng.integers(0, depth)))
+                ks.update(int(x) for x in keep)
+            if rng.random() < 0.2:                     # leading blocks of a few whole chains
+                for c in (members[int(j)] for j in rng.integers(0, sz, 2)):
+                    ks.update(int(x) for x in c[:int(rng.integers(0, len(c) + 1))])
+            cg.append(sorted(ks))
+        caches.append(cg)
+    M, Mo, s, _ = _prefix_case(chains_list, caches, D, set_sizes)
+    assert s == 0
+    np.testing.assert_array_equal(M, Mo)
+    assert (Mo > 20).mean() > 0.1
+
+
 def test_prefix_match_workspace_checks():
     netkv = nk()
     tables = torch.zeros(netkv.netkv_cache_index_bytes(1, 4, 4) // 8, dtype=torch.int64,
