@@ -106,6 +106,100 @@ __global__ void __launch_bounds__(256) base_kernel(
   }
 }
 
+// Base scores for pools of more than 32 decodes.  A block takes one chunk of 256 * NPT
+// decodes of one stream; each thread owns NPT consecutive decodes, whose links it loads
+// once, and walks the arrivals given to the block (every grid.y-th event of the stream).
+// An arrival's request fields and the thread's NPT prefix hits are loaded one arrival
+// ahead, so the per-arrival chain of dependent loads overlaps the previous arrival's
+// scoring; prefix hits are read 8 bytes and scores written 16 bytes at a time when the
+// rows allow it.
+template <int NPT>
+__global__ void __launch_bounds__(256) base_wide_kernel(
+    TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
+    const uint32_t* __restrict__ len, const uint32_t* __restrict__ prefill,
+    const uint32_t* __restrict__ snap, const uint16_t* __restrict__ M,
+    const float* __restrict__ UB, uint32_t n_snap, const uint32_t* __restrict__ events,
+    const uint64_t* __restrict__ event_off, float* __restrict__ base, int* status) {
+  constexpr uint32_t kChunk = 256u * NPT;
+  constexpr uint32_t kBad = 0xffffffffu;
+  const uint32_t D = t.D, N = t.N;
+  const uint32_t n_chunks = (D + kChunk - 1) / kChunk;
+  const bool vec = NPT == 4 && (D % 4u == 0) && ((reinterpret_cast<uintptr_t>(M) & 7u) == 0) &&
+                   ((reinterpret_cast<uintptr_t>(base) & 15u) == 0);
+  const float4 lat = make_float4(t.lat[0], t.lat[1], t.lat[2], t.lat[3]);
+  for (uint64_t sc = blockIdx.x; sc < (uint64_t)n_streams * n_chunks; sc += gridDim.x) {
+    const uint32_t stream = (uint32_t)(sc / n_chunks);
+    const uint32_t d0 = (uint32_t)(sc % n_chunks) * kChunk + threadIdx.x * NPT;
+    uint4 ld[NPT];
+#pragma unroll
+    for (int j = 0; j < NPT; ++j)
+      ld[j] = d0 + j < D ? __ldg(t.links + __ldg(t.dec + d0 + j)) : make_uint4(0, 0, 0, 0);
+    const netkv_weights w = W[stream];
+    const uint64_t e0 = event_off[stream], e1 = event_off[stream + 1];
+
+    // request fields of an event: kBad r for departures and events to skip
+    auto fields = [&](uint64_t e, uint32_t& r, uint32_t& l, uint32_t& pr, uint32_t& k,
+                      uint32_t* m) {
+      r = kBad;
+      if (e >= e1) return;
+      const uint32_t code = __ldg(events + e);
+      const uint32_t rr = code & 0x7fffffffu;
+      if ((code >> 31) || rr >= R) return;
+      l = __ldg(len + rr);
+      pr = __ldg(prefill + rr);
+      k = __ldg(snap + rr);
+      if (pr >= t.P || k >= n_snap || l == 0) return;
+      r = rr;
+      const uint16_t* mrow = M + (uint64_t)rr * D + d0;
+      if (vec) {
+        if (d0 < D) {
+          const uint2 v = __ldg(reinterpret_cast<const uint2*>(mrow));
+          m[0] = v.x & 0xffffu;
+          m[1] = v.x >> 16;
+          m[2] = v.y & 0xffffu;
+          m[3] = v.y >> 16;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < NPT; ++j) m[j] = d0 + j < D ? (uint32_t)__ldg(mrow + j) : 0u;
+      }
+    };
+
+    uint32_t nr, nl = 0, npr = 0, nk = 0, nm[NPT];
+#pragma unroll
+    for (int j = 0; j < NPT; ++j) nm[j] = 0;
+    uint64_t e = e0 + blockIdx.y;
+    fields(e, nr, nl, npr, nk, nm);
+    for (; e < e1; e += gridDim.y) {
+      const uint32_t r = nr, l = nl, pr = npr, k = nk;
+      uint32_t m[NPT];
+#pragma unroll
+      for (int j = 0; j < NPT; ++j) m[j] = nm[j];
+      fields(e + gridDim.y, nr, nl, npr, nk, nm);
+      if (r == kBad) continue;
+      const uint32_t pinst = __ldg(t.pre + pr);
+      const uint4 lp = __ldg(t.links + pinst);
+      const float4 ubp = __ldg(reinterpret_cast<const float4*>(UB) + (uint64_t)k * N + pinst);
+      const float* ub_row = UB + (uint64_t)k * N * 4;
+      float out[NPT];
+#pragma unroll
+      for (int j = 0; j < NPT; ++j) {
+        const int tau = tier_of(lp, ld[j]);
+        const float ubd = d0 + j < D ? __ldg(ub_row + (uint64_t)ld[j].x * 4 + tau) : 1.0f;
+        out[j] = base_score(w, l, m[j], pick4(ubp, tau), ubd, pick4(lat, tau), status);
+      }
+      float* brow = base + (uint64_t)r * D + d0;
+      if (vec) {
+        if (d0 < D) *reinterpret_cast<float4*>(brow) = make_float4(out[0], out[1], out[2], out[3]);
+      } else {
+#pragma unroll
+        for (int j = 0; j < NPT; ++j)
+          if (d0 + j < D) brow[j] = out[j];
+      }
+    }
+  }
+}
+
 // LPS = lanes per stream.  LPS == 32: one stream per CTA of BLOCK threads.  LPS < 32
 // (BLOCK == 32, NPT == 1, D <= LPS): a warp runs 32 / LPS streams side by side, one per
 // segment of LPS lanes, so that small decode pools still use every lane.
@@ -385,6 +479,318 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
   }
 }
 
+// ---- staged greedy: one CTA per stream with precomputed base scores ----------------
+// Everything an event needs is copied into shared memory with cp.async STAGES events
+// before the event is processed: each thread copies its own NPT base scores of an
+// arrival's row, and lane 0 of each warp copies the event's request fields (length,
+// prefill rank, snapshot and, for a departure, the decision recorded so far) into a
+// record slot private to its warp.  A thread waits only for its own copies, and a warp
+// reads its record after a warp barrier, so the ring needs no block barrier; the one
+// block barrier per arrival is the argmin's.  A departure's decision may have been made
+// after its record was copied: each warp keeps the last kRing arrivals' decisions.
+// Event codes come from a shared two-chunk circular buffer (a chunk is BLOCK events,
+// one per thread), refilled a chunk ahead with two block barriers per chunk.
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+  const unsigned sa = (unsigned)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(sa), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async4(void* smem, const void* gmem) {
+  const unsigned sa = (unsigned)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(sa), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;\n" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
+
+constexpr int kRing = 16;  // arrivals remembered per warp (>= STAGES + 1)
+
+// Order-preserving 32-bit keys of fp32 scores, so that warp-wide redux minima give the
+// (score, rank) argmin; kNoKey (above every float's key) stands for "no candidate".
+constexpr uint32_t kNoKey = 0xffffffffu;
+__device__ __forceinline__ uint32_t score_key(float x) {
+  const uint32_t u = __float_as_uint(__fadd_rn(x, 0.0f));  // -0 and +0 tie, as compared
+  return u ^ ((uint32_t)((int32_t)u >> 31) | 0x80000000u);
+}
+__device__ __forceinline__ float key_score(uint32_t k) {
+  if (k == kNoKey) return __int_as_float(0x7f800000);
+  return __uint_as_float(k ^ ((k >> 31) ? 0x80000000u : 0xffffffffu));
+}
+// Block-free argmin over the 32 lanes of a warp: (best key, its lowest rank, second key),
+// where a lane offers (key, rank, key of its own runner-up).
+__device__ __forceinline__ void warp_argmin_keys(uint32_t& key, uint32_t& rank, uint32_t& key2) {
+  const uint32_t bk = __reduce_min_sync(0xffffffffu, key);
+  const uint32_t br = __reduce_min_sync(0xffffffffu, key == bk ? rank : kNone);
+  // the winning lane offers its runner-up; every other lane its best
+  const uint32_t sk = __reduce_min_sync(0xffffffffu, (key == bk && rank == br) ? key2 : key);
+  key = bk;
+  rank = br;
+  key2 = sk;
+}
+
+template <int NPT, int BLOCK, int STAGES>
+__global__ void __launch_bounds__(BLOCK) schedule_staged_kernel(
+    TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
+    const float* __restrict__ base, const uint32_t* __restrict__ len,
+    const uint32_t* __restrict__ prefill, const uint32_t* __restrict__ snap, uint32_t n_snap,
+    const uint32_t* __restrict__ events, const uint64_t* __restrict__ event_off,
+    const int64_t* __restrict__ load_init, int32_t* dec, float* __restrict__ best,
+    float* __restrict__ second, int64_t* __restrict__ load_final, int* status) {
+  static_assert(kRing >= STAGES + 1 && kRing <= 32, "ring covers the staging distance");
+  static_assert((BLOCK & (BLOCK - 1)) == 0 && STAGES < BLOCK, "code chunks");
+  constexpr int NW = BLOCK / 32;
+  constexpr uint32_t kBad = 0xffffffffu;
+  extern __shared__ __align__(16) float ring[];  // [STAGES][BLOCK * NPT]
+  __shared__ __align__(16) uint32_t rec[NW][STAGES][4];  // length, prefill, snapshot, decision
+  __shared__ uint32_t aring_r[NW][kRing];
+  __shared__ int32_t aring_d[NW][kRing];
+  __shared__ uint32_t s_k[2][NW];
+  __shared__ uint32_t s_i[2][NW];
+  __shared__ uint32_t s_k2[2][NW];
+  __shared__ uint32_t codes[2 * BLOCK];  // event e at (e - e0) mod 2 * BLOCK
+  const uint32_t tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  const uint32_t stream = blockIdx.x;
+  if (stream >= n_streams) return;
+  const uint32_t D = t.D;
+  const bool vec = NPT % 4 == 0 && (D % 4u == 0) && ((reinterpret_cast<uintptr_t>(base) & 15u) == 0);
+  const netkv_weights w = W[stream];
+  const float inf = __int_as_float(0x7f800000);
+
+  // per owned decode: load (active tokens), headroom cap - load clamped to 32 bits (0
+  // for ranks past D) and theta * load, the last two redone only when the load changes
+  int64_t load[NPT];
+  uint32_t hr[NPT];
+  float lt[NPT];
+  auto refresh = [&](int j) {
+    const int64_t h = w.cap_tokens - load[j];
+    hr[j] = tid * NPT + j >= D ? 0u : h <= 0 ? 0u : h >= 0xffffffffll ? 0xffffffffu : (uint32_t)h;
+    lt[j] = w.theta_s_per_token * (float)load[j];
+  };
+#pragma unroll
+  for (int j = 0; j < NPT; ++j) {
+    const uint32_t d = tid * NPT + j;
+    load[j] = (load_init && d < D) ? load_init[(uint64_t)stream * D + d] : 0;
+    refresh(j);
+  }
+  // add `delta` tokens to decode dd: only its owner thread does any work
+  auto adjust = [&](uint32_t dd, int64_t delta) {
+    const uint32_t jj = dd - tid * NPT;
+    if (jj < (uint32_t)NPT) {
+#pragma unroll
+      for (int j = 0; j < NPT; ++j)
+        if (jj == (uint32_t)j) {
+          load[j] += delta;
+          refresh(j);
+        }
+    }
+  };
+  if (lane < (uint32_t)kRing) {
+    aring_r[wid][lane] = kBad;
+    aring_d[wid][lane] = -1;
+  }
+  __syncwarp();
+  const uint64_t e0 = event_off[stream], e1 = event_off[stream + 1];
+
+  auto code_at = [&](uint64_t e) -> uint32_t { return e < e1 ? __ldg(events + e) : kBad; };
+  // copies for one event into slot `slot` (one commit group per event, possibly empty)
+  auto stage = [&](uint32_t code, uint32_t slot) {
+    const uint32_t r = code & 0x7fffffffu;
+    if (code != kBad && r < R) {
+      if (lane == 0) {
+        uint32_t* rc = rec[wid][slot];
+        cp_async4(rc + 0, len + r);
+        if (code >> 31) {
+          cp_async4(rc + 3, dec + r);
+        } else {
+          cp_async4(rc + 1, prefill + r);
+          cp_async4(rc + 2, snap + r);
+        }
+      }
+      if (!(code >> 31)) {
+        const float* src = base + (uint64_t)r * D + tid * NPT;
+        float* dst = ring + (size_t)slot * (BLOCK * NPT) + tid * NPT;
+        if (vec) {
+#pragma unroll
+          for (int j = 0; j < NPT; j += 4)
+            if (tid * NPT + j < D) cp_async16(dst + j, src + j);
+        } else {
+#pragma unroll
+          for (int j = 0; j < NPT; ++j)
+            if (tid * NPT + j < D) cp_async4(dst + j, src + j);
+        }
+      }
+    }
+    cp_async_commit();
+  };
+
+  codes[tid] = code_at(e0 + tid);
+  codes[BLOCK + tid] = code_at(e0 + BLOCK + tid);
+  uint32_t next_code = code_at(e0 + 2 * BLOCK + tid);  // chunk 2, stored when chunk 1 starts
+  __syncthreads();
+  auto code_of = [&](uint64_t e) -> uint32_t {
+    return codes[(uint32_t)((e - e0) & (2 * BLOCK - 1))];
+  };
+#pragma unroll
+  for (int i = 0; i < STAGES; ++i) stage(code_of(e0 + i), (uint32_t)i);
+
+  uint32_t slot = 0, parity = 0, n_arr = 0;
+  for (uint64_t e = e0; e < e1; ++e) {
+    const uint64_t off = e - e0;
+    if (off != 0 && (off & (BLOCK - 1)) == 0) {
+      // chunk k = off / BLOCK starts: chunk k - 1 is done everywhere; chunk k + 1 goes
+      // into its place
+      __syncthreads();
+      codes[(uint32_t)((off - BLOCK) & (2 * BLOCK - 1)) + tid] = next_code;
+      __syncthreads();
+      next_code = code_at(e + 2 * BLOCK + tid);
+    }
+    const uint32_t code = code_of(e);
+    const uint32_t ahead = code_of(e + STAGES);  // its copies go to the slot read here
+    const uint32_t cur = slot;
+    slot = slot + 1 == STAGES ? 0 : slot + 1;
+    cp_async_wait<STAGES - 1>();  // this thread's copies for event e have landed
+    __syncwarp();                  // and lane 0's record is visible to the warp
+
+    const uint32_t r = code & 0x7fffffffu;
+    if (r >= R) {
+      if (tid == 0) flag_status(status, NETKV_DEV_ERANGE);
+      __syncwarp();
+      stage(ahead, cur);
+      continue;
+    }
+    const uint4 f = *reinterpret_cast<const uint4*>(rec[wid][cur]);
+    const uint32_t l = f.x;
+    if (code >> 31) {  // departure: release the tokens of a dispatched request
+      int32_t dd = (int32_t)f.w;
+      const uint32_t hit = __ballot_sync(0xffffffffu, lane < (uint32_t)kRing &&
+                                                          aring_r[wid][lane] == r);
+      if (hit) dd = aring_d[wid][__ffs(hit) - 1];  // decided after the record was copied
+      __syncwarp();
+      stage(ahead, cur);
+      if (dd >= 0 && (uint32_t)dd < D) adjust((uint32_t)dd, -(int64_t)l);
+      continue;
+    }
+    const bool ok = f.y < t.P && f.z < n_snap && l != 0;
+    const uint32_t ra = n_arr;
+    n_arr = n_arr + 1 == (uint32_t)kRing ? 0 : n_arr + 1;
+    if (!ok) {
+      __syncwarp();
+      stage(ahead, cur);
+      if (tid == 0) {
+        flag_status(status, l == 0 ? NETKV_DEV_EDOMAIN : NETKV_DEV_ERANGE);
+        best[r] = inf;
+        second[r] = inf;
+      }
+      if (lane == 0) {
+        *((volatile int32_t*)(dec + r)) = -1;
+        aring_r[wid][ra] = r;
+        aring_d[wid][ra] = -1;
+      }
+      continue;
+    }
+
+    float bs[NPT];
+    const float* src = ring + (size_t)cur * (BLOCK * NPT) + tid * NPT;
+    if (vec) {
+#pragma unroll
+      for (int j = 0; j < NPT; j += 4) {
+        const float4 v = *reinterpret_cast<const float4*>(src + j);
+        bs[j] = v.x;
+        bs[j + 1] = v.y;
+        bs[j + 2] = v.z;
+        bs[j + 3] = v.w;
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < NPT; ++j) bs[j] = src[j];
+    }
+    // (score, rank) argmin with the second-best score, in two independent chains (even
+    // and odd j) merged at the end; candidates are met in rank order within a chain
+    float b = inf, s2 = inf, bo = inf, so = inf;
+    uint32_t bi = kNone, bio = kNone;
+#pragma unroll
+    for (int j = 0; j < NPT; ++j) {
+      const uint32_t d = tid * NPT + j;
+      const bool feasible = l <= hr[j];  // load + l <= cap (l >= 1 here)
+      const float sc = __fmaf_rn(w.w_load, lt[j], bs[j]);
+      float& cb = (j & 1) ? bo : b;
+      float& cs = (j & 1) ? so : s2;
+      uint32_t& ci = (j & 1) ? bio : bi;
+      const bool take = feasible && (ci == kNone || sc < cb);
+      cs = take ? cb : (feasible ? fminf(cs, sc) : cs);
+      cb = take ? sc : cb;
+      ci = take ? d : ci;
+    }
+    if (NPT > 1) combine(b, bi, s2, bo, bio, so);
+    __syncwarp();                // every lane has read the record and its scores
+    stage(ahead, cur);  // before the slot is refilled
+    uint32_t kb = bi == kNone ? kNoKey : score_key(b);
+    uint32_t ks = score_key(s2);
+    warp_argmin_keys(kb, bi, ks);
+    if (NW > 1) {
+      if (lane == 0) {
+        s_k[parity][wid] = kb;
+        s_i[parity][wid] = bi;
+        s_k2[parity][wid] = ks;
+      }
+      __syncthreads();
+      const uint32_t q = lane % NW;  // every lane holds some warp's partial
+      kb = s_k[parity][q];
+      bi = s_i[parity][q];
+      ks = s_k2[parity][q];
+      warp_argmin_keys(kb, bi, ks);
+      parity ^= 1u;
+    }
+    b = key_score(kb);
+    s2 = key_score(ks);
+    const int32_t dstar = kb == kNoKey ? -1 : (int32_t)bi;
+    if (dstar >= 0) adjust((uint32_t)dstar, (int64_t)l);
+    if (lane == 0) {
+      *((volatile int32_t*)(dec + r)) = dstar;
+      aring_r[wid][ra] = r;
+      aring_d[wid][ra] = dstar;
+    }
+    if (tid == 0) {
+      best[r] = b;
+      second[r] = s2;
+    }
+  }
+  cp_async_wait<0>();
+#pragma unroll
+  for (int j = 0; j < NPT; ++j) {
+    const uint32_t d = tid * NPT + j;
+    if (d < D) load_final[(uint64_t)stream * D + d] = load[j];
+  }
+}
+
+constexpr int kStages = 8;
+
+template <int NPT, int BLOCK>
+netkv_status launch_staged(const TopoArgs& t, uint32_t n_streams, const netkv_weights* d_w,
+                           uint32_t R, const uint32_t* d_len, const uint32_t* d_prefill,
+                           const uint32_t* d_snap, uint32_t n_snap, const uint32_t* d_events,
+                           const uint64_t* d_event_off, const int64_t* d_load_init,
+                           int32_t* d_dec, float* d_best, float* d_second,
+                           int64_t* d_load_final, const float* d_base, int* d_status,
+                           cudaStream_t s) {
+  const size_t smem = sizeof(float) * (size_t)kStages * BLOCK * NPT;
+  if (smem > 48u * 1024u) {
+    static bool raised = false;  // the same value every time: a benign race
+    if (!raised) {
+      NETKV_CUDA_TRY(cudaFuncSetAttribute(schedule_staged_kernel<NPT, BLOCK, kStages>,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+      raised = true;
+    }
+  }
+  schedule_staged_kernel<NPT, BLOCK, kStages><<<n_streams, BLOCK, smem, s>>>(
+      t, n_streams, d_w, R, d_base, d_len, d_prefill, d_snap, n_snap, d_events, d_event_off,
+      d_load_init, d_dec, d_best, d_second, d_load_final, d_status);
+  return netkv_launch_status();
+}
+
 template <int NPT, int BLOCK, int LPS>
 netkv_status launch(const TopoArgs& t, uint32_t n_streams, const netkv_weights* d_w, uint32_t R,
                     const uint32_t* d_len, const uint32_t* d_prefill, const uint32_t* d_snap,
@@ -404,13 +810,53 @@ netkv_status launch(const TopoArgs& t, uint32_t n_streams, const netkv_weights* 
     else if (D <= 16)
       base_kernel<16><<<bgrid, 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,
                                             d_UB, n_snap, d_events, d_event_off, d_base, d_status);
-    else
+    else if (D <= 32)
       base_kernel<32><<<bgrid, 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,
                                             d_UB, n_snap, d_events, d_event_off, d_base, d_status);
+    else {
+      // one block per (stream, chunk of decodes) and arrival segment, ~32 blocks per SM
+      int dev = 0, sms = 0;
+      cudaGetDevice(&dev);
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+      const uint32_t chunk = D <= 256 ? 256u : 1024u;
+      const uint64_t gx = (uint64_t)n_streams * ((D + chunk - 1) / chunk);
+      const uint64_t want = (uint64_t)(sms > 0 ? sms : 1) * 32;
+      const unsigned wx = (unsigned)(gx < (1u << 20) ? gx : (1u << 20));
+      const unsigned wy = (unsigned)(gx >= want ? 1 : (want + gx - 1) / gx < 65535 ? (want + gx - 1) / gx : 65535);
+      if (D <= 256)
+        base_wide_kernel<1><<<dim3(wx, wy), 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill,
+                                                         d_snap, d_M, d_UB, n_snap, d_events,
+                                                         d_event_off, d_base, d_status);
+      else
+        base_wide_kernel<4><<<dim3(wx, wy), 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill,
+                                                         d_snap, d_M, d_UB, n_snap, d_events,
+                                                         d_event_off, d_base, d_status);
+    }
     if (netkv_launch_status() != NETKV_OK) return NETKV_ECUDA;
-    schedule_kernel<NPT, BLOCK, LPS, true><<<grid, BLOCK, 0, s>>>(
-        t, n_streams, d_w, R, d_base, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events,
-        d_event_off, d_load_init, d_dec, d_best, d_second, d_load_final, d_status);
+    if (LPS == 32) {
+      // one CTA per stream: the walk is bound by each warp's chain of dependent
+      // instructions per event; 16 warps (4 per scheduler) measured best on 4,096 decodes
+      const uint32_t D = t.D;
+      if (D <= 32) return launch_staged<1, 32>(t, n_streams, d_w, R, d_len, d_prefill, d_snap,
+                                               n_snap, d_events, d_event_off, d_load_init, d_dec,
+                                               d_best, d_second, d_load_final, d_base, d_status, s);
+      if (D <= 256) return launch_staged<1, 256>(t, n_streams, d_w, R, d_len, d_prefill, d_snap,
+                                                 n_snap, d_events, d_event_off, d_load_init, d_dec,
+                                                 d_best, d_second, d_load_final, d_base, d_status, s);
+      if (D <= 1024) return launch_staged<2, 512>(t, n_streams, d_w, R, d_len, d_prefill, d_snap,
+                                                  n_snap, d_events, d_event_off, d_load_init, d_dec,
+                                                  d_best, d_second, d_load_final, d_base, d_status, s);
+      if (D <= 2048) return launch_staged<4, 512>(t, n_streams, d_w, R, d_len, d_prefill, d_snap,
+                                                  n_snap, d_events, d_event_off, d_load_init, d_dec,
+                                                  d_best, d_second, d_load_final, d_base, d_status, s);
+      return launch_staged<8, 512>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, n_snap,
+                                   d_events, d_event_off, d_load_init, d_dec, d_best, d_second,
+                                   d_load_final, d_base, d_status, s);
+    } else {
+      schedule_kernel<NPT, BLOCK, LPS, true><<<grid, BLOCK, 0, s>>>(
+          t, n_streams, d_w, R, d_base, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events,
+          d_event_off, d_load_init, d_dec, d_best, d_second, d_load_final, d_status);
+    }
   } else {
     schedule_kernel<NPT, BLOCK, LPS, false><<<grid, BLOCK, 0, s>>>(
         t, n_streams, d_w, R, nullptr, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events,

@@ -409,7 +409,10 @@ def test_single_stream_64gpu_full():
                                            ((1, 8, 8, 20), "mod5", 1024),  # 256 threads, 4 each
                                            ((3, 5, 7, 11), "alternate", 577),
                                            ((1, 8, 8, 80), "mod5", 4096),  # 1024 threads, 4 each
-                                           ((1, 2, 3, 5), "alternate", 15)])
+                                           ((1, 2, 3, 5), "alternate", 15),
+                                           ((2, 3, 4, 2), "alternate", 24),  # one warp, 1 each
+                                           ((1, 5, 5, 5), "mod5", 100),      # 256 threads, ragged
+                                           ((1, 7, 11, 17), "mod5", 1047)])  # 512 threads, 4 each
 def test_schedule_block_shapes(fanout, rule, D):
     spec = synth.Spec(name="shape", fanout=fanout, role_rule=rule, n_streams=2,
                       requests_per_stream=120, rate_per_s=40.0, len_median=2048.0,
