@@ -135,13 +135,18 @@ __global__ void __launch_bounds__(256) base_wide_kernel(
     for (int j = 0; j < NPT; ++j)
       ld[j] = d0 + j < D ? __ldg(t.links + __ldg(t.dec + d0 + j)) : make_uint4(0, 0, 0, 0);
     const netkv_weights w = W[stream];
+    // a contiguous range of the stream's events, so that consecutive arrivals share
+    // their snapshot's level-bottleneck row in L1
     const uint64_t e0 = event_off[stream], e1 = event_off[stream + 1];
+    const uint64_t span = (e1 - e0 + gridDim.y - 1) / gridDim.y;
+    const uint64_t eb = e0 + blockIdx.y * span;
+    const uint64_t ee = min(e1, eb + span);
 
     // request fields of an event: kBad r for departures and events to skip
     auto fields = [&](uint64_t e, uint32_t& r, uint32_t& l, uint32_t& pr, uint32_t& k,
                       uint32_t* m) {
       r = kBad;
-      if (e >= e1) return;
+      if (e >= ee) return;
       const uint32_t code = __ldg(events + e);
       const uint32_t rr = code & 0x7fffffffu;
       if ((code >> 31) || rr >= R) return;
@@ -153,7 +158,7 @@ __global__ void __launch_bounds__(256) base_wide_kernel(
       const uint16_t* mrow = M + (uint64_t)rr * D + d0;
       if (vec) {
         if (d0 < D) {
-          const uint2 v = __ldg(reinterpret_cast<const uint2*>(mrow));
+          const uint2 v = __ldcs(reinterpret_cast<const uint2*>(mrow));
           m[0] = v.x & 0xffffu;
           m[1] = v.x >> 16;
           m[2] = v.y & 0xffffu;
@@ -161,21 +166,21 @@ __global__ void __launch_bounds__(256) base_wide_kernel(
         }
       } else {
 #pragma unroll
-        for (int j = 0; j < NPT; ++j) m[j] = d0 + j < D ? (uint32_t)__ldg(mrow + j) : 0u;
+        for (int j = 0; j < NPT; ++j) m[j] = d0 + j < D ? (uint32_t)__ldcs(mrow + j) : 0u;
       }
     };
 
     uint32_t nr, nl = 0, npr = 0, nk = 0, nm[NPT];
 #pragma unroll
     for (int j = 0; j < NPT; ++j) nm[j] = 0;
-    uint64_t e = e0 + blockIdx.y;
+    uint64_t e = eb;
     fields(e, nr, nl, npr, nk, nm);
-    for (; e < e1; e += gridDim.y) {
+    for (; e < ee; ++e) {
       const uint32_t r = nr, l = nl, pr = npr, k = nk;
       uint32_t m[NPT];
 #pragma unroll
       for (int j = 0; j < NPT; ++j) m[j] = nm[j];
-      fields(e + gridDim.y, nr, nl, npr, nk, nm);
+      fields(e + 1, nr, nl, npr, nk, nm);
       if (r == kBad) continue;
       const uint32_t pinst = __ldg(t.pre + pr);
       const uint4 lp = __ldg(t.links + pinst);
@@ -190,11 +195,11 @@ __global__ void __launch_bounds__(256) base_wide_kernel(
       }
       float* brow = base + (uint64_t)r * D + d0;
       if (vec) {
-        if (d0 < D) *reinterpret_cast<float4*>(brow) = make_float4(out[0], out[1], out[2], out[3]);
+        if (d0 < D) __stcs(reinterpret_cast<float4*>(brow), make_float4(out[0], out[1], out[2], out[3]));
       } else {
 #pragma unroll
         for (int j = 0; j < NPT; ++j)
-          if (d0 + j < D) brow[j] = out[j];
+          if (d0 + j < D) __stcs(brow + j, out[j]);
       }
     }
   }
