@@ -377,7 +377,7 @@ __device__ __forceinline__ void store_hits(uint16_t* __restrict__ M, uint64_t ro
 
 // Leader pass: one task per (leader, decode group), taken in order from a global counter
 // by whole warps, so long and short chains balance across the GPU.
-__global__ void __launch_bounds__(kMatchBlock) match_leaders_kernel(
+__global__ void __launch_bounds__(kMatchBlock, 8) match_leaders_kernel(
     const void* __restrict__ index, uint32_t D, uint32_t log2_cap, uint32_t n_sets,
     const uint64_t* __restrict__ chains, const uint64_t* __restrict__ chain_off,
     const uint32_t* __restrict__ set_off, const int32_t* __restrict__ set_of,
@@ -410,7 +410,7 @@ __global__ void __launch_bounds__(kMatchBlock) match_leaders_kernel(
 }
 
 template <int kMode>
-__global__ void __launch_bounds__(kMatchBlock) match_kernel(
+__global__ void __launch_bounds__(kMatchBlock, 8) match_kernel(
     const void* __restrict__ index, uint32_t D, uint32_t log2_cap, uint32_t n_sets,
     const uint64_t* __restrict__ chains, const uint64_t* __restrict__ chain_off, uint32_t R,
     const uint32_t* __restrict__ set_off, const uint32_t* __restrict__ leader_of,
@@ -492,7 +492,7 @@ __global__ void __launch_bounds__(kMatchBlock) match_kernel(
 // bytes a lane when the rows are 16-byte aligned), and block lcp is then probed in the
 // groups where some leader hit reaches lcp, up to 32 groups at once with one lane per
 // group; a group whose probe finds the block is walked again by the whole warp.
-__global__ void __launch_bounds__(kMatchBlock) match_members_wide_kernel(
+__global__ void __launch_bounds__(kMatchBlock, 6) match_members_wide_kernel(
     const void* __restrict__ index, uint32_t D, uint32_t log2_cap, uint32_t n_sets,
     const uint64_t* __restrict__ chains, const uint64_t* __restrict__ chain_off, uint32_t R,
     const uint32_t* __restrict__ set_off, const uint32_t* __restrict__ leader_of,
