@@ -67,11 +67,11 @@ __device__ __forceinline__ float base_score(const netkv_weights& w, uint32_t l, 
 }
 
 // Base scores of every arrival: base[r][d] = base_score(...) for the stream's weights.
-// No dependence between events, so the arrivals of a stream are spread over the
-// segments (LPS lanes each) of grid.y blocks; each segment strides over one row's
-// decodes.  Departures and invalid events are skipped (the greedy reports them).
+// No dependence between events, so the events of a stream are split into contiguous
+// ranges over the segments (LPS lanes each) of grid.y blocks; each segment strides over
+// one row's decodes.  Departures and invalid events are skipped (the greedy reports them).
 template <int LPS>
-__global__ void __launch_bounds__(256) base_kernel(
+__global__ void __launch_bounds__(256, 8) base_kernel(
     TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
     const uint32_t* __restrict__ len, const uint32_t* __restrict__ prefill,
     const uint32_t* __restrict__ snap, const uint16_t* __restrict__ M,
@@ -83,10 +83,17 @@ __global__ void __launch_bounds__(256) base_kernel(
   const float4 lat = make_float4(t.lat[0], t.lat[1], t.lat[2], t.lat[3]);
   for (uint32_t stream = blockIdx.x; stream < n_streams; stream += gridDim.x) {
     const netkv_weights w = W[stream];
+    // each segment takes a contiguous range of the stream's events, so consecutive
+    // arrivals share their snapshot's level-bottleneck row in L1
     const uint64_t e0 = event_off[stream], e1 = event_off[stream + 1];
-    for (uint64_t e = e0 + (uint64_t)blockIdx.y * kSegs + seg; e < e1;
-         e += (uint64_t)gridDim.y * kSegs) {
-      const uint32_t code = __ldg(events + e);
+    const uint64_t n_seg = (uint64_t)gridDim.y * kSegs;
+    const uint64_t span = (e1 - e0 + n_seg - 1) / n_seg;
+    const uint64_t eb = e0 + ((uint64_t)blockIdx.y * kSegs + seg) * span;
+    const uint64_t ee = min(e1, eb + span);
+    uint32_t next = eb < ee ? __ldg(events + eb) : 0u;
+    for (uint64_t e = eb; e < ee; ++e) {
+      const uint32_t code = next;
+      if (e + 1 < ee) next = __ldg(events + e + 1);
       const uint32_t r = code & 0x7fffffffu;
       if ((code >> 31) || r >= R) continue;
       const uint32_t l = __ldg(len + r), pr = __ldg(prefill + r), k = __ldg(snap + r);
