@@ -576,17 +576,18 @@ __global__ void __launch_bounds__(BLOCK) schedule_staged_kernel(
   int64_t load[NPT];
   uint32_t hr[NPT];
   float lt[NPT];
+#pragma unroll
+  for (int j = 0; j < NPT; ++j) {
+    const uint32_t d = tid * NPT + j;
+    load[j] = (load_init && d < D) ? load_init[(uint64_t)stream * D + d] : 0;
+  }
   auto refresh = [&](int j) {
     const int64_t h = w.cap_tokens - load[j];
     hr[j] = tid * NPT + j >= D ? 0u : h <= 0 ? 0u : h >= 0xffffffffll ? 0xffffffffu : (uint32_t)h;
     lt[j] = w.theta_s_per_token * (float)load[j];
   };
 #pragma unroll
-  for (int j = 0; j < NPT; ++j) {
-    const uint32_t d = tid * NPT + j;
-    load[j] = (load_init && d < D) ? load_init[(uint64_t)stream * D + d] : 0;
-    refresh(j);
-  }
+  for (int j = 0; j < NPT; ++j) refresh(j);
   // add `delta` tokens to decode dd: only its owner thread does any work
   auto adjust = [&](uint32_t dd, int64_t delta) {
     const uint32_t jj = dd - tid * NPT;
