@@ -162,7 +162,7 @@ class Clocks:
 # the source file they were taken from; a changed source reports null until re-measured.
 MEASURED_TRAFFIC = {
     "prefix_match": {"source": "paper_2606_03910_gb300/csrc/prefix.cu",
-                     "sha256_16": "fcefa147a2eb8929", "bytes": 25_260_000_000},
+                     "sha256_16": "e98bf5d31ac767be", "bytes": 25_613_000_000},
     # the 1,000-snapshot oracle-build sweep (scaled by snapshots for other sizes)
     "oracle_build": {"source": "paper_2606_03910_gb300/csrc/oracle_build.cu",
                      "sha256_16": "01d454368c851284", "bytes": 67_156_540_000},
