@@ -72,6 +72,10 @@ def _declare(l):
     l.oracle_schedule_stream.restype = None
     l.oracle_schedule_stream.argtypes = [P, P, P, P, P, U64, P, P, P, P, P, U64, F64, F64, F64,
                                          F64, I64, U64, P, P, F64, P, P, P, P, P]
+    l.oracle_schedule_stream_inflight.restype = None
+    l.oracle_schedule_stream_inflight.argtypes = [P, P, P, P, P, U64, P, P, P, P, P, P, U64,
+                                                  F64, F64, F64, F64, I64, U64, U32, P, P, P,
+                                                  F64, P, P, P, P, P, P]
 
 
 def _p(a: Optional[np.ndarray]):
@@ -171,9 +175,11 @@ def prefix_match_one(keys, chains, chain_off) -> np.ndarray:
 
 # ------------------------------------------------------------------ greedy
 class StreamResult:
-    def __init__(self, dec, best, second, load, near_ties, mismatches, rejects):
+    def __init__(self, dec, best, second, load, near_ties, mismatches, rejects, xfer_us=None,
+                 xfer_adopted=0, xfer_mismatches=0):
         self.dec, self.best, self.second, self.load = dec, best, second, load
         self.near_ties, self.mismatches, self.rejects = near_ties, mismatches, rejects
+        self.xfer_us, self.xfer_adopted, self.xfer_mismatches = xfer_us, xfer_adopted, xfer_mismatches
 
 
 def schedule_stream(fanout, role, bw, lat, util, length, prefill, snap, M, events,
@@ -204,3 +210,38 @@ def schedule_stream(fanout, role, bw, lat, util, length, prefill, snap, M, event
                                  _p(li), _p(h), float(rel_tol), _p(dec), _p(best), _p(second),
                                  _p(load), _p(counts))
     return StreamResult(dec, best, second, load, int(counts[0]), int(counts[1]), int(counts[2]))
+
+
+def schedule_stream_inflight(fanout, role, bw, lat, util, length, prefill, snap, arrival_us, M,
+                             events, w_net, w_prefix, w_load, theta, cap, bytes_per_token,
+                             inflight_cap, load_init=None, hint=None, xfer_hint=None,
+                             rel_tol=1e-5) -> StreamResult:
+    """Algorithm 1 with self-contention (Eq. 4's n_inflight, Algorithm 1 lines 5 and 14,
+    Sec. IV-C): arrays are indexed by request; arrival_us are the arrival times in
+    microseconds; inflight_cap = 0 turns self-contention off.  xfer_hint: another
+    implementation's transfer times (whole microseconds) to adopt where they differ by at
+    most one.  Returns a StreamResult with xfer_us set."""
+    f, ro = _c(fanout, np.uint32), _c(role, np.uint8)
+    b, la = _c(bw, np.float64), _c(lat, np.float64)
+    u = _c(util, np.float32)
+    ln, pf, sn = _c(length, np.uint32), _c(prefill, np.uint32), _c(snap, np.uint32)
+    ta = _c(arrival_us, np.int64)
+    m = _c(M, np.uint16)
+    ev = _c(events, np.uint32)
+    R = len(ln)
+    D = int((ro == 1).sum())
+    dec = np.full(R, -1, np.int32)
+    best = np.full(R, np.inf); second = np.full(R, np.inf)
+    xfer = np.full(R, -1, np.int32)
+    load = np.zeros(D, np.int64)
+    counts = np.zeros(5, np.int64)
+    li = None if load_init is None else _c(load_init, np.int64)
+    h = None if hint is None else _c(hint, np.int32)
+    xh = None if xfer_hint is None else _c(xfer_hint, np.int32)
+    lib().oracle_schedule_stream_inflight(
+        _p(f), _p(ro), _p(b), _p(la), _p(u), u.shape[1], _p(ln), _p(pf), _p(sn), _p(ta), _p(m),
+        _p(ev), len(ev), float(w_net), float(w_prefix), float(w_load), float(theta), int(cap),
+        int(bytes_per_token), int(inflight_cap), _p(li), _p(h), _p(xh), float(rel_tol), _p(dec),
+        _p(best), _p(second), _p(xfer), _p(load), _p(counts))
+    return StreamResult(dec, best, second, load, int(counts[0]), int(counts[1]), int(counts[2]),
+                        xfer, int(counts[3]), int(counts[4]))

@@ -23,6 +23,12 @@
 //   * Algorithm 1 (Sec. IV-A) as a weighted score: filter by capacity (line 1), reject
 //     when nothing is feasible (line 2), score every candidate (lines 3-11), take the
 //     argmin with the lowest index among equal scores (line 13), then update load.
+//   * Self-contention (Eq. 4's n_inflight, Algorithm 1 lines 5 and 14, Sec. IV-C), in
+//     oracle_schedule_stream_inflight: a per-(prefill, tier) counter divides the
+//     effective bandwidth by 1 + n; a dispatch raises the counter of its tier (saturating
+//     at the cap) and its transfer completes, lowering it again (never below zero), at
+//     the arrival time plus the chosen candidate's transfer time rounded to whole
+//     microseconds.  Completions due at or before an arrival are applied before it.
 //
 // Parity: pinned by the not-gpu tests (worked example of Sec. III-D, closed forms of
 // Eq. 1, the per-tier special case of Eq. 4, brute force on tiny instances,
@@ -31,6 +37,7 @@
 #include <cstdint>
 #include <cstring>
 #include <limits>
+#include <queue>
 #include <unordered_set>
 #include <vector>
 
@@ -318,6 +325,109 @@ void oracle_schedule_stream(const uint32_t* fanout, const uint8_t* role, const d
     best[r] = b1;
     second[r] = b2;
     if (chosen >= 0) load[chosen] += l;
+  }
+  for (uint64_t d = 0; d < D; ++d) load_out[d] = load[d];
+}
+
+// Algorithm 1 with self-contention.  As oracle_schedule_stream, plus:
+//   arrival_us[r]  arrival time of request r in microseconds (events are in time order);
+//   inflight_cap   the counter's maximum (0 turns self-contention off);
+//   xfer_hint[r]   (nullable) another implementation's transfer time of r in whole
+//                  microseconds: when it differs from this one's by at most one (the same
+//                  transfer time rounded from a different precision), it is adopted so
+//                  that both continue from the same completion time (counted);
+//   xfer_us[r]     out: the chosen candidate's transfer time in whole microseconds,
+//                  -1 when r is rejected.
+// counts: near-ties, unexplained decisions, rejects, adopted transfer times, unexplained
+// transfer times.
+void oracle_schedule_stream_inflight(
+    const uint32_t* fanout, const uint8_t* role, const double* bw, const double* lat,
+    const float* util, uint64_t n_links, const uint32_t* len, const uint32_t* prefill,
+    const uint32_t* snap, const int64_t* arrival_us, const uint16_t* M, const uint32_t* events,
+    uint64_t n_events, double w_net, double w_prefix, double w_load, double theta, int64_t cap,
+    uint64_t bytes_per_token, uint32_t inflight_cap, const int64_t* load_init,
+    const int32_t* hint, const int32_t* xfer_hint, double rel_tol, int32_t* dec, double* best,
+    double* second, int32_t* xfer_us, int64_t* load_out, int64_t* counts) {
+  const Tree t = make_tree(fanout);
+  std::vector<uint64_t> pre, decs;
+  ranks(role, t.n, pre, decs);
+  const uint64_t D = decs.size(), P = pre.size();
+  std::vector<int64_t> load(D, 0);
+  if (load_init)
+    for (uint64_t d = 0; d < D; ++d) load[d] = load_init[d];
+  std::vector<uint32_t> inflight(P * 4, 0);  // [prefill rank][tier]
+  // pending completions: (time, prefill rank * 4 + tier), earliest first
+  typedef std::pair<int64_t, uint64_t> Done;
+  std::priority_queue<Done, std::vector<Done>, std::greater<Done>> pending;
+  std::vector<double> score(D), xfer(D);
+  const double inf = std::numeric_limits<double>::infinity();
+
+  for (uint64_t e = 0; e < n_events; ++e) {
+    const uint32_t code = events[e];
+    const uint32_t r = code & 0x7fffffffu;
+    const int64_t l = len[r];
+    if (code >> 31) {  // departure
+      if (dec[r] >= 0) load[dec[r]] -= l;
+      continue;
+    }
+    const int64_t now = arrival_us[r];
+    while (!pending.empty() && pending.top().first <= now) {  // transfers done by now
+      uint32_t& n = inflight[pending.top().second];
+      if (n > 0) n -= 1;
+      pending.pop();
+    }
+    const float* u_row = util + (uint64_t)snap[r] * n_links;
+    const uint64_t pr = prefill[r];
+    const uint64_t p = pre[pr];
+    int32_t arg = -1;
+    for (uint64_t d = 0; d < D; ++d) {
+      int tau = 0;
+      const double b = path_bottleneck(t, bw, u_row, p, decs[d], &tau);
+      const double b_eff = b / (1.0 + (double)inflight[pr * 4 + tau]);  // Eq. 4
+      const int64_t lam = 16 * (int64_t)M[(uint64_t)r * D + d];
+      const double s_eff = (double)((l - lam) * (int64_t)bytes_per_token);
+      xfer[d] = s_eff / b_eff + lat[tau];
+      if (load[d] + l > cap) { score[d] = inf; continue; }
+      const double miss = (double)(l - lam) / (double)l;
+      score[d] = w_net * xfer[d] + w_prefix * miss + w_load * (theta * (double)load[d]);
+      if (arg < 0 || score[d] < score[arg]) arg = (int32_t)d;
+    }
+    double b1 = inf, b2 = inf;
+    if (arg >= 0) {
+      b1 = score[arg];
+      for (uint64_t d = 0; d < D; ++d)
+        if ((int32_t)d != arg && score[d] < b2) b2 = score[d];
+    }
+    int32_t chosen = arg;
+    if (hint && hint[r] != arg) {
+      const int32_t h = hint[r];
+      const bool near = (arg >= 0 && h >= 0 && (uint64_t)h < D && score[h] != inf &&
+                         score[h] - b1 <= rel_tol * std::fabs(b1));
+      counts[near ? 0 : 1] += 1;
+      chosen = (h >= 0 && (uint64_t)h < D) ? h : -1;
+    }
+    dec[r] = chosen;
+    best[r] = b1;
+    second[r] = b2;
+    if (chosen < 0) {
+      counts[2] += 1;
+      xfer_us[r] = -1;
+      continue;
+    }
+    load[chosen] += l;
+    int64_t dt = std::llround(xfer[chosen] * 1e6);  // whole microseconds, half up
+    if (xfer_hint && xfer_hint[r] != dt) {
+      const int64_t diff = (int64_t)xfer_hint[r] - dt;
+      const bool close = xfer_hint[r] >= 0 && diff >= -1 && diff <= 1;
+      counts[close ? 3 : 4] += 1;
+      if (close) dt = xfer_hint[r];
+    }
+    xfer_us[r] = (int32_t)dt;
+    int tau = 0;
+    path_bottleneck(t, bw, u_row, p, decs[chosen], &tau);
+    uint32_t& n = inflight[pr * 4 + tau];  // Algorithm 1 line 14
+    if (n < inflight_cap) n += 1;
+    pending.push(Done(now + dt, pr * 4 + tau));
   }
   for (uint64_t d = 0; d < D; ++d) load_out[d] = load[d];
 }

@@ -130,3 +130,64 @@ def greedy_exact(tree, role, bw, lat, util, length, prefill, snap, M, events,
             best[r] = s
             load[d] += l
     return dec, best, load
+
+
+def greedy_exact_inflight(tree, role, bw, lat, util, length, prefill, snap, arrival_us, M,
+                          events, w, theta, cap, bpt, inflight_cap):
+    """Exact-rational Algorithm 1 with self-contention: the effective bandwidth of a
+    candidate is its path bottleneck over 1 + n[prefill][tier]; a dispatch raises that
+    counter (at most inflight_cap) and its transfer completes, lowering it again (not
+    below zero), at arrival + round-half-up(transfer time in microseconds); completions
+    due at or before an arrival come first.  Returns (dec, best, load, xfer_us)."""
+    pre = [i for i in range(tree.n) if role[i] == 0]
+    dec_inst = [i for i in range(tree.n) if role[i] == 1]
+    D = len(dec_inst)
+    load = [0] * D
+    R = len(length)
+    dec = [-1] * R
+    best = [None] * R
+    xfer_us = [-1] * R
+    n = {}                       # (prefill rank, tier) -> counter
+    pending = []                 # (done time, prefill rank, tier)
+    wn, wp, wl = (frac(x) for x in w)
+    th = frac(theta)
+    for code in events:
+        code = int(code)
+        r = code & 0x7FFFFFFF
+        l = int(length[r])
+        if code >> 31:
+            if dec[r] >= 0:
+                load[dec[r]] -= l
+            continue
+        now = int(arrival_us[r])
+        pending.sort()
+        while pending and pending[0][0] <= now:
+            _, pr, tau = pending.pop(0)
+            n[(pr, tau)] = max(0, n.get((pr, tau), 0) - 1)
+        pr = int(prefill[r])
+        p = pre[pr]
+        u_row = util[int(snap[r])]
+        scores, times = [], []
+        for d in range(D):
+            tau = tree.tier(p, dec_inst[d])
+            miss_tok = l - 16 * int(M[r][d])
+            b_eff = bottleneck(tree, bw, u_row, p, dec_inst[d]) / (1 + n.get((pr, tau), 0))
+            T = Fraction(miss_tok * bpt) / b_eff + frac(lat[tau])
+            times.append((T, tau))
+            if load[d] + l > cap:
+                scores.append(None)
+                continue
+            scores.append(wn * T + wp * Fraction(miss_tok, l) + wl * th * load[d])
+        cands = [(s, d) for d, s in enumerate(scores) if s is not None]
+        if not cands:
+            continue
+        s, d = min(cands)
+        dec[r] = d
+        best[r] = s
+        load[d] += l
+        T, tau = times[d]
+        dt = int((T * 1000000 + Fraction(1, 2)) // 1)
+        xfer_us[r] = dt
+        n[(pr, tau)] = min(inflight_cap, n.get((pr, tau), 0) + 1)
+        pending.append((now + dt, pr, tau))
+    return dec, best, load, xfer_us

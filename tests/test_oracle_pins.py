@@ -237,7 +237,7 @@ def test_prefix_closed_form_under_generator():
 
 
 # --------------------------------------------------------------------- P4: greedy
-def _tiny_problem(seed, D_role="alternate", R=6, cap=None, n_snap=3):
+def _tiny_problem(seed, D_role="alternate", R=6, cap=None, n_snap=3, span=1000):
     rng = np.random.default_rng(seed)
     fanout = (2, 2, 2, 1) if D_role == "alternate" else (2, 2, 2, 2)
     tree = naive.ExplicitTree(fanout)
@@ -253,15 +253,15 @@ def _tiny_problem(seed, D_role="alternate", R=6, cap=None, n_snap=3):
     for r in range(R):
         M[r] = rng.integers(0, int(length[r]) // 16 + 1, size=D)
     # events: arrivals in order, departures interleaved after their arrival
-    t_arr = np.sort(rng.integers(0, 1000, size=R))
-    t_dep = t_arr + rng.integers(1, 600, size=R)
+    t_arr = np.sort(rng.integers(0, span, size=R))
+    t_dep = t_arr + rng.integers(1, 600 * span // 1000, size=R)
     t = np.concatenate([t_dep, t_arr]); typ = np.concatenate([np.zeros(R), np.ones(R)]).astype(int)
     rr = np.concatenate([np.arange(R), np.arange(R)])
     o = np.lexsort((rr, typ, t))
     events = (rr[o].astype(np.uint64) | ((1 - typ[o]).astype(np.uint64) << np.uint64(31))).astype(np.uint32)
     cap = int(cap if cap is not None else rng.integers(3000, 9000))
     return dict(tree=tree, fanout=fanout, role=role, bw=bw, lat=lat, u=u, length=length,
-                prefill=prefill, snap=snap, M=M, events=events, cap=cap)
+                prefill=prefill, snap=snap, M=M, events=events, cap=cap, arrival_us=t_arr)
 
 
 def _run_oracle(pb, w, theta=float(np.float32(1e-6)), bpt=81920, hint=None):
@@ -522,3 +522,127 @@ def test_greedy_capacity_boundary_is_inclusive():
     pb["cap"] = l0 - 1
     res = _run_oracle(pb, (1.0, 1.0, 1.0))
     assert res.dec[0] == -1
+
+
+# ------------------------------------------------ self-contention (NEXT: n_inflight)
+def _run_inflight(pb, w, inflight_cap, theta=float(np.float32(1e-6)), bpt=81920):
+    return oracle.schedule_stream_inflight(pb["fanout"], pb["role"], pb["bw"], pb["lat"], pb["u"],
+                                           pb["length"], pb["prefill"], pb["snap"],
+                                           pb["arrival_us"], pb["M"], pb["events"], w[0], w[1],
+                                           w[2], theta, pb["cap"], bpt, inflight_cap)
+
+
+def test_inflight_off_is_the_plain_greedy():
+    """A cap of 0 keeps every counter at 0: the plain Algorithm 1, value for value."""
+    for seed in range(20):
+        pb = _tiny_problem(seed, span=50_000)
+        w = tuple(float(np.float32(x)) for x in np.random.default_rng(300 + seed).uniform(0, 2, 3))
+        a, b = _run_oracle(pb, w), _run_inflight(pb, w, 0)
+        np.testing.assert_array_equal(a.dec, b.dec)
+        np.testing.assert_array_equal(a.best, b.best)
+        np.testing.assert_array_equal(a.second, b.second)
+        np.testing.assert_array_equal(a.load, b.load)
+        assert ((b.xfer_us >= 0) == (b.dec >= 0)).all()
+
+
+def test_inflight_matches_exact_rational_bruteforce():
+    """Counters, completions and transfer times against an exact-rational evaluator with
+    BFS paths, over caps 1, 2, 3, 16 and arrivals packed into 1 ms up to spread over 0.3 s."""
+    theta = float(np.float32(1e-6))
+    changed = n_cmp = 0
+    for seed in range(48):
+        span = (1000, 50_000, 300_000)[seed % 3]
+        icap = (1, 2, 3, 16)[seed % 4]
+        pb = _tiny_problem(seed, R=8, span=span)
+        w = tuple(float(np.float32(x)) for x in np.random.default_rng(500 + seed).uniform(0, 2, 3))
+        res = _run_inflight(pb, w, icap)
+        dec, best, load, xfer = naive.greedy_exact_inflight(
+            pb["tree"], pb["role"], pb["bw"], pb["lat"], pb["u"], pb["length"], pb["prefill"],
+            pb["snap"], pb["arrival_us"], pb["M"], pb["events"], w, theta, pb["cap"], 81920, icap)
+        assert list(res.dec) == dec
+        assert list(res.load) == load
+        assert list(res.xfer_us) == xfer
+        for r in range(len(dec)):
+            if dec[r] >= 0:
+                assert res.best[r] == pytest.approx(float(best[r]), rel=1e-14)
+                n_cmp += 1
+        plain = _run_inflight(pb, w, 0)
+        changed += int((plain.dec != res.dec).any() or (plain.best != res.best).any())
+    assert n_cmp > 200 and changed > 10
+
+
+def _worked_example_stream(arrival_us, M_rows, c3=0.2):
+    """The worked example of Sec. III-D on a (2,2,2,2) tree: prefill instance 0, decode d1 =
+    instance 4 (same pod: tier 2) and d2 = instance 8 (other pod: tier 3); B2 = 6.25 GB/s,
+    B3 = 3.125 GB/s (B0, B1 larger), every link at c = 0.2 except the pod-spine links of
+    the path to d2 at c3; no latency.  Requests of 100,000 tokens at 100,000 B per token
+    (10 GB aggregate KV), so a hit of M blocks leaves (100,000 - 16 M) * 1e5 bytes."""
+    fanout = (2, 2, 2, 2)
+    role = np.zeros(16, np.uint8)
+    role[[4, 8]] = 1
+    L = oracle.used_links(fanout)
+    u = np.full((1, L), 0.2, np.float32)
+    links, levels = oracle.path_links(fanout, 0, 8)
+    u[0, links[levels == 3]] = c3
+    R = len(arrival_us)
+    t = np.asarray(arrival_us, np.int64)
+    events = np.concatenate([np.arange(R), np.arange(R) | (1 << 31)]).astype(np.uint32)
+    return dict(fanout=fanout, role=role, bw=[100e9, 50e9, 6.25e9, 3.125e9], lat=[0.0] * 4,
+                u=u, length=np.full(R, 100_000, np.uint32), prefill=np.zeros(R, np.uint32),
+                snap=np.zeros(R, np.uint32), M=np.asarray(M_rows, np.uint16), events=events,
+                cap=10 ** 7, arrival_us=t)
+
+
+def _worked(pb, icap):
+    return oracle.schedule_stream_inflight(pb["fanout"], pb["role"], pb["bw"], pb["lat"], pb["u"],
+                                           pb["length"], pb["prefill"], pb["snap"],
+                                           pb["arrival_us"], pb["M"], pb["events"], 1.0, 0.0,
+                                           0.0, 0.0, pb["cap"], 100_000, icap)
+
+
+def test_inflight_worked_example_end_to_end():
+    """Sec. III-D through the greedy: request A (no hits) goes to d1 and stays in flight
+    for 2 s; request B 1 ms later (50% hit on d1, 90% on d2) sees B_eff = 2.5 GB/s on both
+    candidates, T_d1 = 2.0 s and T_d2 = 0.4 s, and with c3 = 0.5, T_d2 = 0.64 s."""
+    g = golden("worked_example.txt")
+    a_rows = [[0, 0], [3125, 5625]]          # 3125 blocks = 50%, 5625 blocks = 90% of 6250
+    res = _worked(_worked_example_stream([0, 1000], a_rows), 16)
+    assert list(res.dec) == [0, 1]
+    assert res.xfer_us[0] == 2_000_000                       # 10 GB at 5 GB/s
+    assert res.best[1] == pytest.approx(g["T_d2"], rel=1e-6)
+    assert res.second[1] == pytest.approx(g["T_d1"], rel=1e-6)   # d1 with one in flight
+    assert res.xfer_us[1] == round(g["T_d2"] * 1e6)
+    # the counter is what doubles d1's time: without it d1 costs 1.0 s
+    off = _worked(_worked_example_stream([0, 1000], a_rows), 0)
+    assert off.second[1] == pytest.approx(g["T_d1"] / 2, rel=1e-6)
+    # c3 raised to 0.5 on d2's path
+    pert = _worked(_worked_example_stream([0, 1000], a_rows, c3=g["c3_perturbed"]), 16)
+    assert pert.best[1] == pytest.approx(g["T_d2_perturbed"], rel=1e-6)
+    assert pert.second[1] == pytest.approx(g["T_d1"], rel=1e-6)
+
+
+def test_inflight_completion_timing_and_cap():
+    """A's transfer ends at 2,000,000 us: an arrival at that instant sees it done, one a
+    microsecond earlier does not.  The counter saturates at the cap and, being a counter,
+    drops on the first completion even while a second transfer is still in flight."""
+    a_rows = [[0, 0], [3125, 5625]]
+    at = _worked(_worked_example_stream([0, 2_000_000], a_rows), 16)
+    before = _worked(_worked_example_stream([0, 1_999_999], a_rows), 16)
+    assert at.second[1] == pytest.approx(1.0, rel=1e-6)
+    assert before.second[1] == pytest.approx(2.0, rel=1e-6)
+    # A1, A2 to d1 (the second sees one in flight: 4.0 s on d1 vs 4.0 s on d2 -> d1, the
+    # lower rank), then C probes the counter: 3.0 s with the cap at 16 (two in flight),
+    # 2.0 s with the cap at 1
+    rows = [[0, 0], [0, 0], [3125, 5625]]
+    t = [0, 10, 20]
+    c16 = _worked(_worked_example_stream(t, rows), 16)
+    c1 = _worked(_worked_example_stream(t, rows), 1)
+    assert list(c16.dec[:2]) == [0, 0] and list(c1.dec[:2]) == [0, 0]
+    assert c16.second[2] == pytest.approx(3.0, rel=1e-6)
+    assert c1.second[2] == pytest.approx(2.0, rel=1e-6)
+    # A1 ends at 2 s and A2 (4 s, dispatched with one in flight) at 10 us + 4 s: at
+    # 2,000,005 us one completion has lowered the saturated counter to 0 although A2 is
+    # still in flight
+    late = _worked(_worked_example_stream([0, 10, 2_000_005], rows), 1)
+    assert list(late.xfer_us[:2]) == [2_000_000, 4_000_000]
+    assert late.second[2] == pytest.approx(1.0, rel=1e-6)
