@@ -13,6 +13,7 @@
  *   netkv_cache_build       decode caches K_d as open-addressing hash tables
  *   netkv_prefix_match      block-level prefix hit M[r][d] (Sec. III-B)
  *   netkv_schedule_streams  the greedy of Algorithm 1 over independent streams
+ *   netkv_schedule_streams_inflight  the same with self-contention (Eq. 4's n_inflight)
  *
  * Conventions for every call:
  *   - Pointers named d_* are device pointers owned by the caller; the library never
@@ -259,6 +260,39 @@ netkv_status netkv_schedule_streams(netkv_topology_t topo, uint32_t n_streams,
                                     const int64_t* d_load_init, int32_t* d_dec, float* d_best,
                                     float* d_second, int64_t* d_load_final, void* d_workspace,
                                     size_t workspace_bytes, int* d_status, netkv_stream_t stream);
+
+/* Algorithm 1 with self-contention (Eq. 4's n_inflight term, Algorithm 1 lines 5 and 14,
+ * Sec. IV-C).  As netkv_schedule_streams without a workspace, and in addition each
+ * stream keeps a counter n[p][tau] per prefill rank and tier (zero at the start of the
+ * call) of its own transfers in flight:
+ *     B_eff  = min(UB[k_r][p][tau], UB[k_r][d][tau]) / (1 + n[p_r][tau])  (Eq. 4)
+ *     T_xfer = s_eff / B_eff + L_tau                                     (Eq. 3)
+ * A dispatch to d* raises n[p_r][tau(p_r, d*)] by one unless it is already at
+ * inflight_cap, and its transfer completes at arrival_us[r] + xfer_us[r], where
+ * xfer_us[r] is its T_xfer rounded to whole microseconds; a completion lowers the
+ * counter by one unless it is zero.  Completions due at or before an arrival's time
+ * are applied before that arrival is scored.  inflight_cap = 0 keeps every counter at
+ * zero: the result is then that of netkv_schedule_streams without a workspace.
+ *
+ *   d_arrival_us [R] int64 arrival time of each request in microseconds; a stream's
+ *                arrivals must be in time order, as its events are
+ *   inflight_cap 0 .. 255 (the paper's default is 16)
+ *   d_xfer_us    [R] int32 output: T_xfer of the chosen candidate in whole microseconds
+ *                (at most 2^31 - 1), -1 for a rejected arrival
+ * Other arguments as for netkv_schedule_streams.  Limits: fewer than 16,384 prefill
+ * ranks; the counters (4 bytes per prefill rank) and the pending completions of a
+ * stream live in shared memory, 4,096 pending completions per stream for pools of more
+ * than 16 decodes and 256 for smaller ones (packed several streams to a warp); a
+ * completion that does not fit sets EFULL and is dropped (its counter is not lowered).
+ * Host errors: EINVAL for a cap above 255, too many prefill ranks or missing buffers.
+ */
+netkv_status netkv_schedule_streams_inflight(
+    netkv_topology_t topo, uint32_t n_streams, const netkv_weights* d_w, uint32_t R,
+    const uint32_t* d_len, const uint32_t* d_prefill, const uint32_t* d_snap,
+    const int64_t* d_arrival_us, const uint16_t* d_M, const float* d_UB, uint32_t n_snap,
+    const uint32_t* d_events, const uint64_t* d_event_off, uint32_t inflight_cap,
+    const int64_t* d_load_init, int32_t* d_dec, float* d_best, float* d_second,
+    int32_t* d_xfer_us, int64_t* d_load_final, int* d_status, netkv_stream_t stream);
 
 /* ------------------------------------------------------------------ transfers
  * Asynchronous copy of `bytes` bytes by a kernel (SM loads and stores).  Either side may

@@ -14,7 +14,7 @@ from typing import Optional
 
 import numpy as np
 
-from . import prefix_match, schedule_stream, up_bottleneck
+from . import prefix_match, schedule_stream, schedule_stream_inflight, up_bottleneck
 
 
 @dataclasses.dataclass
@@ -74,3 +74,34 @@ def run_stream(w, s: int, theta: float, cap: int, bytes_per_token: int,
     UB = up_bottleneck(spec.fanout, spec.tier_bw, util)
     return OracleStream(r0, r1, M, res.dec, res.best, res.second, res.load, res.near_ties,
                         res.mismatches, res.rejects, snaps, UB)
+
+
+def run_stream_inflight(w, s: int, theta: float, cap: int, bytes_per_token: int,
+                        inflight_cap: int, hint: Optional[np.ndarray] = None,
+                        xfer_hint: Optional[np.ndarray] = None, rel_tol: float = 1e-5,
+                        M: Optional[np.ndarray] = None) -> OracleStream:
+    """Oracle for stream s with self-contention (Eq. 4's n_inflight, Algorithm 1 lines 5
+    and 14).  hint / xfer_hint: another implementation's decisions and transfer times
+    for the stream's requests (local order).  The result carries xfer_us."""
+    from synth import request_set
+    r0, r1, ev_local, snaps, snap_local = stream_problem(w, s)
+    util = w.util()[snaps] if w.n_snap * w.L < (1 << 24) else np.stack([w.util(int(k), int(k) + 1)[0] for k in snaps])
+    if M is None:
+        g = int(request_set(w)[r0]) if r1 > r0 else 0
+        keys, key_off = stream_cache_keys(w, g)
+        chains = w.chains(r0, r1)
+        chain_off = (w.chain_off[r0:r1 + 1] - w.chain_off[r0]).astype(np.uint64)
+        M = prefix_match(keys, key_off, w.D, chains, chain_off,
+                         np.array([0, r1 - r0], np.uint32))
+    wn, wp, wl = (float(x) for x in w.weights[s])
+    spec = w.spec
+    res = schedule_stream_inflight(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, util,
+                                   w.length[r0:r1], w.prefill[r0:r1], snap_local,
+                                   w.arrival_us[r0:r1], M, ev_local, wn, wp, wl, theta, cap,
+                                   bytes_per_token, inflight_cap, hint=hint, xfer_hint=xfer_hint,
+                                   rel_tol=rel_tol)
+    UB = up_bottleneck(spec.fanout, spec.tier_bw, util)
+    out = OracleStream(r0, r1, M, res.dec, res.best, res.second, res.load, res.near_ties,
+                       res.mismatches, res.rejects, snaps, UB)
+    out.xfer_us, out.xfer_adopted, out.xfer_mismatches = res.xfer_us, res.xfer_adopted, res.xfer_mismatches
+    return out

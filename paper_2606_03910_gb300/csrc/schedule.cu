@@ -66,6 +66,83 @@ __device__ __forceinline__ float base_score(const netkv_weights& w, uint32_t l, 
   return w.w_net * T + w.w_prefix * miss;
 }
 
+// Self-contention (Eq. 4's n_inflight, Algorithm 1 lines 5 and 14, Sec. IV-C): the
+// candidate's bandwidth is divided by 1 + n; T is returned for the completion time.
+__device__ __forceinline__ float contended_score(const netkv_weights& w, uint32_t l, uint32_t m,
+                                                 float ub_p, float ub_d, float lat_tau,
+                                                 uint32_t n, float& T, int* status) {
+  uint32_t lam = 16u * m;
+  if (m > l / 16u) {
+    flag_status(status, NETKV_DEV_EDOMAIN);
+    lam = lam < l ? lam : l;
+  }
+  const uint32_t miss_tok = l - lam;
+  const float b_eff = fminf(ub_p, ub_d) / (float)(1u + n);
+  const float s_eff = (float)((int64_t)miss_tok * (int64_t)w.bytes_per_token);
+  T = s_eff / b_eff + lat_tau;
+  const float miss = (float)miss_tok / (float)l;
+  return w.w_net * T + w.w_prefix * miss;
+}
+
+// combine() carrying the winner's transfer time along
+__device__ __forceinline__ void combine_t(float& b, uint32_t& i, float& s, float& tt, float b2,
+                                          uint32_t i2, float s2, float t2) {
+  const bool other = (b2 < b) || (b2 == b && i2 < i);
+  if (other) {
+    s = fminf(s2, b);
+    b = b2;
+    i = i2;
+    tt = t2;
+  } else {
+    s = fminf(s, b2);
+  }
+}
+template <int LPS>
+__device__ __forceinline__ void seg_argmin_t(float& b, uint32_t& i, float& s, float& tt,
+                                             uint32_t mask) {
+#pragma unroll
+  for (int o = LPS / 2; o; o >>= 1) {
+    const float b2 = __shfl_xor_sync(mask, b, o, LPS);
+    const uint32_t i2 = __shfl_xor_sync(mask, i, o, LPS);
+    const float s2 = __shfl_xor_sync(mask, s, o, LPS);
+    const float t2 = __shfl_xor_sync(mask, tt, o, LPS);
+    combine_t(b, i, s, tt, b2, i2, s2, t2);
+  }
+}
+
+// Pending transfer completions of one stream: a binary min-heap in shared memory kept by
+// the stream's lead thread, keys (completion time in us << 16) | (prefill rank << 2) | tier.
+struct DoneHeap {
+  unsigned long long* a;
+  uint32_t n, cap;
+  __device__ bool push(unsigned long long k) {
+    if (n == cap) return false;
+    uint32_t i = n++;
+    while (i > 0) {
+      const uint32_t p = (i - 1) >> 1;
+      if (a[p] <= k) break;
+      a[i] = a[p];
+      i = p;
+    }
+    a[i] = k;
+    return true;
+  }
+  __device__ void pop() {
+    const unsigned long long k = a[--n];
+    if (n == 0) return;
+    uint32_t i = 0;
+    for (;;) {
+      uint32_t c = 2 * i + 1;
+      if (c >= n) break;
+      if (c + 1 < n && a[c + 1] < a[c]) ++c;
+      if (a[c] >= k) break;
+      a[i] = a[c];
+      i = c;
+    }
+    a[i] = k;
+  }
+};
+
 // Base scores of every arrival: base[r][d] = base_score(...) for the stream's weights.
 // No dependence between events, so the events of a stream are split into contiguous
 // ranges over the segments (LPS lanes each) of grid.y blocks; each segment strides over
@@ -215,7 +292,14 @@ __global__ void __launch_bounds__(256) base_wide_kernel(
 // LPS = lanes per stream.  LPS == 32: one stream per CTA of BLOCK threads.  LPS < 32
 // (BLOCK == 32, NPT == 1, D <= LPS): a warp runs 32 / LPS streams side by side, one per
 // segment of LPS lanes, so that small decode pools still use every lane.
-template <int NPT, int BLOCK, int LPS, bool kBase>
+// Self-contention (kInfl): each stream keeps n_inflight[prefill][tier] as four 8-bit
+// counters per prefill rank and its pending completions in a heap, both in dynamic
+// shared memory (`infl_bytes` per stream: counters, then `heap_cap` heap keys).  The
+// lead thread applies the completions due by an arrival's time before it is scored
+// (one extra stream barrier per arrival), and after the decision raises the chosen
+// tier's counter (saturating at `inflight_cap`), records the transfer time and pushes
+// its completion.  The argmin carries the winner's transfer time along.
+template <int NPT, int BLOCK, int LPS, bool kBase, bool kInfl = false>
 __global__ void __launch_bounds__(BLOCK) schedule_kernel(
     TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
     const float* __restrict__ base, const uint32_t* __restrict__ len,
@@ -223,12 +307,16 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
     const uint16_t* __restrict__ M, const float* __restrict__ UB, uint32_t n_snap,
     const uint32_t* __restrict__ events, const uint64_t* __restrict__ event_off,
     const int64_t* __restrict__ load_init, int32_t* dec, float* __restrict__ best,
-    float* __restrict__ second, int64_t* __restrict__ load_final, int* status) {
+    float* __restrict__ second, int64_t* __restrict__ load_final, int* status,
+    const int64_t* __restrict__ arrival_us = nullptr, uint32_t inflight_cap = 0,
+    int32_t* __restrict__ xfer_us = nullptr, uint32_t infl_bytes = 0, uint32_t heap_cap = 0) {
   static_assert(LPS == 32 || (BLOCK == 32 && NPT == 1), "packed streams use one warp");
+  static_assert(!(kBase && kInfl), "self-contention scores from UB and M");
   constexpr int NW = BLOCK / 32;
   __shared__ float s_b[2][NW];
   __shared__ uint32_t s_i[2][NW];
   __shared__ float s_s[2][NW];
+  __shared__ float s_t[2][NW];
   const uint32_t lane_w = threadIdx.x & 31, wid = threadIdx.x >> 5;
   const uint32_t seg = LPS == 32 ? 0u : lane_w / LPS;
   const uint32_t stream = LPS == 32 ? blockIdx.x : blockIdx.x * (32 / LPS) + seg;
@@ -258,6 +346,18 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
   const uint64_t e0 = event_off[stream], e1 = event_off[stream + 1];
   uint32_t parity = 0;
 
+  uint32_t* cnt = nullptr;  // n_inflight: byte `tier` of cnt[prefill rank]
+  DoneHeap heap = {nullptr, 0u, 0u};
+  if constexpr (kInfl) {
+    extern __shared__ __align__(16) unsigned char infl_smem[];
+    unsigned char* mine = infl_smem + (size_t)(LPS == 32 ? 0u : seg) * infl_bytes;
+    cnt = reinterpret_cast<uint32_t*>(mine);
+    heap.a = reinterpret_cast<unsigned long long*>(mine + (size_t)((t.P * 4u + 15u) & ~15u));
+    heap.cap = heap_cap;
+    for (uint32_t i = tid; i < t.P; i += (LPS == 32 ? BLOCK : LPS)) cnt[i] = 0u;
+    if (LPS == 32) __syncthreads(); else __syncwarp(smask);
+  }
+
   // Software pipeline over events.  When event e is processed, its operands were
   // requested PD iterations earlier: event e+PD+1 gets its level bottlenecks (and, for a
   // departure, its decision) requested, event e+FD+1 its request fields and prefix hits,
@@ -272,6 +372,7 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
   const uint32_t kBad = 0xffffffffu;
   uint32_t cq[CD + 1];                        // event codes, index i = event e+i
   uint32_t lq[FD + 1], pq[FD + 1], kq[FD + 1], mq[FD + 1][NPT];
+  int64_t tq[FD + 1];                         // arrival times (self-contention only)
   float4 ubpq[PD + 1];
   float ubdq[PD + 1][NPT];
   int tauq[PD + 1][NPT];
@@ -343,14 +444,22 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
 
 #pragma unroll
   for (int i = 0; i <= CD; ++i) cq[i] = (e0 + i < e1) ? __ldg(events + e0 + i) : kBad;
+  auto time_of = [&](uint32_t code) -> int64_t {
+    if (!kInfl || code == kBad || (code >> 31) || (code & 0x7fffffffu) >= R) return 0;
+    return __ldg(arrival_us + (code & 0x7fffffffu));
+  };
 #pragma unroll
-  for (int i = 0; i <= FD; ++i) fields(cq[i], lq[i], pq[i], kq[i], mq[i]);
+  for (int i = 0; i <= FD; ++i) {
+    fields(cq[i], lq[i], pq[i], kq[i], mq[i]);
+    tq[i] = time_of(cq[i]);
+  }
 #pragma unroll
   for (int i = 0; i <= PD; ++i) operands(cq[i], pq[i], kq[i], ubpq[i], ubdq[i], tauq[i], decq[i]);
 
   for (uint64_t e = e0; e < e1; ++e) {
     // take event e's operands, then advance the pipeline by one event
     const uint32_t code = cq[0], l = lq[0], pr = pq[0], k = kq[0];
+    const int64_t now = tq[0];
     const float4 ubp = ubpq[0];
     float ubd[NPT];
     int tau[NPT];
@@ -369,6 +478,7 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
       lq[i] = lq[i + 1];
       pq[i] = pq[i + 1];
       kq[i] = kq[i + 1];
+      tq[i] = tq[i + 1];
 #pragma unroll
       for (int j = 0; j < NPT; ++j) mq[i][j] = mq[i + 1][j];
     }
@@ -384,6 +494,7 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
     }
     cq[CD] = (e + 1 + CD < e1) ? __ldg(events + e + 1 + CD) : kBad;
     fields(cq[FD], lq[FD], pq[FD], kq[FD], mq[FD]);
+    tq[FD] = time_of(cq[FD]);
     operands(cq[PD], pq[PD], kq[PD], ubpq[PD], ubdq[PD], tauq[PD], decq[PD]);
 
     const uint32_t r = code & 0x7fffffffu;
@@ -408,6 +519,7 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
         flag_status(status, l == 0 ? NETKV_DEV_EDOMAIN : NETKV_DEV_ERANGE);
         best[r] = inf;
         second[r] = inf;
+        if (kInfl) xfer_us[r] = -1;
       }
       if (lane == 0) *((volatile int32_t*)(dec + r)) = -1;
 #pragma unroll
@@ -420,16 +532,35 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
       continue;
     }
 
-    float b = inf, s2 = inf;
+    uint32_t cw = 0;  // self-contention counters of the request's prefill, a byte per tier
+    if constexpr (kInfl) {
+      if (lead_thread) {  // transfers completed by now (Algorithm 1 line 14's callback)
+        while (heap.n > 0 && (int64_t)(heap.a[0] >> 16) <= now) {
+          const uint32_t pt = (uint32_t)(heap.a[0] & 0xffffu);
+          heap.pop();
+          uint32_t* c = cnt + (pt >> 2);
+          const uint32_t sh = 8u * (pt & 3u);
+          if ((*c >> sh) & 0xffu) *c -= 1u << sh;
+        }
+      }
+      if (LPS == 32) __syncthreads(); else __syncwarp(smask);
+      cw = cnt[pr];
+    }
+    float b = inf, s2 = inf, bt = 0.0f;
     uint32_t bi = kNone;
 #pragma unroll
     for (int j = 0; j < NPT; ++j) {
       const uint32_t d = tid * NPT + j;
       if (d < D) {
         const bool feasible = load[j] + (int64_t)l <= w.cap_tokens;
-        float sc;
+        float sc, tj = 0.0f;
         if (kBase) {
           sc = __uint_as_float(m[j]) + w.w_load * (w.theta_s_per_token * (float)load[j]);
+        } else if (kInfl) {
+          const float net_prefix =
+              contended_score(w, l, m[j], pick4(ubp, tau[j]), ubd[j], pick4(lat, tau[j]),
+                              (cw >> (8 * tau[j])) & 0xffu, tj, status);
+          sc = net_prefix + w.w_load * (w.theta_s_per_token * (float)load[j]);
         } else {
           const float net_prefix = base_score(w, l, m[j], pick4(ubp, tau[j]), ubd[j],
                                               pick4(lat, tau[j]), status);
@@ -440,18 +571,21 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
             s2 = b;
             b = sc;
             bi = d;
+            bt = tj;
           } else if (sc < s2) {
             s2 = sc;
           }
         }
       }
     }
-    seg_argmin<LPS>(b, bi, s2, smask);
+    if constexpr (kInfl) seg_argmin_t<LPS>(b, bi, s2, bt, smask);
+    else seg_argmin<LPS>(b, bi, s2, smask);
     if (NW > 1) {
       if (lane == 0) {
         s_b[parity][wid] = b;
         s_i[parity][wid] = bi;
         s_s[parity][wid] = s2;
+        if (kInfl) s_t[parity][wid] = bt;
       }
       __syncthreads();
       b = inf;
@@ -461,11 +595,32 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
         b = s_b[parity][lane];
         bi = s_i[parity][lane];
         s2 = s_s[parity][lane];
+        if (kInfl) bt = s_t[parity][lane];
       }
-      seg_argmin<32>(b, bi, s2, 0xffffffffu);
+      if constexpr (kInfl) seg_argmin_t<32>(b, bi, s2, bt, 0xffffffffu);
+      else seg_argmin<32>(b, bi, s2, 0xffffffffu);
       parity ^= 1u;
     }
     const int32_t dstar = bi == kNone ? -1 : (int32_t)bi;
+    if constexpr (kInfl) {
+      if (lead_thread) {
+        if (dstar < 0) {
+          xfer_us[r] = -1;
+        } else {  // the dispatch's tier counter (Algorithm 1 line 14) and its completion
+          const double us = (double)bt * 1e6;
+          const int64_t dt = us < 2147483647.0 ? (int64_t)llrint(us) : 2147483647ll;
+          xfer_us[r] = (int32_t)dt;
+          const uint4 lp = __ldg(t.links + __ldg(t.pre + pr));
+          const uint4 lo = __ldg(t.links + __ldg(t.dec + (uint32_t)dstar));
+          const uint32_t ts = (uint32_t)tier_of(lp, lo);
+          uint32_t* c = cnt + pr;
+          const uint32_t sh = 8u * ts;
+          if (((*c >> sh) & 0xffu) < inflight_cap) *c += 1u << sh;
+          if (!heap.push(((unsigned long long)(now + dt) << 16) | ((unsigned long long)pr << 2) | ts))
+            flag_status(status, NETKV_DEV_EFULL);
+        }
+      }
+    }
     if (dstar >= 0) {
 #pragma unroll
       for (int j = 0; j < NPT; ++j)
@@ -780,6 +935,9 @@ __global__ void __launch_bounds__(BLOCK) schedule_staged_kernel(
 }
 
 constexpr int kStages = 8;
+constexpr uint32_t kHeapPerStream = 4096;       // pending completions, one stream per CTA
+constexpr uint32_t kHeapPerPackedStream = 256;  // pending completions, packed streams
+constexpr size_t kInflightSmemMax = 200u * 1024u;
 
 template <int NPT, int BLOCK>
 netkv_status launch_staged(const TopoArgs& t, uint32_t n_streams, const netkv_weights* d_w,
@@ -878,6 +1036,39 @@ netkv_status launch(const TopoArgs& t, uint32_t n_streams, const netkv_weights* 
   return netkv_launch_status();
 }
 
+// Self-contention launch: dynamic shared memory per stream holds the counters (four
+// bytes per prefill rank) and a heap of pending completions.
+template <int NPT, int BLOCK, int LPS>
+netkv_status launch_inflight(const TopoArgs& t, uint32_t n_streams, const netkv_weights* d_w,
+                             uint32_t R, const uint32_t* d_len, const uint32_t* d_prefill,
+                             const uint32_t* d_snap, const int64_t* d_arrival_us,
+                             const uint16_t* d_M, const float* d_UB, uint32_t n_snap,
+                             const uint32_t* d_events, const uint64_t* d_event_off,
+                             uint32_t inflight_cap, const int64_t* d_load_init, int32_t* d_dec,
+                             float* d_best, float* d_second, int32_t* d_xfer_us,
+                             int64_t* d_load_final, int* d_status, cudaStream_t s) {
+  const uint32_t per_cta = LPS == 32 ? 1u : 32u / LPS;
+  const unsigned grid = (n_streams + per_cta - 1) / per_cta;
+  const uint32_t heap_cap = LPS == 32 ? kHeapPerStream : kHeapPerPackedStream;
+  const uint32_t infl_bytes = ((t.P * 4u + 15u) & ~15u) + heap_cap * 8u;
+  const size_t smem = (size_t)per_cta * infl_bytes;
+  if (smem > kInflightSmemMax) return NETKV_EINVAL;
+  if (smem > 48u * 1024u) {
+    static bool raised = false;  // the same value every time: a benign race
+    if (!raised) {
+      NETKV_CUDA_TRY(cudaFuncSetAttribute(schedule_kernel<NPT, BLOCK, LPS, false, true>,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)kInflightSmemMax));
+      raised = true;
+    }
+  }
+  schedule_kernel<NPT, BLOCK, LPS, false, true><<<grid, BLOCK, smem, s>>>(
+      t, n_streams, d_w, R, nullptr, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events,
+      d_event_off, d_load_init, d_dec, d_best, d_second, d_load_final, d_status, d_arrival_us,
+      inflight_cap, d_xfer_us, infl_bytes, heap_cap);
+  return netkv_launch_status();
+}
+
 }  // namespace
 
 extern "C" size_t netkv_schedule_workspace_size(uint32_t R, uint32_t D) {
@@ -919,5 +1110,42 @@ extern "C" netkv_status netkv_schedule_streams(
   if (D <= 1024) NETKV_SCHED(4, 256, 32);
   if (D <= 4096) NETKV_SCHED(4, 1024, 32);
 #undef NETKV_SCHED
+  return NETKV_EINVAL;
+}
+
+extern "C" netkv_status netkv_schedule_streams_inflight(
+    netkv_topology_t topo, uint32_t n_streams, const netkv_weights* d_w, uint32_t R,
+    const uint32_t* d_len, const uint32_t* d_prefill, const uint32_t* d_snap,
+    const int64_t* d_arrival_us, const uint16_t* d_M, const float* d_UB, uint32_t n_snap,
+    const uint32_t* d_events, const uint64_t* d_event_off, uint32_t inflight_cap,
+    const int64_t* d_load_init, int32_t* d_dec, float* d_best, float* d_second,
+    int32_t* d_xfer_us, int64_t* d_load_final, int* d_status, netkv_stream_t stream) {
+  if (!topo || !d_w || !d_event_off || !d_load_final) return NETKV_EINVAL;
+  if (inflight_cap > 255) return NETKV_EINVAL;
+  if (n_streams == 0) return NETKV_OK;
+  if (n_streams > 0x7fffffffu) return NETKV_EINVAL;
+  if (R > 0 && (!d_len || !d_prefill || !d_snap || !d_arrival_us || !d_M || !d_UB || !d_dec ||
+                !d_best || !d_second || !d_xfer_us || !d_events))
+    return NETKV_EINVAL;
+  if (!aligned_to(d_w, 8) || !aligned_to(d_UB, 16) || !aligned_to(d_event_off, 8) ||
+      !aligned_to(d_load_final, 8) || (d_load_init && !aligned_to(d_load_init, 8)) ||
+      (d_arrival_us && !aligned_to(d_arrival_us, 8)))
+    return NETKV_EINVAL;
+  const TopoArgs t = topo_args(topo);
+  if (t.P >= (1u << 14)) return NETKV_EINVAL;  // prefill rank in a completion key
+  const uint32_t D = t.D;
+  cudaStream_t s = (cudaStream_t)stream;
+#define NETKV_INFL(NPT, BLOCK, LPS)                                                             \
+  return launch_inflight<NPT, BLOCK, LPS>(t, n_streams, d_w, R, d_len, d_prefill, d_snap,      \
+                                          d_arrival_us, d_M, d_UB, n_snap, d_events,           \
+                                          d_event_off, inflight_cap, d_load_init, d_dec,       \
+                                          d_best, d_second, d_xfer_us, d_load_final, d_status, s)
+  if (D <= 8) NETKV_INFL(1, 32, 8);
+  if (D <= 16) NETKV_INFL(1, 32, 16);
+  if (D <= 32) NETKV_INFL(1, 32, 32);
+  if (D <= 256) NETKV_INFL(1, 256, 32);
+  if (D <= 1024) NETKV_INFL(4, 256, 32);
+  if (D <= 4096) NETKV_INFL(4, 1024, 32);
+#undef NETKV_INFL
   return NETKV_EINVAL;
 }

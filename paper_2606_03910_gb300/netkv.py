@@ -33,7 +33,7 @@ EXPORTS = ("netkv_topology_create", "netkv_topology_destroy", "netkv_topology_qu
            "netkv_oracle_build", "netkv_cache_index_bytes", "netkv_cache_build",
            "netkv_prefix_match_workspace_size",
            "netkv_prefix_match", "netkv_prefix_match_static", "netkv_schedule_workspace_size",
-           "netkv_schedule_streams",
+           "netkv_schedule_streams", "netkv_schedule_streams_inflight",
            "netkv_copy_async", "netkv_version")
 
 
@@ -73,6 +73,9 @@ _lib.netkv_schedule_workspace_size.argtypes = [_U32, _U32]
 _lib.netkv_schedule_workspace_size.restype = C.c_size_t
 _lib.netkv_schedule_streams.argtypes = [_P, _U32, _P, _U32, _P, _P, _P, _P, _P, _U32, _P, _P,
                                         _P, _P, _P, _P, _P, _P, C.c_size_t, _P, _P]
+_lib.netkv_schedule_streams_inflight.argtypes = [_P, _U32, _P, _U32, _P, _P, _P, _P, _P, _P,
+                                                 _U32, _P, _P, _U32, _P, _P, _P, _P, _P, _P,
+                                                 _P, _P]
 _lib.netkv_copy_async.argtypes = [_P, _P, C.c_size_t, _P]
 for _f in EXPORTS:
     if _f not in ("netkv_version", "netkv_prefix_match_workspace_size", "netkv_cache_index_bytes",
@@ -204,6 +207,18 @@ def netkv_schedule_streams(topo: Topology, n_streams: int, weights, R: int, leng
         _ptr(snap), _ptr(M), _ptr(UB), int(n_snap), _ptr(events), _ptr(event_off),
         _ptr(load_init), _ptr(dec), _ptr(best), _ptr(second), _ptr(load_final), _ptr(workspace),
         ws_bytes, _ptr(status), _stream(stream)))
+
+
+def netkv_schedule_streams_inflight(topo: Topology, n_streams: int, weights, R: int, length,
+                                    prefill, snap, arrival_us, M, UB, n_snap: int, events,
+                                    event_off, inflight_cap: int, load_init, dec, best, second,
+                                    xfer_us, load_final, status=None, stream=None) -> None:
+    """Algorithm 1 with self-contention; see include/netkv.h."""
+    _check("netkv_schedule_streams_inflight", _lib.netkv_schedule_streams_inflight(
+        topo.handle, int(n_streams), _ptr(weights), int(R), _ptr(length), _ptr(prefill),
+        _ptr(snap), _ptr(arrival_us), _ptr(M), _ptr(UB), int(n_snap), _ptr(events),
+        _ptr(event_off), int(inflight_cap), _ptr(load_init), _ptr(dec), _ptr(best),
+        _ptr(second), _ptr(xfer_us), _ptr(load_final), _ptr(status), _stream(stream)))
 
 
 def netkv_copy_async(dst, src, nbytes: int, stream=None) -> None:

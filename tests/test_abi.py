@@ -41,6 +41,15 @@ def test_library_exports_every_declared_symbol(lib):
     assert set(lib.EXPORTS) <= set(declared())
 
 
+def test_every_entry_point_declares_its_argument_types(lib):
+    """Without argtypes ctypes passes Python ints as 32-bit C ints, truncating device
+    pointers; every entry point of the binding must declare its argument types."""
+    for name in lib.EXPORTS:
+        if name == "netkv_version":
+            continue
+        assert getattr(lib._lib, name).argtypes is not None, name
+
+
 def test_version_and_host_validation(lib):
     assert lib.netkv_version() >= 1
     import numpy as np
@@ -57,6 +66,9 @@ def test_version_and_host_validation(lib):
                                      None, None, None, None, None, None, 0, None,
                                      None) == lib.NETKV_EINVAL
     assert so.netkv_schedule_workspace_size(10, 8) == 512
+    assert so.netkv_schedule_streams_inflight(None, 1, None, 0, None, None, None, None, None,
+                                              None, 0, None, None, 16, None, None, None, None,
+                                              None, None, None, None) == lib.NETKV_EINVAL
     assert so.netkv_topology_destroy(None) == lib.NETKV_EINVAL
 
 
