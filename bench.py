@@ -46,6 +46,9 @@ def parse():
                     help="replicas: the 4,096-stream scoring step (default); sweep: the "
                          "oracle-build sweep (1,000 snapshots x 2,048 x 8,192 pairs)")
     ap.add_argument("--snapshots", type=int, default=1000)
+    ap.add_argument("--inflight", type=int, default=0,
+                    help="self-contention counter cap (Eq. 4's n_inflight; the paper uses 16); "
+                         "0 = the plain greedy")
     ap.add_argument("--streams", type=int, default=4096)
     ap.add_argument("--cpu-streams", type=int, default=24)
     ap.add_argument("--no-cpu", action="store_true")
@@ -198,13 +201,17 @@ def measured_peaks():
 
 
 # ------------------------------------------------------------------ CPU oracle
-def cpu_oracle_sample(w, streams, theta, cap, bpt):
-    """Time the CPU oracle on whole streams of the workload; returns (decisions, seconds)."""
-    from oracle.workload import run_stream
+def cpu_oracle_sample(w, streams, theta, cap, bpt, inflight=0):
+    """Time the CPU oracle on whole streams of the workload (with self-contention when
+    inflight > 0); returns (decisions, seconds)."""
+    from oracle.workload import run_stream, run_stream_inflight
     t0 = time.perf_counter()
     dec = 0
     for s in streams:
-        res = run_stream(w, int(s), theta, cap, bpt)
+        if inflight > 0:
+            res = run_stream_inflight(w, int(s), theta, cap, bpt, inflight)
+        else:
+            res = run_stream(w, int(s), theta, cap, bpt)
         dec += int(res.dec.shape[0])
     return dec, time.perf_counter() - t0
 
@@ -277,12 +284,13 @@ def run_reference(args):
     order = np.random.default_rng(1).permutation(args.streams)
     k = 0
     for _ in range(args.warmup):
-        cpu_oracle_sample(w, order[k:k + per_step], theta, spec.cap_tokens, synth.BYTES_PER_TOKEN_SHARD)
+        cpu_oracle_sample(w, order[k:k + per_step], theta, spec.cap_tokens, synth.BYTES_PER_TOKEN_SHARD,
+                          args.inflight)
         k = (k + per_step) % args.streams
     dec_total, secs = 0, 0.0
     for _ in range(args.steps):
         d, s = cpu_oracle_sample(w, order[k:k + per_step], theta, spec.cap_tokens,
-                                 synth.BYTES_PER_TOKEN_SHARD)
+                                 synth.BYTES_PER_TOKEN_SHARD, args.inflight)
         dec_total += d
         secs += s
         k = (k + per_step) % args.streams
@@ -345,7 +353,7 @@ def workload_spec(kind: str, streams: int, rank: int):
     return spec
 
 
-def setup_workload(spec, dev, table_batch: int = 256):
+def setup_workload(spec, dev, table_batch: int = 256, inflight: bool = False):
     """A generated workload on `dev`: its inputs, the resident cache index and the step's
     device buffers.  Returns (workload, scorer, step inputs, step outputs)."""
     import torch
@@ -374,7 +382,9 @@ def setup_workload(spec, dev, table_batch: int = 256):
     x = StepInputs(util=sdev.util(w, device=dev), chains=chains, chain_off=ra["chain_off"],
                    set_off=ra["set_off"], length=ra["length"], prefill=ra["prefill"],
                    snap=ra["snap"], events=ra["events"], event_off=ra["event_off"],
-                   weights=weights_tensor(w.weights, theta, spec.cap_tokens, bpt, device=dev))
+                   weights=weights_tensor(w.weights, theta, spec.cap_tokens, bpt, device=dev),
+                   arrival_us=(torch.from_numpy(w.arrival_us.astype(np.int64)).to(dev)
+                               if inflight else None))
     out = sc.alloc_outputs(x.n_snap, x.R, x.n_streams)
     return w, sc, x, out
 
@@ -414,8 +424,9 @@ def run_netkv(args):
     from paper_2606_03910_gb300.pipeline import StepInputs
 
     w, sc, x, out = setup_workload(workload_spec(args.workload, args.streams, rank), dev,
-                                   args.table_batch)
+                                   args.table_batch, inflight=args.inflight > 0)
     sc.share_prefixes = not args.no_share
+    sc.inflight_cap = args.inflight
     theta = float(np.float32(synth.THETA_S_PER_TOKEN))
     bpt = synth.BYTES_PER_TOKEN_SHARD
     spec = w.spec
@@ -458,7 +469,8 @@ def run_netkv(args):
     R, D = x.R, sc.D
     # level bottlenecks 1; prefix match 4 (group insert, group resolve, leaders, members)
     # with a workspace or 1 without; greedy 2 (base scores + walk) with a workspace or 1
-    launches_per_step = 1 + (4 if sc.share_prefixes else 1) + (2 if sc.precompute_scores else 1)
+    launches_per_step = 1 + (4 if sc.share_prefixes else 1) + (
+        1 if sc.inflight_cap > 0 else (2 if sc.precompute_scores else 1))
     n_input_tensors = sum(1 for f in dataclasses.fields(StepInputs)
                           if isinstance(getattr(x, f.name), torch.Tensor))
     decisions = R * world
@@ -534,7 +546,7 @@ def run_netkv(args):
     if rank == 0 and world == 1 and not args.no_cpu and args.workload == "replicas":
         sample = np.random.default_rng(0).choice(args.streams, size=min(args.cpu_streams, args.streams),
                                                  replace=False)
-        d, secs = cpu_oracle_sample(w, sample, theta, spec.cap_tokens, bpt)
+        d, secs = cpu_oracle_sample(w, sample, theta, spec.cap_tokens, bpt, args.inflight)
         cpu = {"value": d / secs, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                "sample": f"{len(sample)} of {args.streams} streams, whole streams "
                          f"({d} decisions in {secs:.1f} s)"}
@@ -551,7 +563,9 @@ def run_netkv(args):
                 "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                 "dtype": "f32", "data": "synthetic",
-                "config": workload_config(args.streams, world, kind=args.workload),
+                "config": workload_config(args.streams, world, kind=args.workload,
+                                          extra={"inflight_cap": args.inflight}
+                                          if args.inflight else None),
                 "scores_per_s": value * D, "gpu_launches": launches_per_step * args.steps,
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk}
         print(json.dumps(line), flush=True)

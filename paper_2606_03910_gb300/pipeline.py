@@ -8,6 +8,7 @@ CUDA stream:
 2. ``netkv_prefix_match``  -> M[r][d] for every request and decode (with a
    workspace, so that requests sharing a prefix share the probing)
 3. ``netkv_schedule_streams`` -> decisions, best/second scores, final loads
+   (``netkv_schedule_streams_inflight`` when ``inflight_cap`` > 0: self-contention)
 
 ``step_host`` is the same step from host buffers: it copies the step's inputs
 host->device (``netkv_copy_async``: SM-driven reads of pinned host memory), runs
@@ -38,6 +39,7 @@ class StepInputs:
     event_off: torch.Tensor   # i64 [n_streams+1]
     weights: torch.Tensor     # u8 [n_streams * 32] (netkv_weights)
     load_init: Optional[torch.Tensor] = None
+    arrival_us: Optional[torch.Tensor] = None  # i64 [R], for self-contention
 
     @property
     def R(self) -> int:
@@ -65,6 +67,7 @@ class StepOutputs:
     second: torch.Tensor      # f32 [R]
     load_final: torch.Tensor  # i64 [n_streams, D]
     status: torch.Tensor      # i32 [1]
+    xfer_us: Optional[torch.Tensor] = None  # i32 [R], with self-contention
 
 
 class Scorer:
@@ -85,6 +88,8 @@ class Scorer:
         self.workspace = None
         self.precompute_scores = True
         self.sched_workspace = None
+        # self-contention counter cap (Eq. 4's n_inflight); 0 = the plain greedy
+        self.inflight_cap = 0
 
     def _sched_workspace(self, R: int):
         """Greedy workspace (base scores of every arrival), grown on demand."""
@@ -124,7 +129,8 @@ class Scorer:
             best=torch.empty(R, dtype=torch.float32, device=dev),
             second=torch.empty(R, dtype=torch.float32, device=dev),
             load_final=torch.empty((n_streams, self.D), dtype=torch.int64, device=dev),
-            status=torch.zeros(1, dtype=torch.int32, device=dev))
+            status=torch.zeros(1, dtype=torch.int32, device=dev),
+            xfer_us=torch.empty(R, dtype=torch.int32, device=dev))
 
     def oracle_build(self, x: StepInputs, out: StepOutputs, stream=None) -> None:
         netkv.netkv_oracle_build(self.topo, x.util, x.n_snap, 1.0, None, out.UB, out.status, stream)
@@ -135,6 +141,13 @@ class Scorer:
                                  out.status, stream, workspace=self._workspace(x.R))
 
     def schedule(self, x: StepInputs, out: StepOutputs, stream=None) -> None:
+        if self.inflight_cap > 0:
+            netkv.netkv_schedule_streams_inflight(
+                self.topo, x.n_streams, x.weights, x.R, x.length, x.prefill, x.snap,
+                x.arrival_us, out.M, out.UB, x.n_snap, x.events, x.event_off, self.inflight_cap,
+                x.load_init, out.dec, out.best, out.second, out.xfer_us, out.load_final,
+                out.status, stream)
+            return
         netkv.netkv_schedule_streams(self.topo, x.n_streams, x.weights, x.R, x.length, x.prefill,
                                      x.snap, out.M, out.UB, x.n_snap, x.events, x.event_off,
                                      x.load_init, out.dec, out.best, out.second, out.load_final,

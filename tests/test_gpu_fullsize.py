@@ -51,3 +51,44 @@ def test_bench_workload_repeatable(fullsize):
     sc.step(x, out)
     torch.cuda.synchronize()
     assert torch.equal(out.dec, dec) and torch.equal(out.M, M) and torch.equal(out.best, best)
+
+
+def test_bench_workload_with_self_contention(fullsize):
+    """bench.py --inflight 16: the same workload and step with the self-contention greedy
+    (counter cap 16, the paper's default); three whole streams against the oracle with
+    decisions and transfer times exact (near-ties and one-microsecond roundings replayed
+    and counted), scores within 1e-5 and final loads exact."""
+    import dataclasses
+    import synth
+    from oracle.workload import run_stream_inflight
+    from tests.gpu_common import THETA, host, rel_close
+    w, sc, x, out = fullsize
+    x2 = dataclasses.replace(x, arrival_us=torch.from_numpy(w.arrival_us.astype(np.int64)).cuda())
+    o = sc.alloc_outputs(x.n_snap, x.R, x.n_streams)
+    sc.inflight_cap = 16
+    try:
+        sc.step(x2, o)
+        torch.cuda.synchronize()
+    finally:
+        sc.inflight_cap = 0
+    assert int(o.status.item()) == 0
+    assert torch.equal(o.M, out.M)
+    dec, xfer = host(o.dec), host(o.xfer_us)
+    best, second, load = host(o.best), host(o.second), host(o.load_final)
+    near = adopted = 0
+    for s in (0, 2047, 4095):
+        r0, r1 = int(w.req_off[s]), int(w.req_off[s + 1])
+        res = run_stream_inflight(w, s, THETA, w.spec.cap_tokens, synth.BYTES_PER_TOKEN_SHARD, 16,
+                                  hint=dec[r0:r1], xfer_hint=xfer[r0:r1],
+                                  M=host(out.M[r0:r1]).view(np.uint16))
+        assert res.mismatches == 0 and res.xfer_mismatches == 0
+        np.testing.assert_array_equal(res.dec, dec[r0:r1])
+        np.testing.assert_array_equal(res.xfer_us, xfer[r0:r1])
+        ev = w.events[w.event_off[s]:w.event_off[s + 1]]
+        arr = (ev[(ev >> 31) == 0] & 0x7FFFFFFF).astype(np.int64) - r0
+        assert rel_close(best[r0:r1][arr], res.best[arr]).all()
+        assert rel_close(second[r0:r1][arr], res.second[arr]).all()
+        np.testing.assert_array_equal(load[s], res.load)
+        near += res.near_ties
+        adopted += res.xfer_adopted
+    assert near <= 5 and adopted <= 5
