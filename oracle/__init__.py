@@ -70,8 +70,12 @@ def _declare(l):
     l.oracle_prefix_match_one.restype = None
     l.oracle_prefix_match_one.argtypes = [P, U64, P, P, U64, P]
     l.oracle_schedule_stream.restype = None
-    l.oracle_schedule_stream.argtypes = [P, P, P, P, P, U64, P, P, P, P, P, U64, F64, F64, F64,
+    l.oracle_schedule_stream.argtypes = [P, P, P, P, P, P, U64, P, P, P, P, P, U64, F64, F64, F64,
                                          F64, I64, U64, P, P, F64, P, P, P, P, P]
+    l.oracle_cost_matrix_directed.restype = None
+    l.oracle_cost_matrix_directed.argtypes = [P, P, P, P, P, P, U64, U64, F64, P]
+    l.oracle_level_bottleneck_directed.restype = None
+    l.oracle_level_bottleneck_directed.argtypes = [P, P, P, P, P, U64, U64, P]
     l.oracle_schedule_stream_inflight.restype = None
     l.oracle_schedule_stream_inflight.argtypes = [P, P, P, P, P, U64, P, P, P, P, P, P, U64,
                                                   F64, F64, F64, F64, I64, U64, U32, P, P, P,
@@ -145,6 +149,32 @@ def cost_entries(fanout, role, bw, lat, util, s, p, d, kv_bytes) -> np.ndarray:
     return out
 
 
+def cost_matrix_directed(fanout, role, bw, lat, util_up, util_down, kv_bytes) -> np.ndarray:
+    """C[s][p][d] with directed links: the prefill's links at their upward utilisation,
+    the decode's at their downward one."""
+    f, ro = _c(fanout, np.uint32), _c(role, np.uint8)
+    b, la = _c(bw, np.float64), _c(lat, np.float64)
+    uu, ud = _c(util_up, np.float32), _c(util_down, np.float32)
+    assert uu.shape == ud.shape
+    S, L = uu.shape
+    P = int((ro == 0).sum()); D = int((ro == 1).sum())
+    out = np.zeros((S, P, D), np.float64)
+    lib().oracle_cost_matrix_directed(_p(f), _p(ro), _p(b), _p(la), _p(uu), _p(ud), L, S,
+                                      float(kv_bytes), _p(out))
+    return out
+
+
+def level_bottleneck_directed(fanout, role, bw, util_up, util_down) -> np.ndarray:
+    """UB[s][i][k] with directed links: prefill instances at upward, decode instances at
+    downward utilisation."""
+    f, ro, b = _c(fanout, np.uint32), _c(role, np.uint8), _c(bw, np.float64)
+    uu, ud = _c(util_up, np.float32), _c(util_down, np.float32)
+    S, L = uu.shape
+    out = np.zeros((S, len(ro), 4), np.float64)
+    lib().oracle_level_bottleneck_directed(_p(f), _p(ro), _p(b), _p(uu), _p(ud), L, S, _p(out))
+    return out
+
+
 def up_bottleneck(fanout, bw, util) -> np.ndarray:
     f, b, u = _c(fanout, np.uint32), _c(bw, np.float64), _c(util, np.float32)
     S, L = u.shape
@@ -184,7 +214,8 @@ class StreamResult:
 
 def schedule_stream(fanout, role, bw, lat, util, length, prefill, snap, M, events,
                     w_net, w_prefix, w_load, theta, cap, bytes_per_token,
-                    load_init=None, hint=None, rel_tol=1e-5, dec_inout=None) -> StreamResult:
+                    load_init=None, hint=None, rel_tol=1e-5, dec_inout=None,
+                    util_down=None) -> StreamResult:
     """Run one stream's events.  Arrays are indexed by global request index r.
 
     ``dec_inout`` (int32 [R]) carries decisions across streams that share request
@@ -204,7 +235,9 @@ def schedule_stream(fanout, role, bw, lat, util, length, prefill, snap, M, event
     counts = np.zeros(3, np.int64)
     li = None if load_init is None else _c(load_init, np.int64)
     h = None if hint is None else _c(hint, np.int32)
-    lib().oracle_schedule_stream(_p(f), _p(ro), _p(b), _p(la), _p(u), u.shape[1], _p(ln), _p(pf),
+    ud = None if util_down is None else _c(util_down, np.float32)
+    assert ud is None or ud.shape == u.shape
+    lib().oracle_schedule_stream(_p(f), _p(ro), _p(b), _p(la), _p(u), _p(ud), u.shape[1], _p(ln), _p(pf),
                                  _p(sn), _p(m), _p(ev), len(ev), float(w_net), float(w_prefix),
                                  float(w_load), float(theta), int(cap), int(bytes_per_token),
                                  _p(li), _p(h), float(rel_tol), _p(dec), _p(best), _p(second),

@@ -16,6 +16,9 @@
 //     self-contention count n_inflight = 0 (the paper allows n_inflight == 0 when
 //     telemetry already covers the scheduler's flows).  With one utilisation per tier
 //     this is exactly B_tau * (1 - c_tau) (Sec. III-D, per-tier collapse).
+//   * Directed links (optional): one utilisation per link and direction; a transfer
+//     climbs the source's links at their upward utilisation and descends the
+//     destination's at their downward one.
 //   * Transfer time, Eq. 3: T = s / B_eff + L_tau.
 //   * Block-level prefix hit (Sec. III-B): lambda = 16 * |LCP_block(h_r, K_d)|, the number
 //     of leading blocks of the request's hash chain that are all in decode d's cache.
@@ -93,6 +96,23 @@ double path_bottleneck(const Tree& t, const double* bw, const float* u_row,
     const uint64_t ei = uplink(t, i, h), ej = uplink(t, j, h);
     const double ri = bw[h] * (1.0 - (double)u_row[ei]);
     const double rj = bw[h] * (1.0 - (double)u_row[ej]);
+    if (ri < b) b = ri;
+    if (rj < b) b = rj;
+  }
+  if (tau_out) *tau_out = tau;
+  return b;
+}
+
+// Directed links (one utilisation per link and direction): a transfer from instance i to
+// instance j climbs i's links (their upward utilisation) and descends j's links (their
+// downward utilisation).  With u_up == u_down this is path_bottleneck.
+double path_bottleneck_dir(const Tree& t, const double* bw, const float* u_up,
+                           const float* u_down, uint64_t i, uint64_t j, int* tau_out) {
+  const int tau = tier(t, i, j);
+  double b = std::numeric_limits<double>::infinity();
+  for (int h = 0; h <= tau; ++h) {
+    const double ri = bw[h] * (1.0 - (double)u_up[uplink(t, i, h)]);
+    const double rj = bw[h] * (1.0 - (double)u_down[uplink(t, j, h)]);
     if (ri < b) b = ri;
     if (rj < b) b = rj;
   }
@@ -203,6 +223,48 @@ void oracle_up_bottleneck(const uint32_t* fanout, const double* bw, const float*
     }
 }
 
+// Directed links: the same matrix with transfers climbing the prefill's links at their
+// upward utilisation util_up and descending the decode's at their downward utilisation
+// util_down (both [n_snap][n_links]).
+void oracle_cost_matrix_directed(const uint32_t* fanout, const uint8_t* role, const double* bw,
+                                 const double* lat, const float* util_up, const float* util_down,
+                                 uint64_t n_links, uint64_t n_snap, double kv_bytes, double* C) {
+  const Tree t = make_tree(fanout);
+  std::vector<uint64_t> pre, dec;
+  ranks(role, t.n, pre, dec);
+  const uint64_t P = pre.size(), D = dec.size();
+#pragma omp parallel for collapse(2) schedule(static)
+  for (uint64_t s = 0; s < n_snap; ++s)
+    for (uint64_t p = 0; p < P; ++p)
+      for (uint64_t d = 0; d < D; ++d) {
+        int tau = 0;
+        const double b = path_bottleneck_dir(t, bw, util_up + s * n_links, util_down + s * n_links,
+                                             pre[p], dec[d], &tau);
+        C[(s * P + p) * D + d] = kv_bytes / b + lat[tau];
+      }
+}
+
+// Level bottlenecks with directed links: for a prefill instance the climb at upward
+// utilisation, for a decode instance at downward utilisation (the direction a transfer
+// crosses its links): UB[s][i][k] = min over h <= k of bw[h] * (1 - u_dir(i)[s][uplink(i,h)]).
+void oracle_level_bottleneck_directed(const uint32_t* fanout, const uint8_t* role,
+                                      const double* bw, const float* util_up,
+                                      const float* util_down, uint64_t n_links, uint64_t n_snap,
+                                      double* UB) {
+  const Tree t = make_tree(fanout);
+#pragma omp parallel for collapse(2) schedule(static)
+  for (uint64_t s = 0; s < n_snap; ++s)
+    for (uint64_t i = 0; i < t.n; ++i) {
+      const float* u = (role[i] ? util_down : util_up) + s * n_links;
+      double b = std::numeric_limits<double>::infinity();
+      for (int k = 0; k < 4; ++k) {
+        const double r = bw[k] * (1.0 - (double)u[uplink(t, i, k)]);
+        if (r < b) b = r;
+        UB[(s * t.n + i) * 4 + k] = b;
+      }
+    }
+}
+
 // ---------------------------------------------------------------- prefix match
 // M[r][d] = number of leading blocks of chain r found in cache K_{g(r),d}, where the
 // cache of (set g, decode d) is the key list keys[key_off[g*D+d] .. key_off[g*D+d+1]),
@@ -266,8 +328,11 @@ void oracle_prefix_match_one(const uint64_t* keys, uint64_t n_keys, const uint64
 //
 // best/second: the minimum score and the minimum over the other feasible candidates
 // (+inf when absent), both from the oracle's own scores.
+// util_down: NULL for undirected links, else the downward utilisation rows (util then
+// holds the upward ones).
 void oracle_schedule_stream(const uint32_t* fanout, const uint8_t* role, const double* bw,
-                            const double* lat, const float* util, uint64_t n_links,
+                            const double* lat, const float* util, const float* util_down,
+                            uint64_t n_links,
                             const uint32_t* len, const uint32_t* prefill, const uint32_t* snap,
                             const uint16_t* M, const uint32_t* events, uint64_t n_events,
                             double w_net, double w_prefix, double w_load, double theta,
@@ -293,12 +358,13 @@ void oracle_schedule_stream(const uint32_t* fanout, const uint8_t* role, const d
       continue;
     }
     const float* u_row = util + (uint64_t)snap[r] * n_links;
+    const float* d_row = util_down ? util_down + (uint64_t)snap[r] * n_links : u_row;
     const uint64_t p = pre[prefill[r]];
     int32_t arg = -1;
     for (uint64_t d = 0; d < D; ++d) {
       if (load[d] + l > cap) { score[d] = inf; continue; }
       int tau = 0;
-      const double b = path_bottleneck(t, bw, u_row, p, decs[d], &tau);
+      const double b = path_bottleneck_dir(t, bw, u_row, d_row, p, decs[d], &tau);
       const int64_t lam = 16 * (int64_t)M[(uint64_t)r * D + d];
       const double s_eff = (double)((l - lam) * (int64_t)bytes_per_token);
       const double T = s_eff / b + lat[tau];

@@ -14,7 +14,8 @@ from typing import Optional
 
 import numpy as np
 
-from . import prefix_match, schedule_stream, schedule_stream_inflight, up_bottleneck
+from . import (level_bottleneck_directed, prefix_match, schedule_stream, schedule_stream_inflight,
+               up_bottleneck)
 
 
 @dataclasses.dataclass
@@ -49,16 +50,25 @@ def stream_cache_keys(w, g: int):
     return np.concatenate(keys), off
 
 
+def _rows(w, snaps, direction):
+    if w.n_snap * w.L < (1 << 24):
+        return w.util(direction=direction)[snaps]
+    return np.stack([w.util(int(k), int(k) + 1, direction)[0] for k in snaps])
+
+
 def run_stream(w, s: int, theta: float, cap: int, bytes_per_token: int,
                hint: Optional[np.ndarray] = None, rel_tol: float = 1e-5,
-               M: Optional[np.ndarray] = None) -> OracleStream:
+               M: Optional[np.ndarray] = None, directed: bool = False) -> OracleStream:
     """Oracle for stream s of workload w (per-stream table sets and telemetry, or shared).
 
     hint: decisions of another implementation for this stream's requests (local order).
+    directed: links carry separate upward and downward utilisations (the generator's
+    "up" and "down" rows); UB is then the directed level bottleneck.
     """
     from synth import request_set
     r0, r1, ev_local, snaps, snap_local = stream_problem(w, s)
-    util = w.util()[snaps] if w.n_snap * w.L < (1 << 24) else np.stack([w.util(int(k), int(k) + 1)[0] for k in snaps])
+    util = _rows(w, snaps, "up")
+    util_down = _rows(w, snaps, "down") if directed else None
     if M is None:
         g = int(request_set(w)[r0]) if r1 > r0 else 0
         keys, key_off = stream_cache_keys(w, g)
@@ -70,8 +80,10 @@ def run_stream(w, s: int, theta: float, cap: int, bytes_per_token: int,
     spec = w.spec
     res = schedule_stream(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, util,
                           w.length[r0:r1], w.prefill[r0:r1], snap_local, M, ev_local,
-                          wn, wp, wl, theta, cap, bytes_per_token, hint=hint, rel_tol=rel_tol)
-    UB = up_bottleneck(spec.fanout, spec.tier_bw, util)
+                          wn, wp, wl, theta, cap, bytes_per_token, hint=hint, rel_tol=rel_tol,
+                          util_down=util_down)
+    UB = up_bottleneck(spec.fanout, spec.tier_bw, util) if not directed else \
+        level_bottleneck_directed(spec.fanout, w.role, spec.tier_bw, util, util_down)
     return OracleStream(r0, r1, M, res.dec, res.best, res.second, res.load, res.near_ties,
                         res.mismatches, res.rejects, snaps, UB)
 
@@ -85,7 +97,7 @@ def run_stream_inflight(w, s: int, theta: float, cap: int, bytes_per_token: int,
     for the stream's requests (local order).  The result carries xfer_us."""
     from synth import request_set
     r0, r1, ev_local, snaps, snap_local = stream_problem(w, s)
-    util = w.util()[snaps] if w.n_snap * w.L < (1 << 24) else np.stack([w.util(int(k), int(k) + 1)[0] for k in snaps])
+    util = _rows(w, snaps, "up")
     if M is None:
         g = int(request_set(w)[r0]) if r1 > r0 else 0
         keys, key_off = stream_cache_keys(w, g)

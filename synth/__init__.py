@@ -283,9 +283,9 @@ class Workload:
         """Cached block hashes of decode d in table set g (insertion list)."""
         return cache_keys(self, g, d)
 
-    def util(self, s0: int = 0, s1: Optional[int] = None) -> np.ndarray:
+    def util(self, s0: int = 0, s1: Optional[int] = None, direction: str = "up") -> np.ndarray:
         s1 = self.n_snap if s1 is None else s1
-        return utilisation(self, np.arange(s0, s1))
+        return utilisation(self, np.arange(s0, s1), direction)
 
 
 def distinct_keys_per_group(w: Workload, group: int = 64) -> int:
@@ -341,13 +341,20 @@ def cache_keys(w: Workload, g: int, d: int) -> np.ndarray:
     return np.concatenate(parts).astype(U64)
 
 
-def utilisation(w: Workload, snaps: np.ndarray) -> np.ndarray:
+DOWN_SEED = 1 << 40  # downward utilisations (directed links) draw from seed + DOWN_SEED
+
+
+def utilisation(w: Workload, snaps: np.ndarray, direction: str = "up") -> np.ndarray:
+    """Utilisation rows of snapshots `snaps`.  direction "up" is the undirected row (and
+    the upward one of directed links); "down" is an independent draw of the same
+    distribution for the downward direction."""
     spec = w.spec
     snaps = np.asarray(snaps, dtype=np.int64)
     e = np.arange(w.L, dtype=np.int64)
     out = np.empty((len(snaps), w.L), np.float32)
+    shift = 0 if direction == "up" else DOWN_SEED
     for j, s in enumerate(snaps):
-        seed = int(w.snap_seed[s])
+        seed = int(w.snap_seed[s]) + shift
         loc = int(w.snap_local[s])
         if spec.util_mode == "uniform09":
             out[j] = uniform09_f32(draw(seed, P_UTIL, loc, e))

@@ -15,7 +15,7 @@ from typing import Optional
 
 import numpy as np
 
-from . import (GOLDEN, MASK64, P_FILLER, P_ROOTHASH, P_TAIL, P_UTIL, Workload, _mix, stream_key,
+from . import (DOWN_SEED, GOLDEN, MASK64, P_FILLER, P_ROOTHASH, P_TAIL, P_UTIL, Workload, _mix, stream_key,
                U64)
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -131,14 +131,17 @@ def keys(w: Workload, g0: int = 0, g1: Optional[int] = None, device="cuda", stre
     return out
 
 
-def util(w: Workload, s0: int = 0, s1: Optional[int] = None, device="cuda", stream=None):
+def util(w: Workload, s0: int = 0, s1: Optional[int] = None, device="cuda", stream=None,
+         direction: str = "up"):
     """Utilisation rows [s0, s1) as a device fp32 tensor [s1-s0, L] (uniform modes on the
-    device; Beta rows are generated on the host and copied)."""
+    device; Beta rows are generated on the host and copied).  direction as for
+    synth.utilisation."""
     import torch
     s1 = w.n_snap if s1 is None else s1
     if w.spec.util_mode != "uniform09":
-        return torch.from_numpy(w.util(s0, s1)).to(device)
-    rk = row_keys(w.snap_seed[s0:s1], P_UTIL, w.snap_local[s0:s1])
+        return torch.from_numpy(w.util(s0, s1, direction)).to(device)
+    shift = 0 if direction == "up" else DOWN_SEED
+    rk = row_keys(w.snap_seed[s0:s1] + shift, P_UTIL, w.snap_local[s0:s1])
     d_rk = torch.from_numpy(rk.view(np.int64)).to(device)
     out = torch.empty((s1 - s0, w.L), dtype=torch.float32, device=device)
     _check(lib().synth_util_uniform09(out.data_ptr(), s1 - s0, w.L, d_rk.data_ptr(),

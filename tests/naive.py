@@ -66,6 +66,30 @@ class ExplicitTree:
             edges.append(e)
         return edges[::-1]
 
+    def path_steps(self, i: int, j: int) -> List[Tuple[int, bool]]:
+        """(edge, climbing) along the path from instance i to instance j: climbing when the
+        step goes from a vertex to one higher in the tree (instance < node < leaf < pod <
+        spine)."""
+        height = {"inst": 0, "node": 1, "leaf": 2, "pod": 3, "spine": 4}
+        src, dst = ("inst", i), ("inst", j)
+        prev = {src: None}
+        q = deque([src])
+        while q:
+            v = q.popleft()
+            if v == dst:
+                break
+            for w, e in self.adj[v]:
+                if w not in prev:
+                    prev[w] = (v, e)
+                    q.append(w)
+        steps = []
+        v = dst
+        while prev[v] is not None:
+            u, e = prev[v]
+            steps.append((e, height[v[0]] > height[u[0]]))
+            v = u
+        return steps[::-1]
+
     def tier(self, i: int, j: int) -> int:
         # the highest level among the path's edges is the tier of the pair
         return max(self.level[e] for e in self.path(i, j))
@@ -77,6 +101,13 @@ def frac(x) -> Fraction:
 
 def bottleneck(tree: ExplicitTree, bw, u_row, i, j) -> Fraction:
     return min(frac(bw[tree.level[e]]) * (1 - frac(u_row[e])) for e in tree.path(i, j))
+
+
+def bottleneck_directed(tree: ExplicitTree, bw, u_up_row, u_down_row, i, j) -> Fraction:
+    """Directed links: each step of the path from i to j at the utilisation of the
+    direction it crosses the link in."""
+    return min(frac(bw[tree.level[e]]) * (1 - frac((u_up_row if up else u_down_row)[e]))
+               for e, up in tree.path_steps(i, j))
 
 
 def cost(tree, bw, lat, u_row, i, j, kv) -> Fraction:
@@ -93,8 +124,9 @@ def lcp_blocks(chain: Sequence[int], cache: Sequence[int]) -> int:
 
 
 def greedy_exact(tree, role, bw, lat, util, length, prefill, snap, M, events,
-                 w, theta, cap, bpt):
-    """Exact-rational Algorithm 1 with the weighted score; returns (dec, best_scores)."""
+                 w, theta, cap, bpt, util_down=None):
+    """Exact-rational Algorithm 1 with the weighted score; returns (dec, best_scores).
+    util_down: downward rows for directed links (util then holds the upward ones)."""
     pre = [i for i in range(tree.n) if role[i] == 0]
     dec_inst = [i for i in range(tree.n) if role[i] == 1]
     D = len(dec_inst)
@@ -120,8 +152,9 @@ def greedy_exact(tree, role, bw, lat, util, length, prefill, snap, M, events,
                 scores.append(None)
                 continue
             miss_tok = l - 16 * int(M[r][d])
-            T = Fraction(miss_tok * bpt) / bottleneck(tree, bw, u_row, p, dec_inst[d]) \
-                + frac(lat[tree.tier(p, dec_inst[d])])
+            b = bottleneck(tree, bw, u_row, p, dec_inst[d]) if util_down is None else \
+                bottleneck_directed(tree, bw, u_row, util_down[int(snap[r])], p, dec_inst[d])
+            T = Fraction(miss_tok * bpt) / b + frac(lat[tree.tier(p, dec_inst[d])])
             scores.append(wn * T + wp * Fraction(miss_tok, l) + wl * th * load[d])
         cands = [(s, d) for d, s in enumerate(scores) if s is not None]
         if cands:

@@ -646,3 +646,115 @@ def test_inflight_completion_timing_and_cap():
     late = _worked(_worked_example_stream([0, 10, 2_000_005], rows), 1)
     assert list(late.xfer_us[:2]) == [2_000_000, 4_000_000]
     assert late.second[2] == pytest.approx(1.0, rel=1e-6)
+
+
+# ------------------------------------------------- directed links (NEXT: per direction)
+def test_directed_with_equal_rows_is_undirected():
+    """Equal upward and downward rows give the undirected matrix, level bottlenecks and
+    greedy, value for value."""
+    rng = np.random.default_rng(41)
+    for fanout in ((2, 2, 2, 2), (1, 2, 3, 2)):
+        tree = naive.ExplicitTree(fanout)
+        role = (np.arange(tree.n) % 3 == 1).astype(np.uint8)
+        bw, lat = [900e9, 400e9, 200e9, 100e9], [1e-6, 3e-6, 6e-6, 10e-6]
+        u = rng.uniform(0, 0.9, size=(3, tree.n_edges)).astype(np.float32)
+        np.testing.assert_array_equal(oracle.cost_matrix_directed(fanout, role, bw, lat, u, u, 1e9),
+                                      oracle.cost_matrix(fanout, role, bw, lat, u, 1e9))
+        np.testing.assert_array_equal(oracle.level_bottleneck_directed(fanout, role, bw, u, u),
+                                      oracle.up_bottleneck(fanout, bw, u))
+    for seed in range(10):
+        pb = _tiny_problem(seed)
+        w = (0.7, 1.1, 0.4)
+        a = _run_oracle(pb, w)
+        b = oracle.schedule_stream(pb["fanout"], pb["role"], pb["bw"], pb["lat"], pb["u"],
+                                   pb["length"], pb["prefill"], pb["snap"], pb["M"], pb["events"],
+                                   w[0], w[1], w[2], float(np.float32(1e-6)), pb["cap"], 81920,
+                                   util_down=pb["u"])
+        np.testing.assert_array_equal(a.dec, b.dec)
+        np.testing.assert_array_equal(a.best, b.best)
+
+
+def test_directed_matrix_matches_exact_rational_bfs():
+    """Every (snapshot, prefill, decode) against the exact-rational evaluator that takes
+    each step of the BFS path at the utilisation of its direction; P != D, all tiers."""
+    rng = np.random.default_rng(42)
+    for fanout, rule in (((2, 2, 2, 2), 3), ((2, 3, 2, 2), 2)):
+        tree = naive.ExplicitTree(fanout)
+        role = (np.arange(tree.n) % rule == 0).astype(np.uint8)
+        bw, lat = [900e9, 400e9, 200e9, 100e9], [1e-6, 3e-6, 6e-6, 10e-6]
+        up = rng.uniform(0, 0.95, size=(2, tree.n_edges)).astype(np.float32)
+        down = rng.uniform(0, 0.95, size=(2, tree.n_edges)).astype(np.float32)
+        C = oracle.cost_matrix_directed(fanout, role, bw, lat, up, down, 2.5e9)
+        pre = [i for i in range(tree.n) if role[i] == 0]
+        dec = [i for i in range(tree.n) if role[i] == 1]
+        taus = set()
+        for s in range(2):
+            for a, p in enumerate(pre):
+                for b, d in enumerate(dec):
+                    exact = naive.frac(2.5e9) / naive.bottleneck_directed(tree, bw, up[s], down[s], p, d) \
+                        + naive.frac(lat[tree.tier(p, d)])
+                    assert C[s, a, b] == pytest.approx(float(exact), rel=1e-14)
+                    taus.add(tree.tier(p, d))
+        assert taus == {0, 1, 2, 3}
+        # and the level bottlenecks the library's kernels consume
+        UB = oracle.level_bottleneck_directed(fanout, role, bw, up, down)
+        for s in range(2):
+            for i in range(tree.n):
+                row = up[s] if role[i] == 0 else down[s]
+                for k in range(4):
+                    climb = [naive.frac(bw[h]) * (1 - naive.frac(row[e]))
+                             for h, e in enumerate(_up_links(tree, i)[:k + 1])]
+                    assert UB[s, i, k] == pytest.approx(float(min(climb)), rel=1e-14)
+
+
+def _up_links(tree, i):
+    """Links from instance i up to the spine, level 0..3, read off the explicit tree."""
+    v, out = ("inst", i), []
+    height = {"inst": 0, "node": 1, "leaf": 2, "pod": 3, "spine": 4}
+    while v[0] != "spine":
+        for w, e in tree.adj[v]:
+            if height[w[0]] == height[v[0]] + 1:
+                out.append(e)
+                v = w
+                break
+    return out
+
+
+def test_directed_links_use_the_direction_crossed():
+    """A congested upward level-0 link of the prefill slows every transfer from it; the
+    same congestion on that link's downward direction slows none of them (the prefill
+    only sends), and on a decode's downward level-0 link only the transfers to it."""
+    fanout = (2, 2, 2, 2)
+    role = (np.arange(16) % 2).astype(np.uint8)        # even instances prefill, odd decode
+    bw, lat = [900e9, 400e9, 200e9, 100e9], [0.0] * 4
+    L = oracle.used_links(fanout)
+    base = np.zeros((1, L), np.float32)
+    clean = oracle.cost_matrix_directed(fanout, role, bw, lat, base, base, 1e9)
+    up = base.copy(); up[0, 0] = 0.99                 # instance 0's level-0 link, upward
+    C = oracle.cost_matrix_directed(fanout, role, bw, lat, up, base, 1e9)
+    np.testing.assert_allclose(C[0, 0], 1e9 / (900e9 * (1.0 - float(np.float32(0.99)))), rtol=1e-12)
+    np.testing.assert_array_equal(C[0, 1:], clean[0, 1:])
+    C = oracle.cost_matrix_directed(fanout, role, bw, lat, base, up, 1e9)
+    np.testing.assert_array_equal(C, clean)           # downward on a prefill's link: unused
+    down = base.copy(); down[0, 1] = 0.99             # instance 1 (decode rank 0), downward
+    C = oracle.cost_matrix_directed(fanout, role, bw, lat, base, down, 1e9)
+    np.testing.assert_allclose(C[0, :, 0], 1e9 / (900e9 * (1.0 - float(np.float32(0.99)))), rtol=1e-12)
+    np.testing.assert_array_equal(C[0, :, 1:], clean[0, :, 1:])
+
+
+def test_directed_greedy_matches_exact_rational_bruteforce():
+    theta = float(np.float32(1e-6))
+    for seed in range(20):
+        pb = _tiny_problem(seed)
+        down = np.random.default_rng(900 + seed).uniform(0, 0.9, size=pb["u"].shape).astype(np.float32)
+        w = tuple(float(np.float32(x)) for x in np.random.default_rng(700 + seed).uniform(0, 2, 3))
+        res = oracle.schedule_stream(pb["fanout"], pb["role"], pb["bw"], pb["lat"], pb["u"],
+                                     pb["length"], pb["prefill"], pb["snap"], pb["M"], pb["events"],
+                                     w[0], w[1], w[2], theta, pb["cap"], 81920, util_down=down)
+        dec, best, load = naive.greedy_exact(pb["tree"], pb["role"], pb["bw"], pb["lat"], pb["u"],
+                                             pb["length"], pb["prefill"], pb["snap"], pb["M"],
+                                             pb["events"], w, theta, pb["cap"], 81920, util_down=down)
+        assert list(res.dec) == dec and list(res.load) == load
+        for r in range(len(dec)):
+            if dec[r] >= 0:
+                assert res.best[r] == pytest.approx(float(best[r]), rel=1e-14)
