@@ -46,6 +46,8 @@ def parse():
                     help="replicas: the 4,096-stream scoring step (default); sweep: the "
                          "oracle-build sweep (1,000 snapshots x 2,048 x 8,192 pairs)")
     ap.add_argument("--snapshots", type=int, default=1000)
+    ap.add_argument("--directed", action="store_true",
+                    help="directed links: separate upward and downward utilisation rows")
     ap.add_argument("--inflight", type=int, default=0,
                     help="self-contention counter cap (Eq. 4's n_inflight; the paper uses 16); "
                          "0 = the plain greedy")
@@ -201,9 +203,9 @@ def measured_peaks():
 
 
 # ------------------------------------------------------------------ CPU oracle
-def cpu_oracle_sample(w, streams, theta, cap, bpt, inflight=0):
+def cpu_oracle_sample(w, streams, theta, cap, bpt, inflight=0, directed=False):
     """Time the CPU oracle on whole streams of the workload (with self-contention when
-    inflight > 0); returns (decisions, seconds)."""
+    inflight > 0, with directed links when directed); returns (decisions, seconds)."""
     from oracle.workload import run_stream, run_stream_inflight
     t0 = time.perf_counter()
     dec = 0
@@ -211,7 +213,7 @@ def cpu_oracle_sample(w, streams, theta, cap, bpt, inflight=0):
         if inflight > 0:
             res = run_stream_inflight(w, int(s), theta, cap, bpt, inflight)
         else:
-            res = run_stream(w, int(s), theta, cap, bpt)
+            res = run_stream(w, int(s), theta, cap, bpt, directed=directed)
         dec += int(res.dec.shape[0])
     return dec, time.perf_counter() - t0
 
@@ -353,7 +355,8 @@ def workload_spec(kind: str, streams: int, rank: int):
     return spec
 
 
-def setup_workload(spec, dev, table_batch: int = 256, inflight: bool = False):
+def setup_workload(spec, dev, table_batch: int = 256, inflight: bool = False,
+                   directed: bool = False):
     """A generated workload on `dev`: its inputs, the resident cache index and the step's
     device buffers.  Returns (workload, scorer, step inputs, step outputs)."""
     import torch
@@ -384,7 +387,8 @@ def setup_workload(spec, dev, table_batch: int = 256, inflight: bool = False):
                    snap=ra["snap"], events=ra["events"], event_off=ra["event_off"],
                    weights=weights_tensor(w.weights, theta, spec.cap_tokens, bpt, device=dev),
                    arrival_us=(torch.from_numpy(w.arrival_us.astype(np.int64)).to(dev)
-                               if inflight else None))
+                               if inflight else None),
+                   util_down=sdev.util(w, device=dev, direction="down") if directed else None)
     out = sc.alloc_outputs(x.n_snap, x.R, x.n_streams)
     return w, sc, x, out
 
@@ -424,7 +428,8 @@ def run_netkv(args):
     from paper_2606_03910_gb300.pipeline import StepInputs
 
     w, sc, x, out = setup_workload(workload_spec(args.workload, args.streams, rank), dev,
-                                   args.table_batch, inflight=args.inflight > 0)
+                                   args.table_batch, inflight=args.inflight > 0,
+                                   directed=args.directed)
     sc.share_prefixes = not args.no_share
     sc.inflight_cap = args.inflight
     theta = float(np.float32(synth.THETA_S_PER_TOKEN))
@@ -482,7 +487,7 @@ def run_netkv(args):
         # 8-byte chain block + 16-byte index entry per examined block, 2-byte M store
         "prefix_match": 24 * examined + 2 * R * D,
         # per snapshot: the utilisation row (L floats), 16-byte UB of every instance
-        "oracle_build": x.n_snap * (4 * w.L + 16 * sc.N),
+        "oracle_build": x.n_snap * ((8 if x.util_down is not None else 4) * w.L + 16 * sc.N),
         # per arrival: event, len/prefill/snap, per candidate base score (4 B) + the
         # dec/best/second stores; per departure: event, len, dec
         "schedule": R * (4 + 12 + 4 * D + 12) + R * 12 + 2 * 8 * D * x.n_streams,
@@ -546,7 +551,8 @@ def run_netkv(args):
     if rank == 0 and world == 1 and not args.no_cpu and args.workload == "replicas":
         sample = np.random.default_rng(0).choice(args.streams, size=min(args.cpu_streams, args.streams),
                                                  replace=False)
-        d, secs = cpu_oracle_sample(w, sample, theta, spec.cap_tokens, bpt, args.inflight)
+        d, secs = cpu_oracle_sample(w, sample, theta, spec.cap_tokens, bpt, args.inflight,
+                                    args.directed)
         cpu = {"value": d / secs, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                "sample": f"{len(sample)} of {args.streams} streams, whole streams "
                          f"({d} decisions in {secs:.1f} s)"}
@@ -564,8 +570,10 @@ def run_netkv(args):
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                 "dtype": "f32", "data": "synthetic",
                 "config": workload_config(args.streams, world, kind=args.workload,
-                                          extra={"inflight_cap": args.inflight}
-                                          if args.inflight else None),
+                                          extra=dict(([("inflight_cap", args.inflight)]
+                                                      if args.inflight else []) +
+                                                     ([("links", "directed")]
+                                                      if args.directed else [])) or None),
                 "scores_per_s": value * D, "gpu_launches": launches_per_step * args.steps,
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk}
         print(json.dumps(line), flush=True)
@@ -680,6 +688,8 @@ def run_sweep(args):
 
 def main():
     args = parse()
+    if args.inflight and args.directed:
+        raise SystemExit("--inflight and --directed are measured one at a time")
     if args.impl == "reference":
         return run_reference(args)
     if args.workload == "sweep":

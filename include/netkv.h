@@ -10,6 +10,7 @@
  *   netkv_topology_create   the four-tier instance tree (Sec. III-A, III-E)
  *   netkv_oracle_build      network cost oracle C[s][p][d] from per-link utilisation
  *                           snapshots, and the per-instance level bottlenecks UB
+ *                           (netkv_oracle_build_directed: per link and direction)
  *   netkv_cache_build       decode caches K_d as open-addressing hash tables
  *   netkv_prefix_match      block-level prefix hit M[r][d] (Sec. III-B)
  *   netkv_schedule_streams  the greedy of Algorithm 1 over independent streams
@@ -118,6 +119,20 @@ netkv_status netkv_topology_query(netkv_topology_t topo, uint32_t* n_instances, 
 netkv_status netkv_oracle_build(netkv_topology_t topo, const float* d_util, uint32_t n_snap,
                                 double kv_bytes, float* d_C, float* d_UB, int* d_status,
                                 netkv_stream_t stream);
+
+/* The same with directed links (the per-link generalisation of Eq. 4's c_tau, one
+ * utilisation per link and direction): a transfer from prefill p to decode d climbs p's
+ * links at their upward utilisation and descends d's at their downward utilisation,
+ *     C[s][p][d] = kv_bytes / min(UB[s][p][tau], UB[s][d][tau]) + L_tau
+ * with UB of a prefill instance computed from d_util_up and of a decode instance from
+ * d_util_down (both [n_snap][n_links], same layout and domain as d_util above).  UB
+ * keeps its layout, so netkv_schedule_streams consumes it unchanged.  With equal rows
+ * the results are those of netkv_oracle_build.
+ */
+netkv_status netkv_oracle_build_directed(netkv_topology_t topo, const float* d_util_up,
+                                         const float* d_util_down, uint32_t n_snap,
+                                         double kv_bytes, float* d_C, float* d_UB,
+                                         int* d_status, netkv_stream_t stream);
 
 /* ------------------------------------------------------------------ caches
  * Decode caches K_d (Sec. III-C), the sets of block hashes each decode instance holds.

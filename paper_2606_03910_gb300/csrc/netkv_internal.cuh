@@ -17,6 +17,7 @@ struct netkv_topology {
   uint4* d_links;      // [N] (level-0, level-1, level-2, level-3 link of instance i)
   uint32_t* d_pre;     // [P] instance of prefill rank p
   uint32_t* d_dec;     // [D] instance of decode rank d
+  uint8_t* d_role;     // [N] 0 = prefill, 1 = decode
 };
 
 // fp32 constants of a topology passed to kernels by value
@@ -24,6 +25,7 @@ struct TopoArgs {
   const uint4* links;
   const uint32_t* pre;
   const uint32_t* dec;
+  const uint8_t* role;
   uint32_t N, P, D, n_links;
   float bw[4];
   float lat[4];
@@ -34,6 +36,7 @@ inline TopoArgs topo_args(const netkv_topology* t) {
   a.links = t->d_links;
   a.pre = t->d_pre;
   a.dec = t->d_dec;
+  a.role = t->d_role;
   a.N = t->N;
   a.P = t->P;
   a.D = t->D;

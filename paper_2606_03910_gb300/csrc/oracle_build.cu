@@ -1,7 +1,9 @@
 // Network cost oracle (Sec. III-D Eq. 3 and Eq. 4, Sec. III-E) with per-link congestion.
 //
 // level_bottleneck_kernel: UB[s][i][k] = min_{h<=k} B_h (1 - u[s][link_h(i)]), one
-//   thread per (snapshot, instance), one 16-byte store each.
+//   thread per (snapshot, instance), one 16-byte store each.  With directed links
+//   (kDir) a prefill instance's climb reads the upward row and a decode instance's the
+//   downward row: the directions a transfer from prefill to decode crosses them in.
 // oracle_build_kernel: C[s][p][d] = kv / min(UB[s][p][tau], UB[s][d][tau]) + L_tau.
 //   Division is monotone (correctly rounded, positive operands), so
 //   kv / min(a, b) == max(kv / a, kv / b) exactly; each block therefore divides once per
@@ -41,23 +43,27 @@ __device__ __forceinline__ float4 quotients(float kv, const float4& b) {
   return make_float4(kv / b.x, kv / b.y, kv / b.z, kv / b.w);
 }
 
+template <bool kDir>
 __global__ void __launch_bounds__(kBlock) level_bottleneck_kernel(
-    TopoArgs t, const float* __restrict__ util, uint32_t n_snap, float4* __restrict__ UB,
-    int* status) {
+    TopoArgs t, const float* __restrict__ util, const float* __restrict__ util_down,
+    uint32_t n_snap, float4* __restrict__ UB, int* status) {
   const uint64_t total = (uint64_t)n_snap * t.N;
   for (uint64_t idx = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
        idx += (uint64_t)gridDim.x * blockDim.x) {
     const uint64_t s = idx / t.N;
     const uint32_t i = (uint32_t)(idx - s * t.N);
     const uint4 l = __ldg(t.links + i);
-    UB[idx] = level_bottlenecks(t, util + s * t.n_links, l, status);
+    const float* rows = (kDir && __ldg(t.role + i)) ? util_down : util;
+    UB[idx] = level_bottlenecks(t, rows + s * t.n_links, l, status);
   }
 }
 
+// util_down: the decode side's rows (the downward utilisations of directed links; the
+// same pointer as util for undirected links).
 template <bool kVec>
 __global__ void __launch_bounds__(kBlock) oracle_build_kernel(
-    TopoArgs t, const float* __restrict__ util, uint32_t n_snap, float kv, float* __restrict__ C,
-    int* status) {
+    TopoArgs t, const float* __restrict__ util, const float* __restrict__ util_down,
+    uint32_t n_snap, float kv, float* __restrict__ C, int* status) {
   __shared__ float4 s_q[kPTile];
   __shared__ uint4 s_l[kPTile];
   const float4 lat = make_float4(t.lat[0], t.lat[1], t.lat[2], t.lat[3]);
@@ -65,6 +71,7 @@ __global__ void __launch_bounds__(kBlock) oracle_build_kernel(
 
   for (uint32_t s = blockIdx.y; s < n_snap; s += gridDim.y) {
     const float* row = util + (uint64_t)s * t.n_links;
+    const float* row_d = util_down + (uint64_t)s * t.n_links;
     uint4 ld[kPerThread];
     float4 qd[kPerThread];
 #pragma unroll
@@ -72,7 +79,7 @@ __global__ void __launch_bounds__(kBlock) oracle_build_kernel(
       const uint32_t d = d0 + j;
       if (d < t.D) {
         ld[j] = __ldg(t.links + __ldg(t.dec + d));
-        qd[j] = quotients(kv, level_bottlenecks(t, row, ld[j], status));
+        qd[j] = quotients(kv, level_bottlenecks(t, row_d, ld[j], status));
       } else {
         ld[j] = make_uint4(0, 0, 0, 0);
         qd[j] = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -113,12 +120,13 @@ __global__ void __launch_bounds__(kBlock) oracle_build_kernel(
 
 }  // namespace
 
-extern "C" netkv_status netkv_oracle_build(netkv_topology_t topo, const float* d_util,
-                                           uint32_t n_snap, double kv_bytes, float* d_C,
-                                           float* d_UB, int* d_status, netkv_stream_t stream) {
-  if (!topo || !d_util || (!d_C && !d_UB)) return NETKV_EINVAL;
+static netkv_status oracle_build(netkv_topology_t topo, const float* d_util, const float* d_util_down,
+                          bool directed, uint32_t n_snap, double kv_bytes, float* d_C,
+                          float* d_UB, int* d_status, netkv_stream_t stream) {
+  if (!topo || !d_util || !d_util_down || (!d_C && !d_UB)) return NETKV_EINVAL;
   if (!(kv_bytes > 0) || !(kv_bytes < 3.0e38)) return NETKV_EINVAL;
-  if (!aligned_to(d_util, 4) || (d_C && !aligned_to(d_C, 4)) || (d_UB && !aligned_to(d_UB, 16)))
+  if (!aligned_to(d_util, 4) || !aligned_to(d_util_down, 4) || (d_C && !aligned_to(d_C, 4)) ||
+      (d_UB && !aligned_to(d_UB, 16)))
     return NETKV_EINVAL;
   if (n_snap == 0) return NETKV_OK;
   const TopoArgs t = topo_args(topo);
@@ -127,20 +135,38 @@ extern "C" netkv_status netkv_oracle_build(netkv_topology_t topo, const float* d
     const uint64_t total = (uint64_t)n_snap * t.N;
     const uint64_t blocks = (total + kBlock - 1) / kBlock;
     const unsigned grid = (unsigned)(blocks < (1u << 20) ? blocks : (1u << 20));
-    level_bottleneck_kernel<<<grid, kBlock, 0, s>>>(t, d_util, n_snap,
-                                                    reinterpret_cast<float4*>(d_UB), d_status);
+    if (directed)
+      level_bottleneck_kernel<true><<<grid, kBlock, 0, s>>>(
+          t, d_util, d_util_down, n_snap, reinterpret_cast<float4*>(d_UB), d_status);
+    else
+      level_bottleneck_kernel<false><<<grid, kBlock, 0, s>>>(
+          t, d_util, d_util, n_snap, reinterpret_cast<float4*>(d_UB), d_status);
     if (netkv_launch_status() != NETKV_OK) return NETKV_ECUDA;
   }
   if (d_C) {
     const dim3 grid((t.D + kDChunk - 1) / kDChunk, n_snap < 65535u ? n_snap : 65535u);
     const bool vec = (t.D % 4 == 0) && aligned_to(d_C, 16);
     if (vec)
-      oracle_build_kernel<true><<<grid, kBlock, 0, s>>>(t, d_util, n_snap, (float)kv_bytes, d_C,
-                                                        d_status);
+      oracle_build_kernel<true><<<grid, kBlock, 0, s>>>(t, d_util, d_util_down, n_snap,
+                                                        (float)kv_bytes, d_C, d_status);
     else
-      oracle_build_kernel<false><<<grid, kBlock, 0, s>>>(t, d_util, n_snap, (float)kv_bytes, d_C,
-                                                         d_status);
+      oracle_build_kernel<false><<<grid, kBlock, 0, s>>>(t, d_util, d_util_down, n_snap,
+                                                         (float)kv_bytes, d_C, d_status);
     if (netkv_launch_status() != NETKV_OK) return NETKV_ECUDA;
   }
   return NETKV_OK;
+}
+
+extern "C" netkv_status netkv_oracle_build(netkv_topology_t topo, const float* d_util,
+                                           uint32_t n_snap, double kv_bytes, float* d_C,
+                                           float* d_UB, int* d_status, netkv_stream_t stream) {
+  return oracle_build(topo, d_util, d_util, false, n_snap, kv_bytes, d_C, d_UB, d_status, stream);
+}
+
+extern "C" netkv_status netkv_oracle_build_directed(netkv_topology_t topo, const float* d_util_up,
+                                                    const float* d_util_down, uint32_t n_snap,
+                                                    double kv_bytes, float* d_C, float* d_UB,
+                                                    int* d_status, netkv_stream_t stream) {
+  return oracle_build(topo, d_util_up, d_util_down, true, n_snap, kv_bytes, d_C, d_UB, d_status,
+                      stream);
 }

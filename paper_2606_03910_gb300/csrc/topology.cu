@@ -59,14 +59,16 @@ extern "C" netkv_status netkv_topology_create(const netkv_topology_desc* desc,
   if (cudaGetDevice(&t->device) != cudaSuccess ||
       cudaMalloc(&t->d_links, sizeof(uint4) * N) != cudaSuccess ||
       cudaMalloc(&t->d_pre, sizeof(uint32_t) * t->P) != cudaSuccess ||
-      cudaMalloc(&t->d_dec, sizeof(uint32_t) * t->D) != cudaSuccess) {
+      cudaMalloc(&t->d_dec, sizeof(uint32_t) * t->D) != cudaSuccess ||
+      cudaMalloc(&t->d_role, N) != cudaSuccess) {
     st = NETKV_ENOMEM;
   } else if (cudaMemcpy(t->d_links, links.data(), sizeof(uint4) * N,
                         cudaMemcpyHostToDevice) != cudaSuccess ||
              cudaMemcpy(t->d_pre, pre.data(), sizeof(uint32_t) * t->P,
                         cudaMemcpyHostToDevice) != cudaSuccess ||
              cudaMemcpy(t->d_dec, dec.data(), sizeof(uint32_t) * t->D,
-                        cudaMemcpyHostToDevice) != cudaSuccess) {
+                        cudaMemcpyHostToDevice) != cudaSuccess ||
+             cudaMemcpy(t->d_role, desc->role, N, cudaMemcpyHostToDevice) != cudaSuccess) {
     st = NETKV_ECUDA;
   }
   if (st != NETKV_OK) {
@@ -83,6 +85,7 @@ extern "C" netkv_status netkv_topology_destroy(netkv_topology_t t) {
   cudaFree(t->d_links);
   cudaFree(t->d_pre);
   cudaFree(t->d_dec);
+  cudaFree(t->d_role);
   free(t);
   return NETKV_OK;
 }

@@ -40,6 +40,7 @@ class StepInputs:
     weights: torch.Tensor     # u8 [n_streams * 32] (netkv_weights)
     load_init: Optional[torch.Tensor] = None
     arrival_us: Optional[torch.Tensor] = None  # i64 [R], for self-contention
+    util_down: Optional[torch.Tensor] = None   # f32 [n_snap, n_links], directed links
 
     @property
     def R(self) -> int:
@@ -133,6 +134,10 @@ class Scorer:
             xfer_us=torch.empty(R, dtype=torch.int32, device=dev))
 
     def oracle_build(self, x: StepInputs, out: StepOutputs, stream=None) -> None:
+        if x.util_down is not None:  # directed links: util holds the upward rows
+            netkv.netkv_oracle_build_directed(self.topo, x.util, x.util_down, x.n_snap, 1.0, None,
+                                              out.UB, out.status, stream)
+            return
         netkv.netkv_oracle_build(self.topo, x.util, x.n_snap, 1.0, None, out.UB, out.status, stream)
 
     def prefix_match(self, x: StepInputs, out: StepOutputs, stream=None) -> None:

@@ -32,8 +32,9 @@ def make_scorer(w, device="cuda"):
                   index_log2(w), device=device)
 
 
-def run_gpu(w, sc=None, cap=None, load_init=None):
-    """Whole path on the GPU for workload w; returns (scorer, inputs, outputs)."""
+def run_gpu(w, sc=None, cap=None, load_init=None, directed=False):
+    """Whole path on the GPU for workload w; returns (scorer, inputs, outputs).
+    directed: links carry the generator's upward and downward utilisation rows."""
     import torch
     from paper_2606_03910_gb300.pipeline import StepInputs, weights_tensor
     sc = sc or make_scorer(w)
@@ -45,7 +46,8 @@ def run_gpu(w, sc=None, cap=None, load_init=None):
                    set_off=ra["set_off"], length=ra["length"], prefill=ra["prefill"],
                    snap=ra["snap"], events=ra["events"], event_off=ra["event_off"],
                    weights=weights_tensor(w.weights, THETA, cap, synth.BYTES_PER_TOKEN_SHARD),
-                   load_init=load_init)
+                   load_init=load_init,
+                   util_down=stage.util(w, direction="down") if directed else None)
     out = sc.alloc_outputs(x.n_snap, x.R, x.n_streams)
     sc.step(x, out)
     torch.cuda.synchronize()
@@ -56,7 +58,7 @@ def host(t):
     return t.detach().cpu().numpy()
 
 
-def check_stream(w, s, out, cap=None, M_gpu=None, M_expect=None):
+def check_stream(w, s, out, cap=None, M_gpu=None, M_expect=None, directed=False):
     """Oracle on stream s with the GPU decisions as near-tie hints; asserts parity.
     M_expect: the stream's prefix hits for the oracle's greedy where its own per-stream
     cache sets would not fit (the generator's constructed hits).  Returns the oracle result."""
@@ -65,7 +67,8 @@ def check_stream(w, s, out, cap=None, M_gpu=None, M_expect=None):
     import torch
     r0, r1 = int(w.req_off[s]), int(w.req_off[s + 1])
     dec = host(out.dec[r0:r1])
-    res = run_stream(w, s, THETA, cap, synth.BYTES_PER_TOKEN_SHARD, hint=dec, M=M_expect)
+    res = run_stream(w, s, THETA, cap, synth.BYTES_PER_TOKEN_SHARD, hint=dec, M=M_expect,
+                     directed=directed)
     # prefix hits: bit-exact
     if M_gpu is None:
         M_gpu = host(out.M[r0:r1]).view(np.uint16)
