@@ -70,8 +70,10 @@ def _declare(l):
     l.oracle_prefix_match_one.restype = None
     l.oracle_prefix_match_one.argtypes = [P, U64, P, P, U64, P]
     l.oracle_schedule_stream.restype = None
-    l.oracle_schedule_stream.argtypes = [P, P, P, P, P, P, U64, P, P, P, P, P, U64, F64, F64, F64,
-                                         F64, I64, U64, P, P, F64, P, P, P, P, P]
+    l.oracle_schedule_stream.argtypes = [P, P, P, P, P, P, INT, U64, P, P, P, P, P, U64, F64, F64,
+                                         F64, F64, I64, U64, P, P, F64, P, P, P, P, P]
+    l.oracle_cost_matrix_tiers.restype = None
+    l.oracle_cost_matrix_tiers.argtypes = [P, P, P, P, P, U64, F64, P]
     l.oracle_cost_matrix_directed.restype = None
     l.oracle_cost_matrix_directed.argtypes = [P, P, P, P, P, P, U64, U64, F64, P]
     l.oracle_level_bottleneck_directed.restype = None
@@ -164,6 +166,19 @@ def cost_matrix_directed(fanout, role, bw, lat, util_up, util_down, kv_bytes) ->
     return out
 
 
+def cost_matrix_tiers(fanout, role, bw, lat, c, kv_bytes) -> np.ndarray:
+    """C[s][p][d] of the paper-literal per-tier oracle: kv / (B_tau (1 - c[s][tau])) + L_tau."""
+    f, ro = _c(fanout, np.uint32), _c(role, np.uint8)
+    b, la = _c(bw, np.float64), _c(lat, np.float64)
+    cc = _c(c, np.float32)
+    S = cc.shape[0]
+    assert cc.shape == (S, 4)
+    P = int((ro == 0).sum()); D = int((ro == 1).sum())
+    out = np.zeros((S, P, D), np.float64)
+    lib().oracle_cost_matrix_tiers(_p(f), _p(ro), _p(b), _p(la), _p(cc), S, float(kv_bytes), _p(out))
+    return out
+
+
 def level_bottleneck_directed(fanout, role, bw, util_up, util_down) -> np.ndarray:
     """UB[s][i][k] with directed links: prefill instances at upward, decode instances at
     downward utilisation."""
@@ -215,7 +230,7 @@ class StreamResult:
 def schedule_stream(fanout, role, bw, lat, util, length, prefill, snap, M, events,
                     w_net, w_prefix, w_load, theta, cap, bytes_per_token,
                     load_init=None, hint=None, rel_tol=1e-5, dec_inout=None,
-                    util_down=None) -> StreamResult:
+                    util_down=None, tier_mode=False) -> StreamResult:
     """Run one stream's events.  Arrays are indexed by global request index r.
 
     ``dec_inout`` (int32 [R]) carries decisions across streams that share request
@@ -237,7 +252,9 @@ def schedule_stream(fanout, role, bw, lat, util, length, prefill, snap, M, event
     h = None if hint is None else _c(hint, np.int32)
     ud = None if util_down is None else _c(util_down, np.float32)
     assert ud is None or ud.shape == u.shape
-    lib().oracle_schedule_stream(_p(f), _p(ro), _p(b), _p(la), _p(u), _p(ud), u.shape[1], _p(ln), _p(pf),
+    assert not tier_mode or u.shape[1] == 4
+    lib().oracle_schedule_stream(_p(f), _p(ro), _p(b), _p(la), _p(u), _p(ud), int(bool(tier_mode)),
+                                 u.shape[1], _p(ln), _p(pf),
                                  _p(sn), _p(m), _p(ev), len(ev), float(w_net), float(w_prefix),
                                  float(w_load), float(theta), int(cap), int(bytes_per_token),
                                  _p(li), _p(h), float(rel_tol), _p(dec), _p(best), _p(second),

@@ -16,6 +16,8 @@
 //     self-contention count n_inflight = 0 (the paper allows n_inflight == 0 when
 //     telemetry already covers the scheduler's flows).  With one utilisation per tier
 //     this is exactly B_tau * (1 - c_tau) (Sec. III-D, per-tier collapse).
+//   * Paper-literal per-tier mode (Sec. III-E): B_eff = B_tau * (1 - c_tau) from four
+//     per-tier congestion values, no minimum over a path's lower levels.
 //   * Directed links (optional): one utilisation per link and direction; a transfer
 //     climbs the source's links at their upward utilisation and descends the
 //     destination's at their downward one.
@@ -265,6 +267,27 @@ void oracle_level_bottleneck_directed(const uint32_t* fanout, const uint8_t* rol
     }
 }
 
+// Paper-literal per-tier oracle (Sec. III-E, Eq. 4 with n_inflight = 0): the four maps
+// tier tau(p,d), bandwidth B_tau, congestion c_tau and latency L_tau, so that a pair's
+// bandwidth is B_tau * (1 - c_tau) with no minimum over the lower levels of its path.
+// c: [n_snap][4] per-tier congestion.
+void oracle_cost_matrix_tiers(const uint32_t* fanout, const uint8_t* role, const double* bw,
+                              const double* lat, const float* c, uint64_t n_snap,
+                              double kv_bytes, double* C) {
+  const Tree t = make_tree(fanout);
+  std::vector<uint64_t> pre, dec;
+  ranks(role, t.n, pre, dec);
+  const uint64_t P = pre.size(), D = dec.size();
+#pragma omp parallel for collapse(2) schedule(static)
+  for (uint64_t s = 0; s < n_snap; ++s)
+    for (uint64_t p = 0; p < P; ++p)
+      for (uint64_t d = 0; d < D; ++d) {
+        const int tau = tier(t, pre[p], dec[d]);
+        const double b = bw[tau] * (1.0 - (double)c[s * 4 + tau]);
+        C[(s * P + p) * D + d] = kv_bytes / b + lat[tau];
+      }
+}
+
 // ---------------------------------------------------------------- prefix match
 // M[r][d] = number of leading blocks of chain r found in cache K_{g(r),d}, where the
 // cache of (set g, decode d) is the key list keys[key_off[g*D+d] .. key_off[g*D+d+1]),
@@ -329,10 +352,11 @@ void oracle_prefix_match_one(const uint64_t* keys, uint64_t n_keys, const uint64
 // best/second: the minimum score and the minimum over the other feasible candidates
 // (+inf when absent), both from the oracle's own scores.
 // util_down: NULL for undirected links, else the downward utilisation rows (util then
-// holds the upward ones).
+// holds the upward ones).  tier_mode: util holds per-tier congestion rows c[4] (n_links
+// = 4) and a pair's bandwidth is B_tau * (1 - c_tau), the paper-literal oracle.
 void oracle_schedule_stream(const uint32_t* fanout, const uint8_t* role, const double* bw,
                             const double* lat, const float* util, const float* util_down,
-                            uint64_t n_links,
+                            int tier_mode, uint64_t n_links,
                             const uint32_t* len, const uint32_t* prefill, const uint32_t* snap,
                             const uint16_t* M, const uint32_t* events, uint64_t n_events,
                             double w_net, double w_prefix, double w_load, double theta,
@@ -364,7 +388,13 @@ void oracle_schedule_stream(const uint32_t* fanout, const uint8_t* role, const d
     for (uint64_t d = 0; d < D; ++d) {
       if (load[d] + l > cap) { score[d] = inf; continue; }
       int tau = 0;
-      const double b = path_bottleneck_dir(t, bw, u_row, d_row, p, decs[d], &tau);
+      double b;
+      if (tier_mode) {
+        tau = tier(t, p, decs[d]);
+        b = bw[tau] * (1.0 - (double)u_row[tau]);
+      } else {
+        b = path_bottleneck_dir(t, bw, u_row, d_row, p, decs[d], &tau);
+      }
       const int64_t lam = 16 * (int64_t)M[(uint64_t)r * D + d];
       const double s_eff = (double)((l - lam) * (int64_t)bytes_per_token);
       const double T = s_eff / b + lat[tau];

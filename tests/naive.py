@@ -124,9 +124,11 @@ def lcp_blocks(chain: Sequence[int], cache: Sequence[int]) -> int:
 
 
 def greedy_exact(tree, role, bw, lat, util, length, prefill, snap, M, events,
-                 w, theta, cap, bpt, util_down=None):
+                 w, theta, cap, bpt, util_down=None, tier_mode=False):
     """Exact-rational Algorithm 1 with the weighted score; returns (dec, best_scores).
-    util_down: downward rows for directed links (util then holds the upward ones)."""
+    util_down: downward rows for directed links (util then holds the upward ones).
+    tier_mode: util rows are per-tier congestion c[4] and a pair's bandwidth is
+    B_tau (1 - c_tau) (the paper's four maps)."""
     pre = [i for i in range(tree.n) if role[i] == 0]
     dec_inst = [i for i in range(tree.n) if role[i] == 1]
     D = len(dec_inst)
@@ -152,8 +154,13 @@ def greedy_exact(tree, role, bw, lat, util, length, prefill, snap, M, events,
                 scores.append(None)
                 continue
             miss_tok = l - 16 * int(M[r][d])
-            b = bottleneck(tree, bw, u_row, p, dec_inst[d]) if util_down is None else \
-                bottleneck_directed(tree, bw, u_row, util_down[int(snap[r])], p, dec_inst[d])
+            if tier_mode:
+                tau = tree.tier(p, dec_inst[d])
+                b = frac(bw[tau]) * (1 - frac(u_row[tau]))
+            elif util_down is None:
+                b = bottleneck(tree, bw, u_row, p, dec_inst[d])
+            else:
+                b = bottleneck_directed(tree, bw, u_row, util_down[int(snap[r])], p, dec_inst[d])
             T = Fraction(miss_tok * bpt) / b + frac(lat[tree.tier(p, dec_inst[d])])
             scores.append(wn * T + wp * Fraction(miss_tok, l) + wl * th * load[d])
         cands = [(s, d) for d, s in enumerate(scores) if s is not None]

@@ -758,3 +758,68 @@ def test_directed_greedy_matches_exact_rational_bruteforce():
         for r in range(len(dec)):
             if dec[r] >= 0:
                 assert res.best[r] == pytest.approx(float(best[r]), rel=1e-14)
+
+
+# ------------------------------------- paper-literal per-tier oracle (NEXT: four maps)
+def test_per_tier_worked_example():
+    """Sec. III-D with the paper's per-tier maps (no transfer in flight): d1 on tier 2 at
+    B2 (1 - c) = 5 GB/s, d2 on tier 3 at 2.5 GB/s and, with c3 = 0.5, 1.5625 GB/s."""
+    g = golden("worked_example.txt")
+    fanout = (2, 2, 2, 2)
+    role = np.zeros(16, np.uint8)
+    role[[4, 8]] = 1
+    bw = [100e9, 50e9, g["B2"], g["B3"]]
+    c = np.full((1, 4), g["c"], np.float32)
+    C5 = oracle.cost_matrix_tiers(fanout, role, bw, [0.0] * 4, c, g["s_eff_d1"])
+    C1 = oracle.cost_matrix_tiers(fanout, role, bw, [0.0] * 4, c, g["s_eff_d2"])
+    # d1 without the in-flight transfer: half of the example's 2.0 s
+    assert C5[0, 0, 0] == pytest.approx(g["T_d1"] / 2, rel=1e-7)
+    assert C1[0, 0, 1] == pytest.approx(g["T_d2"], rel=1e-7)
+    c[0, 3] = g["c3_perturbed"]
+    C1 = oracle.cost_matrix_tiers(fanout, role, bw, [0.0] * 4, c, g["s_eff_d2"])
+    assert C1[0, 0, 1] == pytest.approx(g["T_d2_perturbed"], rel=1e-7)
+    assert C1[0, 0, 0] == pytest.approx(g["s_eff_d2"] / (g["B2"] * (1 - float(np.float32(g["c"])))), rel=1e-12)
+
+
+def test_per_tier_is_the_per_link_model_only_when_the_tier_level_is_the_bottleneck():
+    """With every level-k link at c_k the per-link oracle takes min over levels <= tau of
+    B_k (1 - c_k); the per-tier oracle takes B_tau (1 - c_tau).  They agree when that is
+    the minimum and differ when a lower level is congested harder."""
+    rng = np.random.default_rng(77)
+    fanout = (2, 2, 2, 2)
+    tree = naive.ExplicitTree(fanout)
+    role = (np.arange(16) % 2).astype(np.uint8)
+    bw, lat = [900e9, 400e9, 200e9, 100e9], [1e-6, 3e-6, 6e-6, 10e-6]
+    level = np.array([tree.level[e] for e in range(tree.n_edges)])
+    for c in ([0.1, 0.2, 0.3, 0.4], [0.0, 0.0, 0.5, 0.5]):          # tier level is the min
+        cc = np.array([c], np.float32)
+        np.testing.assert_allclose(oracle.cost_matrix_tiers(fanout, role, bw, lat, cc, 1e9),
+                                   oracle.cost_matrix(fanout, role, bw, lat, cc[:, level], 1e9),
+                                   rtol=1e-15)
+    cc = np.array([[0.99, 0.0, 0.0, 0.0]], np.float32)                 # level 0 congested
+    per_tier = oracle.cost_matrix_tiers(fanout, role, bw, lat, cc, 1e9)
+    per_link = oracle.cost_matrix(fanout, role, bw, lat, cc[:, level], 1e9)
+    taus = np.array([[tree.tier(p, d) for d in range(1, 16, 2)] for p in range(0, 16, 2)])
+    assert (per_link[0][taus > 0] > per_tier[0][taus > 0]).all()      # the level-0 link binds
+    np.testing.assert_array_equal(per_link[0][taus == 0], per_tier[0][taus == 0])
+    one_minus_c = 1.0 - cc[0].astype(np.float64)
+    np.testing.assert_allclose(per_tier[0], 1e9 / (np.array(bw)[taus] * one_minus_c[taus])
+                               + np.array(lat)[taus], rtol=1e-15)
+
+
+def test_per_tier_greedy_matches_exact_rational_bruteforce():
+    theta = float(np.float32(1e-6))
+    for seed in range(20):
+        pb = _tiny_problem(seed)
+        c = np.random.default_rng(1100 + seed).uniform(0, 0.9, size=(pb["u"].shape[0], 4)).astype(np.float32)
+        w = tuple(float(np.float32(x)) for x in np.random.default_rng(1200 + seed).uniform(0, 2, 3))
+        res = oracle.schedule_stream(pb["fanout"], pb["role"], pb["bw"], pb["lat"], c,
+                                     pb["length"], pb["prefill"], pb["snap"], pb["M"], pb["events"],
+                                     w[0], w[1], w[2], theta, pb["cap"], 81920, tier_mode=True)
+        dec, best, load = naive.greedy_exact(pb["tree"], pb["role"], pb["bw"], pb["lat"], c,
+                                             pb["length"], pb["prefill"], pb["snap"], pb["M"],
+                                             pb["events"], w, theta, pb["cap"], 81920, tier_mode=True)
+        assert list(res.dec) == dec and list(res.load) == load
+        for r in range(len(dec)):
+            if dec[r] >= 0:
+                assert res.best[r] == pytest.approx(float(best[r]), rel=1e-14)
