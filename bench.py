@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--snapshots", type=int, default=1000)
     ap.add_argument("--directed", action="store_true",
                     help="directed links: separate upward and downward utilisation rows")
+    ap.add_argument("--tiers", action="store_true",
+                    help="the paper's per-tier maps: four congestion values per snapshot")
     ap.add_argument("--inflight", type=int, default=0,
                     help="self-contention counter cap (Eq. 4's n_inflight; the paper uses 16); "
                          "0 = the plain greedy")
@@ -203,7 +205,7 @@ def measured_peaks():
 
 
 # ------------------------------------------------------------------ CPU oracle
-def cpu_oracle_sample(w, streams, theta, cap, bpt, inflight=0, directed=False):
+def cpu_oracle_sample(w, streams, theta, cap, bpt, inflight=0, directed=False, tiers=False):
     """Time the CPU oracle on whole streams of the workload (with self-contention when
     inflight > 0, with directed links when directed); returns (decisions, seconds)."""
     from oracle.workload import run_stream, run_stream_inflight
@@ -213,7 +215,7 @@ def cpu_oracle_sample(w, streams, theta, cap, bpt, inflight=0, directed=False):
         if inflight > 0:
             res = run_stream_inflight(w, int(s), theta, cap, bpt, inflight)
         else:
-            res = run_stream(w, int(s), theta, cap, bpt, directed=directed)
+            res = run_stream(w, int(s), theta, cap, bpt, directed=directed, tiers=tiers)
         dec += int(res.dec.shape[0])
     return dec, time.perf_counter() - t0
 
@@ -356,7 +358,7 @@ def workload_spec(kind: str, streams: int, rank: int):
 
 
 def setup_workload(spec, dev, table_batch: int = 256, inflight: bool = False,
-                   directed: bool = False):
+                   directed: bool = False, tiers: bool = False):
     """A generated workload on `dev`: its inputs, the resident cache index and the step's
     device buffers.  Returns (workload, scorer, step inputs, step outputs)."""
     import torch
@@ -382,7 +384,10 @@ def setup_workload(spec, dev, table_batch: int = 256, inflight: bool = False,
         raise RuntimeError(f"cache build status {int(sc.status.item())}")
     ra = stage.request_arrays(w, device=dev)
     chains, _ = sdev.chains(w, device=dev)
-    x = StepInputs(util=sdev.util(w, device=dev), chains=chains, chain_off=ra["chain_off"],
+    if tiers:  # the paper's per-tier maps: four congestion values per snapshot
+        sc.oracle_mode = "tiers"
+    util = stage.util(w, device=dev, direction="tiers") if tiers else sdev.util(w, device=dev)
+    x = StepInputs(util=util, chains=chains, chain_off=ra["chain_off"],
                    set_off=ra["set_off"], length=ra["length"], prefill=ra["prefill"],
                    snap=ra["snap"], events=ra["events"], event_off=ra["event_off"],
                    weights=weights_tensor(w.weights, theta, spec.cap_tokens, bpt, device=dev),
@@ -429,7 +434,7 @@ def run_netkv(args):
 
     w, sc, x, out = setup_workload(workload_spec(args.workload, args.streams, rank), dev,
                                    args.table_batch, inflight=args.inflight > 0,
-                                   directed=args.directed)
+                                   directed=args.directed, tiers=args.tiers)
     sc.share_prefixes = not args.no_share
     sc.inflight_cap = args.inflight
     theta = float(np.float32(synth.THETA_S_PER_TOKEN))
@@ -487,7 +492,8 @@ def run_netkv(args):
         # 8-byte chain block + 16-byte index entry per examined block, 2-byte M store
         "prefix_match": 24 * examined + 2 * R * D,
         # per snapshot: the utilisation row (L floats), 16-byte UB of every instance
-        "oracle_build": x.n_snap * ((8 if x.util_down is not None else 4) * w.L + 16 * sc.N),
+        "oracle_build": x.n_snap * (16 + 16 * sc.N) if args.tiers else
+                        x.n_snap * ((8 if x.util_down is not None else 4) * w.L + 16 * sc.N),
         # per arrival: event, len/prefill/snap, per candidate base score (4 B) + the
         # dec/best/second stores; per departure: event, len, dec
         "schedule": R * (4 + 12 + 4 * D + 12) + R * 12 + 2 * 8 * D * x.n_streams,
@@ -552,7 +558,7 @@ def run_netkv(args):
         sample = np.random.default_rng(0).choice(args.streams, size=min(args.cpu_streams, args.streams),
                                                  replace=False)
         d, secs = cpu_oracle_sample(w, sample, theta, spec.cap_tokens, bpt, args.inflight,
-                                    args.directed)
+                                    args.directed, args.tiers)
         cpu = {"value": d / secs, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                "sample": f"{len(sample)} of {args.streams} streams, whole streams "
                          f"({d} decisions in {secs:.1f} s)"}
@@ -573,7 +579,9 @@ def run_netkv(args):
                                           extra=dict(([("inflight_cap", args.inflight)]
                                                       if args.inflight else []) +
                                                      ([("links", "directed")]
-                                                      if args.directed else [])) or None),
+                                                      if args.directed else []) +
+                                                     ([("oracle", "per-tier maps")]
+                                                      if args.tiers else [])) or None),
                 "scores_per_s": value * D, "gpu_launches": launches_per_step * args.steps,
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk}
         print(json.dumps(line), flush=True)
@@ -688,8 +696,8 @@ def run_sweep(args):
 
 def main():
     args = parse()
-    if args.inflight and args.directed:
-        raise SystemExit("--inflight and --directed are measured one at a time")
+    if (args.inflight > 0) + args.directed + args.tiers > 1:
+        raise SystemExit("--inflight, --directed and --tiers are measured one at a time")
     if args.impl == "reference":
         return run_reference(args)
     if args.workload == "sweep":

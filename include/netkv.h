@@ -10,7 +10,8 @@
  *   netkv_topology_create   the four-tier instance tree (Sec. III-A, III-E)
  *   netkv_oracle_build      network cost oracle C[s][p][d] from per-link utilisation
  *                           snapshots, and the per-instance level bottlenecks UB
- *                           (netkv_oracle_build_directed: per link and direction)
+ *                           (netkv_oracle_build_directed: per link and direction;
+ *                           netkv_oracle_build_tiers: the paper's per-tier maps)
  *   netkv_cache_build       decode caches K_d as open-addressing hash tables
  *   netkv_prefix_match      block-level prefix hit M[r][d] (Sec. III-B)
  *   netkv_schedule_streams  the greedy of Algorithm 1 over independent streams
@@ -133,6 +134,18 @@ netkv_status netkv_oracle_build_directed(netkv_topology_t topo, const float* d_u
                                          const float* d_util_down, uint32_t n_snap,
                                          double kv_bytes, float* d_C, float* d_UB,
                                          int* d_status, netkv_stream_t stream);
+
+/* The paper-literal per-tier oracle (Sec. III-E: the tier, bandwidth, congestion and
+ * latency maps; Eq. 4 with n_inflight = 0): d_c is [n_snap][4] per-tier congestion
+ * c_tau in [0, 1), and a pair's bandwidth is B_tau * (1 - c_tau) with no minimum over the
+ * lower levels of its path:
+ *     C[s][p][d] = kv_bytes / (B_tau (1 - c[s][tau])) + L_tau
+ * UB[s][i][k] = B_k (1 - c[s][k]) for every instance, so that netkv_schedule_streams
+ * scores with the same maps.  Other arguments and errors as netkv_oracle_build.
+ */
+netkv_status netkv_oracle_build_tiers(netkv_topology_t topo, const float* d_c, uint32_t n_snap,
+                                      double kv_bytes, float* d_C, float* d_UB, int* d_status,
+                                      netkv_stream_t stream);
 
 /* ------------------------------------------------------------------ caches
  * Decode caches K_d (Sec. III-C), the sets of block hashes each decode instance holds.

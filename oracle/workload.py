@@ -58,16 +58,19 @@ def _rows(w, snaps, direction):
 
 def run_stream(w, s: int, theta: float, cap: int, bytes_per_token: int,
                hint: Optional[np.ndarray] = None, rel_tol: float = 1e-5,
-               M: Optional[np.ndarray] = None, directed: bool = False) -> OracleStream:
+               M: Optional[np.ndarray] = None, directed: bool = False,
+               tiers: bool = False) -> OracleStream:
     """Oracle for stream s of workload w (per-stream table sets and telemetry, or shared).
 
     hint: decisions of another implementation for this stream's requests (local order).
     directed: links carry separate upward and downward utilisations (the generator's
     "up" and "down" rows); UB is then the directed level bottleneck.
+    tiers: the paper's per-tier maps (the generator's "tiers" rows, four congestion
+    values per snapshot); UB[s][i][k] is then B_k (1 - c[s][k]) for every instance.
     """
-    from synth import request_set
+    from synth import request_set, utilisation
     r0, r1, ev_local, snaps, snap_local = stream_problem(w, s)
-    util = _rows(w, snaps, "up")
+    util = utilisation(w, snaps, "tiers") if tiers else _rows(w, snaps, "up")
     util_down = _rows(w, snaps, "down") if directed else None
     if M is None:
         g = int(request_set(w)[r0]) if r1 > r0 else 0
@@ -81,9 +84,14 @@ def run_stream(w, s: int, theta: float, cap: int, bytes_per_token: int,
     res = schedule_stream(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, util,
                           w.length[r0:r1], w.prefill[r0:r1], snap_local, M, ev_local,
                           wn, wp, wl, theta, cap, bytes_per_token, hint=hint, rel_tol=rel_tol,
-                          util_down=util_down)
-    UB = up_bottleneck(spec.fanout, spec.tier_bw, util) if not directed else \
-        level_bottleneck_directed(spec.fanout, w.role, spec.tier_bw, util, util_down)
+                          util_down=util_down, tier_mode=tiers)
+    if tiers:
+        per_tier = np.asarray(spec.tier_bw, np.float64) * (1.0 - util.astype(np.float64))
+        UB = np.repeat(per_tier[:, None, :], len(w.role), axis=1)
+    elif directed:
+        UB = level_bottleneck_directed(spec.fanout, w.role, spec.tier_bw, util, util_down)
+    else:
+        UB = up_bottleneck(spec.fanout, spec.tier_bw, util)
     return OracleStream(r0, r1, M, res.dec, res.best, res.second, res.load, res.near_ties,
                         res.mismatches, res.rejects, snaps, UB)
 
@@ -95,7 +103,7 @@ def run_stream_inflight(w, s: int, theta: float, cap: int, bytes_per_token: int,
     """Oracle for stream s with self-contention (Eq. 4's n_inflight, Algorithm 1 lines 5
     and 14).  hint / xfer_hint: another implementation's decisions and transfer times
     for the stream's requests (local order).  The result carries xfer_us."""
-    from synth import request_set
+    from synth import request_set, utilisation
     r0, r1, ev_local, snaps, snap_local = stream_problem(w, s)
     util = _rows(w, snaps, "up")
     if M is None:

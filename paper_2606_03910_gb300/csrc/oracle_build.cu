@@ -5,6 +5,8 @@
 //   (kDir) a prefill instance's climb reads the upward row and a decode instance's the
 //   downward row: the directions a transfer from prefill to decode crosses them in.
 // oracle_build_kernel: C[s][p][d] = kv / min(UB[s][p][tau], UB[s][d][tau]) + L_tau.
+//   In the paper-literal per-tier mode (kTier) UB[s][i][k] = B_k (1 - c[s][k]) for every
+//   instance, from four congestion values per snapshot.
 //   Division is monotone (correctly rounded, positive operands), so
 //   kv / min(a, b) == max(kv / a, kv / b) exactly; each block therefore divides once per
 //   (instance, level) it touches and the per-pair work is a tier test, a max and an
@@ -39,11 +41,22 @@ __device__ __forceinline__ float4 level_bottlenecks(const TopoArgs& t, const flo
   return b;
 }
 
+// Paper-literal per-tier maps (Sec. III-E): level k's bandwidth B_k (1 - c_k) from the
+// snapshot's four per-tier congestion values, with no minimum over lower levels.
+__device__ __forceinline__ float4 tier_bandwidths(const TopoArgs& t, const float* __restrict__ c,
+                                                  int* status) {
+  const float c0 = __ldg(c), c1 = __ldg(c + 1), c2 = __ldg(c + 2), c3 = __ldg(c + 3);
+  if (!(util_ok(c0) && util_ok(c1) && util_ok(c2) && util_ok(c3)))
+    flag_status(status, NETKV_DEV_EDOMAIN);
+  return make_float4(t.bw[0] * (1.0f - c0), t.bw[1] * (1.0f - c1), t.bw[2] * (1.0f - c2),
+                     t.bw[3] * (1.0f - c3));
+}
+
 __device__ __forceinline__ float4 quotients(float kv, const float4& b) {
   return make_float4(kv / b.x, kv / b.y, kv / b.z, kv / b.w);
 }
 
-template <bool kDir>
+template <bool kDir, bool kTier = false>
 __global__ void __launch_bounds__(kBlock) level_bottleneck_kernel(
     TopoArgs t, const float* __restrict__ util, const float* __restrict__ util_down,
     uint32_t n_snap, float4* __restrict__ UB, int* status) {
@@ -54,13 +67,14 @@ __global__ void __launch_bounds__(kBlock) level_bottleneck_kernel(
     const uint32_t i = (uint32_t)(idx - s * t.N);
     const uint4 l = __ldg(t.links + i);
     const float* rows = (kDir && __ldg(t.role + i)) ? util_down : util;
-    UB[idx] = level_bottlenecks(t, rows + s * t.n_links, l, status);
+    UB[idx] = kTier ? tier_bandwidths(t, util + s * 4, status)
+                    : level_bottlenecks(t, rows + s * t.n_links, l, status);
   }
 }
 
 // util_down: the decode side's rows (the downward utilisations of directed links; the
 // same pointer as util for undirected links).
-template <bool kVec>
+template <bool kVec, bool kTier = false>
 __global__ void __launch_bounds__(kBlock) oracle_build_kernel(
     TopoArgs t, const float* __restrict__ util, const float* __restrict__ util_down,
     uint32_t n_snap, float kv, float* __restrict__ C, int* status) {
@@ -79,7 +93,8 @@ __global__ void __launch_bounds__(kBlock) oracle_build_kernel(
       const uint32_t d = d0 + j;
       if (d < t.D) {
         ld[j] = __ldg(t.links + __ldg(t.dec + d));
-        qd[j] = quotients(kv, level_bottlenecks(t, row_d, ld[j], status));
+        qd[j] = quotients(kv, kTier ? tier_bandwidths(t, util + (uint64_t)s * 4, status)
+                                    : level_bottlenecks(t, row_d, ld[j], status));
       } else {
         ld[j] = make_uint4(0, 0, 0, 0);
         qd[j] = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -92,7 +107,8 @@ __global__ void __launch_bounds__(kBlock) oracle_build_kernel(
       for (uint32_t k = threadIdx.x; k < np; k += kBlock) {
         const uint4 l = __ldg(t.links + __ldg(t.pre + p0 + k));
         s_l[k] = l;
-        s_q[k] = quotients(kv, level_bottlenecks(t, row, l, status));
+        s_q[k] = quotients(kv, kTier ? tier_bandwidths(t, util + (uint64_t)s * 4, status)
+                                     : level_bottlenecks(t, row, l, status));
       }
       __syncthreads();
       if (d0 >= t.D) continue;
@@ -120,8 +136,10 @@ __global__ void __launch_bounds__(kBlock) oracle_build_kernel(
 
 }  // namespace
 
+enum OracleMode { kLinks = 0, kDirected = 1, kTiers = 2 };
+
 static netkv_status oracle_build(netkv_topology_t topo, const float* d_util, const float* d_util_down,
-                          bool directed, uint32_t n_snap, double kv_bytes, float* d_C,
+                          int mode, uint32_t n_snap, double kv_bytes, float* d_C,
                           float* d_UB, int* d_status, netkv_stream_t stream) {
   if (!topo || !d_util || !d_util_down || (!d_C && !d_UB)) return NETKV_EINVAL;
   if (!(kv_bytes > 0) || !(kv_bytes < 3.0e38)) return NETKV_EINVAL;
@@ -135,7 +153,10 @@ static netkv_status oracle_build(netkv_topology_t topo, const float* d_util, con
     const uint64_t total = (uint64_t)n_snap * t.N;
     const uint64_t blocks = (total + kBlock - 1) / kBlock;
     const unsigned grid = (unsigned)(blocks < (1u << 20) ? blocks : (1u << 20));
-    if (directed)
+    if (mode == kTiers)
+      level_bottleneck_kernel<false, true><<<grid, kBlock, 0, s>>>(
+          t, d_util, d_util, n_snap, reinterpret_cast<float4*>(d_UB), d_status);
+    else if (mode == kDirected)
       level_bottleneck_kernel<true><<<grid, kBlock, 0, s>>>(
           t, d_util, d_util_down, n_snap, reinterpret_cast<float4*>(d_UB), d_status);
     else
@@ -146,7 +167,13 @@ static netkv_status oracle_build(netkv_topology_t topo, const float* d_util, con
   if (d_C) {
     const dim3 grid((t.D + kDChunk - 1) / kDChunk, n_snap < 65535u ? n_snap : 65535u);
     const bool vec = (t.D % 4 == 0) && aligned_to(d_C, 16);
-    if (vec)
+    if (mode == kTiers && vec)
+      oracle_build_kernel<true, true><<<grid, kBlock, 0, s>>>(t, d_util, d_util, n_snap,
+                                                              (float)kv_bytes, d_C, d_status);
+    else if (mode == kTiers)
+      oracle_build_kernel<false, true><<<grid, kBlock, 0, s>>>(t, d_util, d_util, n_snap,
+                                                               (float)kv_bytes, d_C, d_status);
+    else if (vec)
       oracle_build_kernel<true><<<grid, kBlock, 0, s>>>(t, d_util, d_util_down, n_snap,
                                                         (float)kv_bytes, d_C, d_status);
     else
@@ -160,13 +187,20 @@ static netkv_status oracle_build(netkv_topology_t topo, const float* d_util, con
 extern "C" netkv_status netkv_oracle_build(netkv_topology_t topo, const float* d_util,
                                            uint32_t n_snap, double kv_bytes, float* d_C,
                                            float* d_UB, int* d_status, netkv_stream_t stream) {
-  return oracle_build(topo, d_util, d_util, false, n_snap, kv_bytes, d_C, d_UB, d_status, stream);
+  return oracle_build(topo, d_util, d_util, kLinks, n_snap, kv_bytes, d_C, d_UB, d_status, stream);
 }
 
 extern "C" netkv_status netkv_oracle_build_directed(netkv_topology_t topo, const float* d_util_up,
                                                     const float* d_util_down, uint32_t n_snap,
                                                     double kv_bytes, float* d_C, float* d_UB,
                                                     int* d_status, netkv_stream_t stream) {
-  return oracle_build(topo, d_util_up, d_util_down, true, n_snap, kv_bytes, d_C, d_UB, d_status,
-                      stream);
+  return oracle_build(topo, d_util_up, d_util_down, kDirected, n_snap, kv_bytes, d_C, d_UB,
+                      d_status, stream);
+}
+
+extern "C" netkv_status netkv_oracle_build_tiers(netkv_topology_t topo, const float* d_c,
+                                                 uint32_t n_snap, double kv_bytes, float* d_C,
+                                                 float* d_UB, int* d_status,
+                                                 netkv_stream_t stream) {
+  return oracle_build(topo, d_c, d_c, kTiers, n_snap, kv_bytes, d_C, d_UB, d_status, stream);
 }

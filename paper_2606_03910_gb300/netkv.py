@@ -30,7 +30,8 @@ _NAMES = {1: "NETKV_EINVAL", 2: "NETKV_ENOMEM", 3: "NETKV_ECUDA",
           4: "NETKV_ELIMIT (more requests than the fixed scratch of netkv_prefix_match_static holds)"}
 
 EXPORTS = ("netkv_topology_create", "netkv_topology_destroy", "netkv_topology_query",
-           "netkv_oracle_build", "netkv_oracle_build_directed", "netkv_cache_index_bytes",
+           "netkv_oracle_build", "netkv_oracle_build_directed", "netkv_oracle_build_tiers",
+           "netkv_cache_index_bytes",
            "netkv_cache_build",
            "netkv_prefix_match_workspace_size",
            "netkv_prefix_match", "netkv_prefix_match_static", "netkv_schedule_workspace_size",
@@ -63,6 +64,7 @@ _lib.netkv_topology_destroy.argtypes = [_P]
 _lib.netkv_topology_query.argtypes = [_P, _P, _P, _P, _P]
 _lib.netkv_oracle_build.argtypes = [_P, _P, _U32, _F64, _P, _P, _P, _P]
 _lib.netkv_oracle_build_directed.argtypes = [_P, _P, _P, _U32, _F64, _P, _P, _P, _P]
+_lib.netkv_oracle_build_tiers.argtypes = [_P, _P, _U32, _F64, _P, _P, _P, _P]
 _lib.netkv_cache_index_bytes.argtypes = [_U32, _U32, _U32]
 _lib.netkv_cache_index_bytes.restype = C.c_size_t
 _lib.netkv_cache_build.argtypes = [_P, _U32, _U32, _U32, _P, _P, _P, _P]
@@ -229,6 +231,14 @@ def netkv_oracle_build_directed(topo: Topology, util_up, util_down, n_snap: int,
     _check("netkv_oracle_build_directed", _lib.netkv_oracle_build_directed(
         topo.handle, _ptr(util_up), _ptr(util_down), int(n_snap), float(kv_bytes), _ptr(C),
         _ptr(UB), _ptr(status), _stream(stream)))
+
+
+def netkv_oracle_build_tiers(topo: Topology, c, n_snap: int, kv_bytes: float, C=None, UB=None,
+                             status=None, stream=None) -> None:
+    """The paper-literal per-tier oracle; see include/netkv.h."""
+    _check("netkv_oracle_build_tiers", _lib.netkv_oracle_build_tiers(
+        topo.handle, _ptr(c), int(n_snap), float(kv_bytes), _ptr(C), _ptr(UB), _ptr(status),
+        _stream(stream)))
 
 
 def netkv_copy_async(dst, src, nbytes: int, stream=None) -> None:

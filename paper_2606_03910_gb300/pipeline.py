@@ -91,6 +91,9 @@ class Scorer:
         self.sched_workspace = None
         # self-contention counter cap (Eq. 4's n_inflight); 0 = the plain greedy
         self.inflight_cap = 0
+        # "links": per-link utilisation rows; "tiers": the paper's per-tier maps, x.util
+        # then holds four congestion values per snapshot
+        self.oracle_mode = "links"
 
     def _sched_workspace(self, R: int):
         """Greedy workspace (base scores of every arrival), grown on demand."""
@@ -134,6 +137,10 @@ class Scorer:
             xfer_us=torch.empty(R, dtype=torch.int32, device=dev))
 
     def oracle_build(self, x: StepInputs, out: StepOutputs, stream=None) -> None:
+        if self.oracle_mode == "tiers":
+            netkv.netkv_oracle_build_tiers(self.topo, x.util, x.n_snap, 1.0, None, out.UB,
+                                           out.status, stream)
+            return
         if x.util_down is not None:  # directed links: util holds the upward rows
             netkv.netkv_oracle_build_directed(self.topo, x.util, x.util_down, x.n_snap, 1.0, None,
                                               out.UB, out.status, stream)

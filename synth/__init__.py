@@ -342,14 +342,25 @@ def cache_keys(w: Workload, g: int, d: int) -> np.ndarray:
 
 
 DOWN_SEED = 1 << 40  # downward utilisations (directed links) draw from seed + DOWN_SEED
+TIER_SEED = 1 << 41  # per-tier congestion rows (the paper's four maps) from seed + TIER_SEED
 
 
 def utilisation(w: Workload, snaps: np.ndarray, direction: str = "up") -> np.ndarray:
     """Utilisation rows of snapshots `snaps`.  direction "up" is the undirected row (and
     the upward one of directed links); "down" is an independent draw of the same
-    distribution for the downward direction."""
+    distribution for the downward direction; "tiers" gives four per-tier congestion
+    values per snapshot, uniform in [0, 0.9), for the paper's per-tier maps."""
     spec = w.spec
     snaps = np.asarray(snaps, dtype=np.int64)
+    if direction == "tiers":  # draw(seed + TIER_SEED, P_UTIL, local index, tier), vectorised
+        seeds = w.snap_seed[snaps].astype(np.int64) + TIER_SEED
+        uniq, inv = np.unique(seeds, return_inverse=True)
+        k = np.array([stream_key(int(x), P_UTIL) for x in uniq], dtype=U64)[inv.reshape(-1)]
+        loc = w.snap_local[snaps].astype(U64)
+        with np.errstate(over="ignore"):
+            k2 = _mix(k + (loc + U64(1)) * U64(GOLDEN))
+            vals = _mix(k2[:, None] + (np.arange(4, dtype=U64)[None, :] + U64(1)) * U64(GOLDEN))
+        return uniform09_f32(vals).astype(np.float32).reshape(len(snaps), 4)
     e = np.arange(w.L, dtype=np.int64)
     out = np.empty((len(snaps), w.L), np.float32)
     shift = 0 if direction == "up" else DOWN_SEED

@@ -64,6 +64,6 @@ def keys(w: Workload, g0: int, g1: int, device="cuda", host_threshold: int = 1 <
 
 def util(w: Workload, device="cuda", host_threshold: int = 1 << 22, direction: str = "up"):
     import torch
-    if w.n_snap * w.L <= host_threshold or w.spec.util_mode != "uniform09":
+    if direction == "tiers" or w.n_snap * w.L <= host_threshold or w.spec.util_mode != "uniform09":
         return torch.from_numpy(w.util(direction=direction)).to(device)
     return sdev.util(w, device=device, direction=direction)

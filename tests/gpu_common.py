@@ -32,7 +32,7 @@ def make_scorer(w, device="cuda"):
                   index_log2(w), device=device)
 
 
-def run_gpu(w, sc=None, cap=None, load_init=None, directed=False):
+def run_gpu(w, sc=None, cap=None, load_init=None, directed=False, tiers=False):
     """Whole path on the GPU for workload w; returns (scorer, inputs, outputs).
     directed: links carry the generator's upward and downward utilisation rows."""
     import torch
@@ -42,7 +42,10 @@ def run_gpu(w, sc=None, cap=None, load_init=None, directed=False):
     sc.load_caches(keys, stage.key_offsets(w, w.n_sets * w.D))
     ra = stage.request_arrays(w)
     cap = w.spec.cap_tokens if cap is None else cap
-    x = StepInputs(util=stage.util(w), chains=stage.chains(w), chain_off=ra["chain_off"],
+    if tiers:
+        sc.oracle_mode = "tiers"
+    x = StepInputs(util=stage.util(w, direction="tiers" if tiers else "up"),
+                   chains=stage.chains(w), chain_off=ra["chain_off"],
                    set_off=ra["set_off"], length=ra["length"], prefill=ra["prefill"],
                    snap=ra["snap"], events=ra["events"], event_off=ra["event_off"],
                    weights=weights_tensor(w.weights, THETA, cap, synth.BYTES_PER_TOKEN_SHARD),
@@ -58,7 +61,7 @@ def host(t):
     return t.detach().cpu().numpy()
 
 
-def check_stream(w, s, out, cap=None, M_gpu=None, M_expect=None, directed=False):
+def check_stream(w, s, out, cap=None, M_gpu=None, M_expect=None, directed=False, tiers=False):
     """Oracle on stream s with the GPU decisions as near-tie hints; asserts parity.
     M_expect: the stream's prefix hits for the oracle's greedy where its own per-stream
     cache sets would not fit (the generator's constructed hits).  Returns the oracle result."""
@@ -68,7 +71,7 @@ def check_stream(w, s, out, cap=None, M_gpu=None, M_expect=None, directed=False)
     r0, r1 = int(w.req_off[s]), int(w.req_off[s + 1])
     dec = host(out.dec[r0:r1])
     res = run_stream(w, s, THETA, cap, synth.BYTES_PER_TOKEN_SHARD, hint=dec, M=M_expect,
-                     directed=directed)
+                     directed=directed, tiers=tiers)
     # prefix hits: bit-exact
     if M_gpu is None:
         M_gpu = host(out.M[r0:r1]).view(np.uint16)
