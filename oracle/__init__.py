@@ -72,6 +72,10 @@ def _declare(l):
     l.oracle_schedule_stream.restype = None
     l.oracle_schedule_stream.argtypes = [P, P, P, P, P, P, INT, U64, P, P, P, P, P, U64, F64, F64,
                                          F64, F64, I64, U64, P, P, F64, P, P, P, P, P]
+    l.oracle_schedule_stream_load.restype = None
+    l.oracle_schedule_stream_load.argtypes = [P, P, P, P, P, U64, P, P, P, P, P, U64, F64, F64,
+                                              F64, U64, F64, F64, I64, I64, I64, P, P, P, F64,
+                                              P, P, P, P, P, P]
     l.oracle_cost_matrix_tiers.restype = None
     l.oracle_cost_matrix_tiers.argtypes = [P, P, P, P, P, U64, F64, P]
     l.oracle_cost_matrix_directed.restype = None
@@ -295,3 +299,40 @@ def schedule_stream_inflight(fanout, role, bw, lat, util, length, prefill, snap,
         _p(best), _p(second), _p(xfer), _p(load), _p(counts))
     return StreamResult(dec, best, second, load, int(counts[0]), int(counts[1]), int(counts[2]),
                         xfer, int(counts[3]), int(counts[4]))
+
+
+class LoadResult(StreamResult):
+    def __init__(self, dec, best, second, n, m, near_ties, mismatches, rejects):
+        super().__init__(dec, best, second, None, near_ties, mismatches, rejects)
+        self.n, self.m = n, m
+
+
+def schedule_stream_load(fanout, role, bw, lat, util, length, prefill, snap, M, events, w_net,
+                         w_prefix, w_load, bytes_per_token, t_a, t_b, beta_max, m_min, m0,
+                         m_init=None, n_init=None, hint=None, rel_tol=1e-5) -> LoadResult:
+    """Algorithm 1 with the paper's compute-load model (Sec. III-C, IV-B): load term
+    T_queue + T_decode from each decode's request count with t_iter(beta) = t_a + t_b beta,
+    feasibility m_d >= s_eff + m_min.  Returns decisions, scores and the final request
+    counts and free memory per decode."""
+    f, ro = _c(fanout, np.uint32), _c(role, np.uint8)
+    b, la = _c(bw, np.float64), _c(lat, np.float64)
+    u = _c(util, np.float32)
+    ln, pf, sn = _c(length, np.uint32), _c(prefill, np.uint32), _c(snap, np.uint32)
+    mm = _c(M, np.uint16)
+    ev = _c(events, np.uint32)
+    R = len(ln)
+    D = int((ro == 1).sum())
+    dec = np.full(R, -1, np.int32)
+    best = np.full(R, np.inf); second = np.full(R, np.inf)
+    n_out = np.zeros(D, np.int32); m_out = np.zeros(D, np.int64)
+    counts = np.zeros(3, np.int64)
+    mi = None if m_init is None else _c(m_init, np.int64)
+    ni = None if n_init is None else _c(n_init, np.int32)
+    h = None if hint is None else _c(hint, np.int32)
+    lib().oracle_schedule_stream_load(
+        _p(f), _p(ro), _p(b), _p(la), _p(u), u.shape[1], _p(ln), _p(pf), _p(sn), _p(mm), _p(ev),
+        len(ev), float(w_net), float(w_prefix), float(w_load), int(bytes_per_token), float(t_a),
+        float(t_b), int(beta_max), int(m_min), int(m0), _p(mi), _p(ni), _p(h), float(rel_tol),
+        _p(dec), _p(best), _p(second), _p(n_out), _p(m_out), _p(counts))
+    return LoadResult(dec, best, second, n_out, m_out, int(counts[0]), int(counts[1]),
+                      int(counts[2]))

@@ -28,6 +28,9 @@
 //   * Algorithm 1 (Sec. IV-A) as a weighted score: filter by capacity (line 1), reject
 //     when nothing is feasible (line 2), score every candidate (lines 3-11), take the
 //     argmin with the lowest index among equal scores (line 13), then update load.
+//   * The compute-load model (Sec. III-C, IV-B, the feasible set of Sec. IV-A), in
+//     oracle_schedule_stream_load: T_queue + T_decode from each decode's request count
+//     and t_iter(beta) = a + b beta, memory feasibility m_d >= s_eff + m_min.
 //   * Self-contention (Eq. 4's n_inflight, Algorithm 1 lines 5 and 14, Sec. IV-C), in
 //     oracle_schedule_stream_inflight: a per-(prefill, tier) counter divides the
 //     effective bandwidth by 1 + n; a dispatch raises the counter of its tier (saturating
@@ -526,6 +529,98 @@ void oracle_schedule_stream_inflight(
     pending.push(Done(now + dt, pr * 4 + tau));
   }
   for (uint64_t d = 0; d < D; ++d) load_out[d] = load[d];
+}
+
+// Algorithm 1 with the paper's compute-load model (Sec. III-C decode state, Sec. IV-B
+// component models, the feasible set of the objective in Sec. IV-A).  Decode d holds n[d]
+// requests (dispatched, not departed) and m[d] bytes of free memory; with the batch
+// beta = min(n, beta_max) and the queue q = n - beta,
+//     T_queue  = max(0, q - (beta_max - beta)) * t_iter(beta),  T_decode = t_iter(beta + 1),
+//     t_iter(beta) = t_a + t_b * beta,
+//     score = w_net * T_xfer + w_prefix * miss + w_load * (T_queue + T_decode)
+// over the feasible set m[d] >= s_eff(d) + m_min.  A dispatch to d* adds one request and
+// takes s_eff(d*) bytes; its departure returns both.  m_init [D] (nullable: m0 each),
+// n_init [D] (nullable: 0).  Outputs n_out, m_out [D].
+void oracle_schedule_stream_load(
+    const uint32_t* fanout, const uint8_t* role, const double* bw, const double* lat,
+    const float* util, uint64_t n_links, const uint32_t* len, const uint32_t* prefill,
+    const uint32_t* snap, const uint16_t* M, const uint32_t* events, uint64_t n_events,
+    double w_net, double w_prefix, double w_load, uint64_t bytes_per_token, double t_a,
+    double t_b, int64_t beta_max, int64_t m_min, int64_t m0, const int64_t* m_init,
+    const int32_t* n_init, const int32_t* hint, double rel_tol, int32_t* dec, double* best,
+    double* second, int32_t* n_out, int64_t* m_out, int64_t* counts) {
+  const Tree t = make_tree(fanout);
+  std::vector<uint64_t> pre, decs;
+  ranks(role, t.n, pre, decs);
+  const uint64_t D = decs.size();
+  std::vector<int64_t> n(D, 0), m(D, m0);
+  for (uint64_t d = 0; d < D; ++d) {
+    if (n_init) n[d] = n_init[d];
+    if (m_init) m[d] = m_init[d];
+  }
+  std::vector<double> score(D);
+  const double inf = std::numeric_limits<double>::infinity();
+  auto s_eff_of = [&](uint32_t r, uint64_t d) {
+    const int64_t l = len[r];
+    return (l - 16 * (int64_t)M[(uint64_t)r * D + d]) * (int64_t)bytes_per_token;
+  };
+  for (uint64_t e = 0; e < n_events; ++e) {
+    const uint32_t code = events[e];
+    const uint32_t r = code & 0x7fffffffu;
+    if (code >> 31) {  // departure: the request leaves its decode and frees its bytes
+      if (dec[r] >= 0) {
+        n[dec[r]] -= 1;
+        m[dec[r]] += s_eff_of(r, (uint64_t)dec[r]);
+      }
+      continue;
+    }
+    const int64_t l = len[r];
+    const float* u_row = util + (uint64_t)snap[r] * n_links;
+    const uint64_t p = pre[prefill[r]];
+    int32_t arg = -1;
+    for (uint64_t d = 0; d < D; ++d) {
+      const int64_t s_eff = s_eff_of(r, d);
+      if (m[d] < s_eff + m_min) { score[d] = inf; continue; }
+      int tau = 0;
+      const double b = path_bottleneck(t, bw, u_row, p, decs[d], &tau);
+      const double T = (double)s_eff / b + lat[tau];
+      const double miss = (double)(l - 16 * (int64_t)M[(uint64_t)r * D + d]) / (double)l;
+      const int64_t beta = n[d] < beta_max ? n[d] : beta_max;
+      const int64_t q = n[d] - beta;
+      const int64_t blocked = q - (beta_max - beta);
+      const double t_iter = t_a + t_b * (double)beta;
+      const double t_queue = (blocked > 0 ? (double)blocked : 0.0) * t_iter;
+      const double t_decode = t_a + t_b * (double)(beta + 1);
+      score[d] = w_net * T + w_prefix * miss + w_load * (t_queue + t_decode);
+      if (arg < 0 || score[d] < score[arg]) arg = (int32_t)d;
+    }
+    double b1 = inf, b2 = inf;
+    if (arg >= 0) {
+      b1 = score[arg];
+      for (uint64_t d = 0; d < D; ++d)
+        if ((int32_t)d != arg && score[d] < b2) b2 = score[d];
+    }
+    int32_t chosen = arg;
+    if (hint && hint[r] != arg) {
+      const int32_t h = hint[r];
+      const bool near = (arg >= 0 && h >= 0 && (uint64_t)h < D && score[h] != inf &&
+                         score[h] - b1 <= rel_tol * std::fabs(b1));
+      counts[near ? 0 : 1] += 1;
+      chosen = (h >= 0 && (uint64_t)h < D) ? h : -1;
+    }
+    if (chosen < 0) counts[2] += 1;
+    dec[r] = chosen;
+    best[r] = b1;
+    second[r] = b2;
+    if (chosen >= 0) {
+      n[chosen] += 1;
+      m[chosen] -= s_eff_of(r, (uint64_t)chosen);
+    }
+  }
+  for (uint64_t d = 0; d < D; ++d) {
+    n_out[d] = (int32_t)n[d];
+    m_out[d] = m[d];
+  }
 }
 
 }  // extern "C"

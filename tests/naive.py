@@ -231,3 +231,51 @@ def greedy_exact_inflight(tree, role, bw, lat, util, length, prefill, snap, arri
         n[(pr, tau)] = min(inflight_cap, n.get((pr, tau), 0) + 1)
         pending.append((now + dt, pr, tau))
     return dec, best, load, xfer_us
+
+
+def greedy_exact_load(tree, role, bw, lat, util, length, prefill, snap, M, events, w, bpt,
+                      t_a, t_b, beta_max, m_min, m0):
+    """Exact-rational Algorithm 1 with the paper's compute-load model: each decode holds n
+    requests and m free bytes; beta = min(n, beta_max), q = n - beta,
+    T_queue = max(0, q - (beta_max - beta)) (a + b beta), T_decode = a + b (beta + 1);
+    feasible iff m >= s_eff + m_min; dispatch n += 1, m -= s_eff, departure undoes it.
+    Returns (dec, best, n, m)."""
+    pre = [i for i in range(tree.n) if role[i] == 0]
+    dec_inst = [i for i in range(tree.n) if role[i] == 1]
+    D = len(dec_inst)
+    n, m = [0] * D, [m0] * D
+    R = len(length)
+    dec, best = [-1] * R, [None] * R
+    wn, wp, wl = (frac(x) for x in w)
+    a, b = frac(t_a), frac(t_b)
+    for code in events:
+        code = int(code)
+        r = code & 0x7FFFFFFF
+        l = int(length[r])
+        if code >> 31:
+            if dec[r] >= 0:
+                d = dec[r]
+                n[d] -= 1
+                m[d] += (l - 16 * int(M[r][d])) * bpt
+            continue
+        p = pre[int(prefill[r])]
+        u_row = util[int(snap[r])]
+        cands = []
+        for d in range(D):
+            miss_tok = l - 16 * int(M[r][d])
+            s_eff = miss_tok * bpt
+            if m[d] < s_eff + m_min:
+                continue
+            T = Fraction(s_eff) / bottleneck(tree, bw, u_row, p, dec_inst[d]) \
+                + frac(lat[tree.tier(p, dec_inst[d])])
+            beta = min(n[d], beta_max)
+            q = n[d] - beta
+            t_queue = max(0, q - (beta_max - beta)) * (a + b * beta)
+            t_decode = a + b * (beta + 1)
+            cands.append((wn * T + wp * Fraction(miss_tok, l) + wl * (t_queue + t_decode), d))
+        if cands:
+            s, d = min(cands)
+            dec[r], best[r] = d, s
+            n[d] += 1
+            m[d] -= (l - 16 * int(M[r][d])) * bpt
+    return dec, best, n, m

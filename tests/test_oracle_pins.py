@@ -823,3 +823,76 @@ def test_per_tier_greedy_matches_exact_rational_bruteforce():
         for r in range(len(dec)):
             if dec[r] >= 0:
                 assert res.best[r] == pytest.approx(float(best[r]), rel=1e-14)
+
+
+# ---------------------------------------- the paper's compute-load model (NEXT)
+T_A, T_B = float(np.float32(0.012)), float(np.float32(0.0004))   # t_iter = a + b beta, seconds
+
+
+def _run_load(pb, w, beta_max=4, m_min=0, m0=None, bpt=81920):
+    m0 = pb["cap"] * bpt if m0 is None else m0
+    return oracle.schedule_stream_load(pb["fanout"], pb["role"], pb["bw"], pb["lat"], pb["u"],
+                                       pb["length"], pb["prefill"], pb["snap"], pb["M"],
+                                       pb["events"], w[0], w[1], w[2], bpt, T_A, T_B, beta_max,
+                                       m_min, m0)
+
+
+def test_load_model_matches_exact_rational_bruteforce():
+    n_cmp = 0
+    for seed in range(40):
+        pb = _tiny_problem(seed, R=10)
+        w = tuple(float(np.float32(x)) for x in np.random.default_rng(1300 + seed).uniform(0, 2, 3))
+        bmax, m_min = (2, 3, 64)[seed % 3], (0, 10 ** 8)[seed % 2]
+        m0 = int(np.random.default_rng(seed).integers(2, 9)) * 10 ** 8
+        res = _run_load(pb, w, bmax, m_min, m0)
+        dec, best, n, m = naive.greedy_exact_load(pb["tree"], pb["role"], pb["bw"], pb["lat"],
+                                                  pb["u"], pb["length"], pb["prefill"], pb["snap"],
+                                                  pb["M"], pb["events"], w, 81920, T_A, T_B, bmax,
+                                                  m_min, m0)
+        assert list(res.dec) == dec and list(res.n) == n and list(res.m) == m
+        for r in range(len(dec)):
+            if dec[r] >= 0:
+                assert res.best[r] == pytest.approx(float(best[r]), rel=1e-14)
+                n_cmp += 1
+    assert n_cmp > 150
+
+
+def _one_decode_stream(R, beta_max, lengths=None, departures=()):
+    """One prefill, one decode (instances 0 and 1 of a (2,1,1,1) tree), R arrivals in
+    order, then the departures listed (request indices) in that order."""
+    fanout = (2, 1, 1, 1)
+    role = np.array([0, 1], np.uint8)
+    L = oracle.used_links(fanout)
+    length = np.full(R, 64, np.uint32) if lengths is None else np.asarray(lengths, np.uint32)
+    events = list(range(R)) + [r | (1 << 31) for r in departures]
+    return dict(fanout=fanout, role=role, bw=[900e9, 400e9, 200e9, 100e9], lat=[0.0] * 4,
+                u=np.zeros((1, L), np.float32), length=length, prefill=np.zeros(R, np.uint32),
+                snap=np.zeros(R, np.uint32), M=np.zeros((R, 1), np.uint16),
+                events=np.array(events, np.uint32), cap=0)
+
+
+def test_load_model_queue_and_decode_terms():
+    """Sec. IV-B on one decode with beta_max = 4 and only the load term: the k-th arrival
+    sees k requests; below beta_max it joins the batch (T_queue = 0, T_decode = a + b(k+1)),
+    above it waits one iteration per blocked predecessor: T_queue = (k - 4)(a + 4b)."""
+    R = 9
+    res = _run_load(_one_decode_stream(R, 4), (0.0, 0.0, 1.0), beta_max=4, m0=10 ** 15)
+    a, b = T_A, T_B
+    for k in range(R):
+        beta = min(k, 4)
+        expect = max(0, k - 4) * (a + b * beta) + a + b * (beta + 1)
+        assert res.best[k] == pytest.approx(expect, rel=1e-15)
+    assert list(res.n) == [R]
+
+
+def test_load_model_memory_filter():
+    """Feasible iff m >= s_eff + m_min (the objective's feasible set, Sec. IV-A): with
+    room for two requests' KV the third is rejected; a departure returns its bytes."""
+    per = 64 * 81920                                  # 64 tokens, no prefix hit
+    pb = _one_decode_stream(3, 64)
+    res = _run_load(pb, (1.0, 1.0, 1.0), beta_max=64, m0=2 * per + 5, m_min=5)
+    assert list(res.dec) == [0, 0, -1] and list(res.m) == [5]
+    pb = _one_decode_stream(3, 64, departures=(0,))
+    pb["events"] = np.array([0, 1, 0 | (1 << 31), 2], np.uint32)
+    res = _run_load(pb, (1.0, 1.0, 1.0), beta_max=64, m0=2 * per + 5, m_min=5)
+    assert list(res.dec) == [0, 0, 0] and list(res.n) == [2] and list(res.m) == [5]
