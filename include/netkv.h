@@ -16,6 +16,7 @@
  *   netkv_prefix_match      block-level prefix hit M[r][d] (Sec. III-B)
  *   netkv_schedule_streams  the greedy of Algorithm 1 over independent streams
  *   netkv_schedule_streams_inflight  the same with self-contention (Eq. 4's n_inflight)
+ *   netkv_schedule_streams_load      the same with the paper's queue/decode-step model
  *
  * Conventions for every call:
  *   - Pointers named d_* are device pointers owned by the caller; the library never
@@ -321,6 +322,43 @@ netkv_status netkv_schedule_streams_inflight(
     const uint32_t* d_events, const uint64_t* d_event_off, uint32_t inflight_cap,
     const int64_t* d_load_init, int32_t* d_dec, float* d_best, float* d_second,
     int32_t* d_xfer_us, int64_t* d_load_final, int* d_status, netkv_stream_t stream);
+
+/* The paper's compute-load model (Sec. III-C decode state, Sec. IV-B component models). */
+typedef struct {
+  float t_a_s, t_b_s;     /* iteration time t_iter(beta) = t_a + t_b * beta, seconds (>= 0) */
+  int32_t beta_max;       /* batch slots per decode (the paper uses 64), >= 1 */
+  int32_t reserved;       /* set to 0 */
+  int64_t m_min_bytes;    /* memory each decode holds back (>= 0) */
+  int64_t m0_bytes;       /* free memory of every decode at the start when d_m_init is NULL */
+} netkv_load_model;       /* 32 bytes */
+
+/* Algorithm 1 with the paper's compute-load model instead of the token load.  Decode d
+ * holds n_d requests (dispatched, not departed) and m_d free bytes; with the batch
+ * beta = min(n_d, beta_max) and the queue q = n_d - beta,
+ *     T_queue  = max(0, q - (beta_max - beta)) * t_iter(beta)         (Sec. IV-B)
+ *     T_decode = t_iter(beta + 1)
+ *     score    = w_net * T_xfer + w_prefix * miss + w_load * (T_queue + T_decode)
+ * over the feasible set m_d >= s_eff(d) + m_min (the objective's feasible set, Sec. IV-A),
+ * s_eff exact in bytes.  A dispatch to d* adds one request to it and takes s_eff(d*)
+ * bytes; the request's departure gives both back.  T_xfer and miss as in
+ * netkv_schedule_streams (without a workspace); the weights' theta and cap_tokens are
+ * not used.
+ *
+ *   model      host pointer to the model's constants
+ *   d_m_init   [n_streams][D] int64 free bytes at the start, or NULL for m0_bytes
+ *   d_n_init   [n_streams][D] int32 requests held at the start, or NULL for 0
+ *   d_m_final  [n_streams][D] int64 output: free bytes after the last event
+ *   d_n_final  [n_streams][D] int32 output: requests held after the last event
+ * Other arguments and errors as netkv_schedule_streams; EINVAL for a missing model,
+ * beta_max < 1 or negative constants.
+ */
+netkv_status netkv_schedule_streams_load(
+    netkv_topology_t topo, uint32_t n_streams, const netkv_weights* d_w,
+    const netkv_load_model* model, uint32_t R, const uint32_t* d_len, const uint32_t* d_prefill,
+    const uint32_t* d_snap, const uint16_t* d_M, const float* d_UB, uint32_t n_snap,
+    const uint32_t* d_events, const uint64_t* d_event_off, const int64_t* d_m_init,
+    const int32_t* d_n_init, int32_t* d_dec, float* d_best, float* d_second, int64_t* d_m_final,
+    int32_t* d_n_final, int* d_status, netkv_stream_t stream);
 
 /* ------------------------------------------------------------------ transfers
  * Asynchronous copy of `bytes` bytes by a kernel (SM loads and stores).  Either side may

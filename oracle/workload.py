@@ -15,7 +15,7 @@ from typing import Optional
 import numpy as np
 
 from . import (level_bottleneck_directed, prefix_match, schedule_stream, schedule_stream_inflight,
-               up_bottleneck)
+               schedule_stream_load, up_bottleneck)
 
 
 @dataclasses.dataclass
@@ -125,3 +125,29 @@ def run_stream_inflight(w, s: int, theta: float, cap: int, bytes_per_token: int,
                        res.mismatches, res.rejects, snaps, UB)
     out.xfer_us, out.xfer_adopted, out.xfer_mismatches = res.xfer_us, res.xfer_adopted, res.xfer_mismatches
     return out
+
+
+def run_stream_load(w, s: int, t_a: float, t_b: float, beta_max: int, m_min: int, m0: int,
+                    bytes_per_token: int, hint: Optional[np.ndarray] = None,
+                    rel_tol: float = 1e-5, M: Optional[np.ndarray] = None):
+    """Oracle for stream s with the paper's compute-load model (Sec. III-C, IV-B); hint: another
+    implementation's decisions for the stream's requests (local order).  Returns the
+    oracle's LoadResult with its prefix hits attached (.M)."""
+    from synth import request_set
+    r0, r1, ev_local, snaps, snap_local = stream_problem(w, s)
+    util = _rows(w, snaps, "up")
+    if M is None:
+        g = int(request_set(w)[r0]) if r1 > r0 else 0
+        keys, key_off = stream_cache_keys(w, g)
+        chains = w.chains(r0, r1)
+        chain_off = (w.chain_off[r0:r1 + 1] - w.chain_off[r0]).astype(np.uint64)
+        M = prefix_match(keys, key_off, w.D, chains, chain_off,
+                         np.array([0, r1 - r0], np.uint32))
+    wn, wp, wl = (float(x) for x in w.weights[s])
+    spec = w.spec
+    res = schedule_stream_load(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, util,
+                               w.length[r0:r1], w.prefill[r0:r1], snap_local, M, ev_local, wn, wp,
+                               wl, bytes_per_token, t_a, t_b, beta_max, m_min, m0, hint=hint,
+                               rel_tol=rel_tol)
+    res.M = M
+    return res

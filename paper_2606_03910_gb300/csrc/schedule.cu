@@ -66,6 +66,13 @@ __device__ __forceinline__ float base_score(const netkv_weights& w, uint32_t l, 
   return w.w_net * T + w.w_prefix * miss;
 }
 
+// The paper's compute-load model (Sec. III-C, IV-B) as kernel parameters.
+struct LoadModel {
+  float t_a, t_b;      // t_iter(beta) = t_a + t_b * beta
+  int32_t beta_max;
+  int64_t m_min, m0;
+};
+
 // Self-contention (Eq. 4's n_inflight, Algorithm 1 lines 5 and 14, Sec. IV-C): the
 // candidate's bandwidth is divided by 1 + n; T is returned for the completion time.
 __device__ __forceinline__ float contended_score(const netkv_weights& w, uint32_t l, uint32_t m,
@@ -299,7 +306,12 @@ __global__ void __launch_bounds__(256) base_wide_kernel(
 // (one extra stream barrier per arrival), and after the decision raises the chosen
 // tier's counter (saturating at `inflight_cap`), records the transfer time and pushes
 // its completion.  The argmin carries the winner's transfer time along.
-template <int NPT, int BLOCK, int LPS, bool kBase, bool kInfl = false>
+// Compute-load model (kLoad): load[j] holds decode j's free bytes and held[j] its request
+// count; a candidate is feasible iff free >= s_eff + m_min, its load term is
+// T_queue + T_decode from the count (beta = min(n, beta_max), q = n - beta), a dispatch
+// takes s_eff bytes and one count and the departure returns them (its prefix hits come
+// through the same pipeline as an arrival's).
+template <int NPT, int BLOCK, int LPS, bool kBase, bool kInfl = false, bool kLoad = false>
 __global__ void __launch_bounds__(BLOCK) schedule_kernel(
     TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
     const float* __restrict__ base, const uint32_t* __restrict__ len,
@@ -309,9 +321,12 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
     const int64_t* __restrict__ load_init, int32_t* dec, float* __restrict__ best,
     float* __restrict__ second, int64_t* __restrict__ load_final, int* status,
     const int64_t* __restrict__ arrival_us = nullptr, uint32_t inflight_cap = 0,
-    int32_t* __restrict__ xfer_us = nullptr, uint32_t infl_bytes = 0, uint32_t heap_cap = 0) {
+    int32_t* __restrict__ xfer_us = nullptr, uint32_t infl_bytes = 0, uint32_t heap_cap = 0,
+    LoadModel lm = LoadModel{0.f, 0.f, 0, 0, 0}, const int32_t* __restrict__ n_init = nullptr,
+    int32_t* __restrict__ n_final = nullptr) {
   static_assert(LPS == 32 || (BLOCK == 32 && NPT == 1), "packed streams use one warp");
   static_assert(!(kBase && kInfl), "self-contention scores from UB and M");
+  static_assert(!(kLoad && (kBase || kInfl)), "the load model scores from UB and M alone");
   constexpr int NW = BLOCK / 32;
   __shared__ float s_b[2][NW];
   __shared__ uint32_t s_i[2][NW];
@@ -331,15 +346,18 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
   const float inf = __int_as_float(0x7f800000);
 
   int64_t load[NPT];
+  int32_t held[NPT];  // compute-load model: requests held by the decode
   uint4 ld[NPT];  // links of the decode instance; .x is the instance index itself
 #pragma unroll
   for (int j = 0; j < NPT; ++j) {
     const uint32_t d = tid * NPT + j;
-    load[j] = 0;
+    load[j] = kLoad ? lm.m0 : 0;
+    held[j] = 0;
     ld[j] = make_uint4(0, 0, 0, 0);
     if (d < D) {
       ld[j] = __ldg(t.links + __ldg(t.dec + d));
       if (load_init) load[j] = load_init[(uint64_t)stream * D + d];
+      if (kLoad && n_init) held[j] = n_init[(uint64_t)stream * D + d];
     }
   }
 
@@ -394,7 +412,17 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
     const uint32_t r = code & 0x7fffffffu;
     if (r >= R) return;
     l = __ldg(len + r);
-    if (code >> 31) return;
+    if (code >> 31) {
+      if (kLoad) {  // the departure returns the bytes its dispatch took
+        const uint16_t* m_row = M + (uint64_t)r * D;
+#pragma unroll
+        for (int j = 0; j < NPT; ++j) {
+          const uint32_t d = tid * NPT + j;
+          if (d < D) m[j] = __ldg(m_row + d);
+        }
+      }
+      return;
+    }
     pr = __ldg(prefill + r);
     k = __ldg(snap + r);
     if (kBase) {  // precomputed network + prefix terms, carried as raw bits
@@ -510,7 +538,15 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
       if (dd >= 0 && (uint32_t)dd < D) {
 #pragma unroll
         for (int j = 0; j < NPT; ++j)
-          if (tid * NPT + j == (uint32_t)dd) load[j] -= l;
+          if (tid * NPT + j == (uint32_t)dd) {
+            if (kLoad) {
+              const uint32_t lam = min(16u * m[j], l);
+              load[j] += (int64_t)(l - lam) * (int64_t)w.bytes_per_token;
+              held[j] -= 1;
+            } else {
+              load[j] -= l;
+            }
+          }
       }
       continue;
     }
@@ -552,9 +588,18 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
     for (int j = 0; j < NPT; ++j) {
       const uint32_t d = tid * NPT + j;
       if (d < D) {
-        const bool feasible = load[j] + (int64_t)l <= w.cap_tokens;
+        bool feasible = load[j] + (int64_t)l <= w.cap_tokens;
         float sc, tj = 0.0f;
-        if (kBase) {
+        if (kLoad) {  // Sec. IV-B: T_queue + T_decode; Sec. IV-A: m_d >= s_eff + m_min
+          const uint32_t lam = min(16u * m[j], l);
+          feasible = load[j] >= (int64_t)(l - lam) * (int64_t)w.bytes_per_token + lm.m_min;
+          const int32_t beta = min(held[j], lm.beta_max);
+          const int32_t blocked = (held[j] - beta) - (lm.beta_max - beta);
+          const float t_queue = (blocked > 0 ? (float)blocked : 0.0f) * (lm.t_a + lm.t_b * (float)beta);
+          const float t_decode = lm.t_a + lm.t_b * (float)(beta + 1);
+          sc = base_score(w, l, m[j], pick4(ubp, tau[j]), ubd[j], pick4(lat, tau[j]), status) +
+               w.w_load * (t_queue + t_decode);
+        } else if (kBase) {
           sc = __uint_as_float(m[j]) + w.w_load * (w.theta_s_per_token * (float)load[j]);
         } else if (kInfl) {
           const float net_prefix =
@@ -602,6 +647,17 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
       parity ^= 1u;
     }
     const int32_t dstar = bi == kNone ? -1 : (int32_t)bi;
+    if constexpr (kLoad) {
+      if (dstar >= 0) {
+#pragma unroll
+        for (int j = 0; j < NPT; ++j)
+          if (tid * NPT + j == (uint32_t)dstar) {
+            const uint32_t lam = min(16u * m[j], l);
+            load[j] -= (int64_t)(l - lam) * (int64_t)w.bytes_per_token;
+            held[j] += 1;
+          }
+      }
+    }
     if constexpr (kInfl) {
       if (lead_thread) {
         if (dstar < 0) {
@@ -621,7 +677,7 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
         }
       }
     }
-    if (dstar >= 0) {
+    if (!kLoad && dstar >= 0) {
 #pragma unroll
       for (int j = 0; j < NPT; ++j)
         if (tid * NPT + j == (uint32_t)dstar) load[j] += l;
@@ -642,7 +698,10 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
 #pragma unroll
   for (int j = 0; j < NPT; ++j) {
     const uint32_t d = tid * NPT + j;
-    if (d < D) load_final[(uint64_t)stream * D + d] = load[j];
+    if (d < D) {
+      load_final[(uint64_t)stream * D + d] = load[j];
+      if (kLoad) n_final[(uint64_t)stream * D + d] = held[j];
+    }
   }
 }
 
@@ -1147,5 +1206,50 @@ extern "C" netkv_status netkv_schedule_streams_inflight(
   if (D <= 1024) NETKV_INFL(4, 256, 32);
   if (D <= 4096) NETKV_INFL(4, 1024, 32);
 #undef NETKV_INFL
+  return NETKV_EINVAL;
+}
+
+extern "C" netkv_status netkv_schedule_streams_load(
+    netkv_topology_t topo, uint32_t n_streams, const netkv_weights* d_w,
+    const netkv_load_model* model, uint32_t R, const uint32_t* d_len, const uint32_t* d_prefill,
+    const uint32_t* d_snap, const uint16_t* d_M, const float* d_UB, uint32_t n_snap,
+    const uint32_t* d_events, const uint64_t* d_event_off, const int64_t* d_m_init,
+    const int32_t* d_n_init, int32_t* d_dec, float* d_best, float* d_second, int64_t* d_m_final,
+    int32_t* d_n_final, int* d_status, netkv_stream_t stream) {
+  if (!topo || !d_w || !model || !d_event_off || !d_m_final || !d_n_final) return NETKV_EINVAL;
+  if (model->beta_max < 1 || !(model->t_a_s >= 0) || !(model->t_b_s >= 0) ||
+      !isfinite(model->t_a_s) || !isfinite(model->t_b_s) || model->m_min_bytes < 0)
+    return NETKV_EINVAL;
+  if (n_streams == 0) return NETKV_OK;
+  if (n_streams > 0x7fffffffu) return NETKV_EINVAL;
+  if (R > 0 && (!d_len || !d_prefill || !d_snap || !d_M || !d_UB || !d_dec || !d_best ||
+                !d_second || !d_events))
+    return NETKV_EINVAL;
+  if (!aligned_to(d_w, 8) || !aligned_to(d_UB, 16) || !aligned_to(d_event_off, 8) ||
+      !aligned_to(d_m_final, 8) || !aligned_to(d_n_final, 4) ||
+      (d_m_init && !aligned_to(d_m_init, 8)) || (d_n_init && !aligned_to(d_n_init, 4)))
+    return NETKV_EINVAL;
+  const TopoArgs t = topo_args(topo);
+  const uint32_t D = t.D;
+  cudaStream_t s = (cudaStream_t)stream;
+  const LoadModel lm = {model->t_a_s, model->t_b_s, model->beta_max, model->m_min_bytes,
+                        model->m0_bytes};
+#define NETKV_LOAD(NPT, BLOCK, LPS)                                                             \
+  do {                                                                                          \
+    const uint32_t per_cta = LPS == 32 ? 1u : 32u / LPS;                                        \
+    schedule_kernel<NPT, BLOCK, LPS, false, false, true>                                        \
+        <<<(n_streams + per_cta - 1) / per_cta, BLOCK, 0, s>>>(                                 \
+            t, n_streams, d_w, R, nullptr, d_len, d_prefill, d_snap, d_M, d_UB, n_snap,         \
+            d_events, d_event_off, d_m_init, d_dec, d_best, d_second, d_m_final, d_status,      \
+            nullptr, 0u, nullptr, 0u, 0u, lm, d_n_init, d_n_final);                             \
+    return netkv_launch_status();                                                               \
+  } while (0)
+  if (D <= 8) NETKV_LOAD(1, 32, 8);
+  if (D <= 16) NETKV_LOAD(1, 32, 16);
+  if (D <= 32) NETKV_LOAD(1, 32, 32);
+  if (D <= 256) NETKV_LOAD(1, 256, 32);
+  if (D <= 1024) NETKV_LOAD(4, 256, 32);
+  if (D <= 4096) NETKV_LOAD(4, 1024, 32);
+#undef NETKV_LOAD
   return NETKV_EINVAL;
 }

@@ -36,6 +36,7 @@ EXPORTS = ("netkv_topology_create", "netkv_topology_destroy", "netkv_topology_qu
            "netkv_prefix_match_workspace_size",
            "netkv_prefix_match", "netkv_prefix_match_static", "netkv_schedule_workspace_size",
            "netkv_schedule_streams", "netkv_schedule_streams_inflight",
+           "netkv_schedule_streams_load",
            "netkv_copy_async", "netkv_version")
 
 
@@ -80,6 +81,15 @@ _lib.netkv_schedule_streams.argtypes = [_P, _U32, _P, _U32, _P, _P, _P, _P, _P, 
 _lib.netkv_schedule_streams_inflight.argtypes = [_P, _U32, _P, _U32, _P, _P, _P, _P, _P, _P,
                                                  _U32, _P, _P, _U32, _P, _P, _P, _P, _P, _P,
                                                  _P, _P]
+class LoadModel(C.Structure):
+    """netkv_load_model: the paper's compute-load model constants (Sec. III-C, IV-B)."""
+    _fields_ = [("t_a_s", C.c_float), ("t_b_s", C.c_float), ("beta_max", C.c_int32),
+                ("reserved", C.c_int32), ("m_min_bytes", C.c_int64), ("m0_bytes", C.c_int64)]
+
+
+_lib.netkv_schedule_streams_load.argtypes = [_P, _U32, _P, C.POINTER(LoadModel), _U32, _P, _P,
+                                             _P, _P, _P, _U32, _P, _P, _P, _P, _P, _P, _P, _P,
+                                             _P, _P, _P]
 _lib.netkv_copy_async.argtypes = [_P, _P, C.c_size_t, _P]
 for _f in EXPORTS:
     if _f not in ("netkv_version", "netkv_prefix_match_workspace_size", "netkv_cache_index_bytes",
@@ -239,6 +249,18 @@ def netkv_oracle_build_tiers(topo: Topology, c, n_snap: int, kv_bytes: float, C=
     _check("netkv_oracle_build_tiers", _lib.netkv_oracle_build_tiers(
         topo.handle, _ptr(c), int(n_snap), float(kv_bytes), _ptr(C), _ptr(UB), _ptr(status),
         _stream(stream)))
+
+
+def netkv_schedule_streams_load(topo: Topology, n_streams: int, weights, model: LoadModel, R: int,
+                                length, prefill, snap, M, UB, n_snap: int, events, event_off,
+                                m_init, n_init, dec, best, second, m_final, n_final,
+                                status=None, stream=None) -> None:
+    """Algorithm 1 with the paper's compute-load model; see include/netkv.h."""
+    _check("netkv_schedule_streams_load", _lib.netkv_schedule_streams_load(
+        topo.handle, int(n_streams), _ptr(weights), C.byref(model), int(R), _ptr(length),
+        _ptr(prefill), _ptr(snap), _ptr(M), _ptr(UB), int(n_snap), _ptr(events), _ptr(event_off),
+        _ptr(m_init), _ptr(n_init), _ptr(dec), _ptr(best), _ptr(second), _ptr(m_final),
+        _ptr(n_final), _ptr(status), _stream(stream)))
 
 
 def netkv_copy_async(dst, src, nbytes: int, stream=None) -> None:

@@ -72,6 +72,13 @@ def test_version_and_host_validation(lib):
     assert so.netkv_topology_destroy(None) == lib.NETKV_EINVAL
 
 
+def test_load_model_layout(lib):
+    """netkv_load_model: two floats, two int32, two int64 in 32 bytes."""
+    M = lib.LoadModel
+    assert C.sizeof(M) == 32
+    assert [getattr(M, f).offset for f, _ in M._fields_] == [0, 4, 8, 12, 16, 24]
+
+
 def test_weights_layout(lib):
     assert lib.WEIGHTS_DTYPE.itemsize == 32
     assert [lib.WEIGHTS_DTYPE.fields[k][1] for k in lib.WEIGHTS_DTYPE.names] == [0, 4, 8, 12, 16, 24]
