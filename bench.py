@@ -33,6 +33,10 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "decisions/sec"
+# the paper's compute-load model for --load-model: t_iter = 12 ms + 0.4 ms per batch slot
+# (free constants: the paper's fit is not printed), 64 batch slots, 1 GB held back and
+# 45 GB free per decode GPU at the start (Sec. VI-A); the same in the CPU oracle leg
+LOAD_MODEL = (float(np.float32(0.012)), float(np.float32(0.0004)), 64, 0, 10 ** 9, 45 * 10 ** 9)
 UNIT = "decisions/s"
 
 
@@ -48,6 +52,9 @@ def parse():
     ap.add_argument("--snapshots", type=int, default=1000)
     ap.add_argument("--directed", action="store_true",
                     help="directed links: separate upward and downward utilisation rows")
+    ap.add_argument("--load-model", action="store_true",
+                    help="the paper's compute-load model (T_queue + T_decode, memory filter) "
+                         "instead of the token load")
     ap.add_argument("--tiers", action="store_true",
                     help="the paper's per-tier maps: four congestion values per snapshot")
     ap.add_argument("--inflight", type=int, default=0,
@@ -172,7 +179,7 @@ MEASURED_TRAFFIC = {
                      "sha256_16": "e98bf5d31ac767be", "bytes": 25_613_000_000},
     # the 1,000-snapshot oracle-build sweep (scaled by snapshots for other sizes)
     "oracle_build": {"source": "paper_2606_03910_gb300/csrc/oracle_build.cu",
-                     "sha256_16": "01d454368c851284", "bytes": 67_156_540_000},
+                     "sha256_16": "006b078542d734e5", "bytes": 67_155_930_000},
 }
 
 
@@ -205,14 +212,18 @@ def measured_peaks():
 
 
 # ------------------------------------------------------------------ CPU oracle
-def cpu_oracle_sample(w, streams, theta, cap, bpt, inflight=0, directed=False, tiers=False):
+def cpu_oracle_sample(w, streams, theta, cap, bpt, inflight=0, directed=False, tiers=False,
+                      load_model=False):
     """Time the CPU oracle on whole streams of the workload (with self-contention when
     inflight > 0, with directed links when directed); returns (decisions, seconds)."""
-    from oracle.workload import run_stream, run_stream_inflight
+    from oracle.workload import run_stream, run_stream_inflight, run_stream_load
     t0 = time.perf_counter()
     dec = 0
     for s in streams:
-        if inflight > 0:
+        if load_model:
+            a, b, bmax, _, m_min, m0 = LOAD_MODEL
+            res = run_stream_load(w, int(s), a, b, bmax, m_min, m0, bpt)
+        elif inflight > 0:
             res = run_stream_inflight(w, int(s), theta, cap, bpt, inflight)
         else:
             res = run_stream(w, int(s), theta, cap, bpt, directed=directed, tiers=tiers)
@@ -437,6 +448,9 @@ def run_netkv(args):
                                    directed=args.directed, tiers=args.tiers)
     sc.share_prefixes = not args.no_share
     sc.inflight_cap = args.inflight
+    if args.load_model:
+        from paper_2606_03910_gb300 import netkv
+        sc.load_model = netkv.LoadModel(*LOAD_MODEL)
     theta = float(np.float32(synth.THETA_S_PER_TOKEN))
     bpt = synth.BYTES_PER_TOKEN_SHARD
     spec = w.spec
@@ -480,7 +494,8 @@ def run_netkv(args):
     # level bottlenecks 1; prefix match 4 (group insert, group resolve, leaders, members)
     # with a workspace or 1 without; greedy 2 (base scores + walk) with a workspace or 1
     launches_per_step = 1 + (4 if sc.share_prefixes else 1) + (
-        1 if sc.inflight_cap > 0 else (2 if sc.precompute_scores else 1))
+        1 if (sc.inflight_cap > 0 or sc.load_model is not None)
+        else (2 if sc.precompute_scores else 1))
     n_input_tensors = sum(1 for f in dataclasses.fields(StepInputs)
                           if isinstance(getattr(x, f.name), torch.Tensor))
     decisions = R * world
@@ -558,7 +573,7 @@ def run_netkv(args):
         sample = np.random.default_rng(0).choice(args.streams, size=min(args.cpu_streams, args.streams),
                                                  replace=False)
         d, secs = cpu_oracle_sample(w, sample, theta, spec.cap_tokens, bpt, args.inflight,
-                                    args.directed, args.tiers)
+                                    args.directed, args.tiers, args.load_model)
         cpu = {"value": d / secs, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                "sample": f"{len(sample)} of {args.streams} streams, whole streams "
                          f"({d} decisions in {secs:.1f} s)"}
@@ -581,7 +596,9 @@ def run_netkv(args):
                                                      ([("links", "directed")]
                                                       if args.directed else []) +
                                                      ([("oracle", "per-tier maps")]
-                                                      if args.tiers else [])) or None),
+                                                      if args.tiers else []) +
+                                                     ([("load", "queue/decode-step model")]
+                                                      if args.load_model else [])) or None),
                 "scores_per_s": value * D, "gpu_launches": launches_per_step * args.steps,
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk}
         print(json.dumps(line), flush=True)
@@ -696,8 +713,9 @@ def run_sweep(args):
 
 def main():
     args = parse()
-    if (args.inflight > 0) + args.directed + args.tiers > 1:
-        raise SystemExit("--inflight, --directed and --tiers are measured one at a time")
+    if (args.inflight > 0) + args.directed + args.tiers + args.load_model > 1:
+        raise SystemExit("--inflight, --directed, --tiers and --load-model are measured one "
+                         "at a time")
     if args.impl == "reference":
         return run_reference(args)
     if args.workload == "sweep":

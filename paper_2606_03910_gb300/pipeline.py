@@ -69,6 +69,7 @@ class StepOutputs:
     load_final: torch.Tensor  # i64 [n_streams, D]
     status: torch.Tensor      # i32 [1]
     xfer_us: Optional[torch.Tensor] = None  # i32 [R], with self-contention
+    held_final: Optional[torch.Tensor] = None  # i32 [n_streams, D], with the load model
 
 
 class Scorer:
@@ -94,6 +95,9 @@ class Scorer:
         # "links": per-link utilisation rows; "tiers": the paper's per-tier maps, x.util
         # then holds four congestion values per snapshot
         self.oracle_mode = "links"
+        # the paper's compute-load model (netkv.LoadModel) instead of the token load;
+        # out.load_final then holds free bytes and out.held_final request counts
+        self.load_model = None
 
     def _sched_workspace(self, R: int):
         """Greedy workspace (base scores of every arrival), grown on demand."""
@@ -134,7 +138,8 @@ class Scorer:
             second=torch.empty(R, dtype=torch.float32, device=dev),
             load_final=torch.empty((n_streams, self.D), dtype=torch.int64, device=dev),
             status=torch.zeros(1, dtype=torch.int32, device=dev),
-            xfer_us=torch.empty(R, dtype=torch.int32, device=dev))
+            xfer_us=torch.empty(R, dtype=torch.int32, device=dev),
+            held_final=torch.empty((n_streams, self.D), dtype=torch.int32, device=dev))
 
     def oracle_build(self, x: StepInputs, out: StepOutputs, stream=None) -> None:
         if self.oracle_mode == "tiers":
@@ -153,6 +158,12 @@ class Scorer:
                                  out.status, stream, workspace=self._workspace(x.R))
 
     def schedule(self, x: StepInputs, out: StepOutputs, stream=None) -> None:
+        if self.load_model is not None:
+            netkv.netkv_schedule_streams_load(
+                self.topo, x.n_streams, x.weights, self.load_model, x.R, x.length, x.prefill,
+                x.snap, out.M, out.UB, x.n_snap, x.events, x.event_off, None, None, out.dec,
+                out.best, out.second, out.load_final, out.held_final, out.status, stream)
+            return
         if self.inflight_cap > 0:
             netkv.netkv_schedule_streams_inflight(
                 self.topo, x.n_streams, x.weights, x.R, x.length, x.prefill, x.snap,
