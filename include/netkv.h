@@ -301,13 +301,19 @@ netkv_status netkv_schedule_streams(netkv_topology_t topo, uint32_t n_streams,
  * xfer_us[r] is its T_xfer rounded to whole microseconds; a completion lowers the
  * counter by one unless it is zero.  Completions due at or before an arrival's time
  * are applied before that arrival is scored.  inflight_cap = 0 keeps every counter at
- * zero: the result is then that of netkv_schedule_streams without a workspace.
+ * zero: the result is then that of netkv_schedule_streams (without a workspace when
+ * d_workspace is NULL).
  *
  *   d_arrival_us [R] int64 arrival time of each request in microseconds; a stream's
  *                arrivals must be in time order, as its events are
  *   inflight_cap 0 .. 255 (the paper's default is 16)
  *   d_xfer_us    [R] int32 output: T_xfer of the chosen candidate in whole microseconds
  *                (at most 2^31 - 1), -1 for a rejected arrival
+ *   d_workspace  NULL, or at least netkv_schedule_inflight_workspace_size(R, D) bytes,
+ *                256-byte aligned: the decision-independent score part and s_eff / Bbot of
+ *                every (arrival, decode) are then computed first in parallel, and the walk
+ *                adds w_net * (s_eff / Bbot) * n and the load term; with inflight_cap = 0
+ *                the result is then netkv_schedule_streams' with a workspace.
  * Other arguments as for netkv_schedule_streams.  Limits: fewer than 16,384 prefill
  * ranks; the counters (4 bytes per prefill rank) and the pending completions of a
  * stream live in shared memory, 4,096 pending completions per stream for pools of more
@@ -315,13 +321,15 @@ netkv_status netkv_schedule_streams(netkv_topology_t topo, uint32_t n_streams,
  * completion that does not fit sets EFULL and is dropped (its counter is not lowered).
  * Host errors: EINVAL for a cap above 255, too many prefill ranks or missing buffers.
  */
+size_t netkv_schedule_inflight_workspace_size(uint32_t R, uint32_t D);
 netkv_status netkv_schedule_streams_inflight(
     netkv_topology_t topo, uint32_t n_streams, const netkv_weights* d_w, uint32_t R,
     const uint32_t* d_len, const uint32_t* d_prefill, const uint32_t* d_snap,
     const int64_t* d_arrival_us, const uint16_t* d_M, const float* d_UB, uint32_t n_snap,
     const uint32_t* d_events, const uint64_t* d_event_off, uint32_t inflight_cap,
     const int64_t* d_load_init, int32_t* d_dec, float* d_best, float* d_second,
-    int32_t* d_xfer_us, int64_t* d_load_final, int* d_status, netkv_stream_t stream);
+    int32_t* d_xfer_us, int64_t* d_load_final, void* d_workspace, size_t workspace_bytes,
+    int* d_status, netkv_stream_t stream);
 
 /* The paper's compute-load model (Sec. III-C decode state, Sec. IV-B component models). */
 typedef struct {

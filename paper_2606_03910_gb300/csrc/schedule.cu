@@ -84,7 +84,8 @@ __device__ __forceinline__ float contended_score(const netkv_weights& w, uint32_
     lam = lam < l ? lam : l;
   }
   const uint32_t miss_tok = l - lam;
-  const float b_eff = fminf(ub_p, ub_d) / (float)(1u + n);
+  const float bb = fminf(ub_p, ub_d);
+  const float b_eff = n ? bb / (float)(1u + n) : bb;
   const float s_eff = (float)((int64_t)miss_tok * (int64_t)w.bytes_per_token);
   T = s_eff / b_eff + lat_tau;
   const float miss = (float)miss_tok / (float)l;
@@ -150,6 +151,15 @@ struct DoneHeap {
   }
 };
 
+// s_eff / Bbot, the factor self-contention multiplies by 1 + n (Eq. 4): written beside
+// the base scores when the greedy runs with self-contention.
+__device__ __forceinline__ float xfer_factor(const netkv_weights& w, uint32_t l, uint32_t m,
+                                             float ub_p, float ub_d) {
+  const uint32_t lam = min(16u * m, l);
+  const float s_eff = (float)((int64_t)(l - lam) * (int64_t)w.bytes_per_token);
+  return s_eff / fminf(ub_p, ub_d);
+}
+
 // Base scores of every arrival: base[r][d] = base_score(...) for the stream's weights.
 // No dependence between events, so the events of a stream are split into contiguous
 // ranges over the segments (LPS lanes each) of grid.y blocks; each segment strides over
@@ -160,7 +170,8 @@ __global__ void __launch_bounds__(256, 8) base_kernel(
     const uint32_t* __restrict__ len, const uint32_t* __restrict__ prefill,
     const uint32_t* __restrict__ snap, const uint16_t* __restrict__ M,
     const float* __restrict__ UB, uint32_t n_snap, const uint32_t* __restrict__ events,
-    const uint64_t* __restrict__ event_off, float* __restrict__ base, int* status) {
+    const uint64_t* __restrict__ event_off, float* __restrict__ base, int* status,
+    float* __restrict__ X = nullptr) {
   constexpr uint32_t kSegs = 256 / LPS;
   const uint32_t seg = threadIdx.x / LPS, sl = threadIdx.x % LPS;
   const uint32_t D = t.D, N = t.N;
@@ -192,6 +203,7 @@ __global__ void __launch_bounds__(256, 8) base_kernel(
         const float ubd = __ldg(ub_row + (uint64_t)ld.x * 4 + tau);
         const uint32_t m = __ldg(M + (uint64_t)r * D + d);
         base[(uint64_t)r * D + d] = base_score(w, l, m, pick4(ubp, tau), ubd, pick4(lat, tau), status);
+        if (X) X[(uint64_t)r * D + d] = xfer_factor(w, l, m, pick4(ubp, tau), ubd);
       }
     }
   }
@@ -210,7 +222,8 @@ __global__ void __launch_bounds__(256) base_wide_kernel(
     const uint32_t* __restrict__ len, const uint32_t* __restrict__ prefill,
     const uint32_t* __restrict__ snap, const uint16_t* __restrict__ M,
     const float* __restrict__ UB, uint32_t n_snap, const uint32_t* __restrict__ events,
-    const uint64_t* __restrict__ event_off, float* __restrict__ base, int* status) {
+    const uint64_t* __restrict__ event_off, float* __restrict__ base, int* status,
+    float* __restrict__ X = nullptr) {
   constexpr uint32_t kChunk = 256u * NPT;
   constexpr uint32_t kBad = 0xffffffffu;
   const uint32_t D = t.D, N = t.N;
@@ -283,6 +296,7 @@ __global__ void __launch_bounds__(256) base_wide_kernel(
         const int tau = tier_of(lp, ld[j]);
         const float ubd = d0 + j < D ? __ldg(ub_row + (uint64_t)ld[j].x * 4 + tau) : 1.0f;
         out[j] = base_score(w, l, m[j], pick4(ubp, tau), ubd, pick4(lat, tau), status);
+        if (X && d0 + j < D) X[(uint64_t)r * D + d0 + j] = xfer_factor(w, l, m[j], pick4(ubp, tau), ubd);
       }
       float* brow = base + (uint64_t)r * D + d0;
       if (vec) {
@@ -323,9 +337,8 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
     const int64_t* __restrict__ arrival_us = nullptr, uint32_t inflight_cap = 0,
     int32_t* __restrict__ xfer_us = nullptr, uint32_t infl_bytes = 0, uint32_t heap_cap = 0,
     LoadModel lm = LoadModel{0.f, 0.f, 0, 0, 0}, const int32_t* __restrict__ n_init = nullptr,
-    int32_t* __restrict__ n_final = nullptr) {
+    int32_t* __restrict__ n_final = nullptr, const float* __restrict__ xf = nullptr) {
   static_assert(LPS == 32 || (BLOCK == 32 && NPT == 1), "packed streams use one warp");
-  static_assert(!(kBase && kInfl), "self-contention scores from UB and M");
   static_assert(!(kLoad && (kBase || kInfl)), "the load model scores from UB and M alone");
   constexpr int NW = BLOCK / 32;
   __shared__ float s_b[2][NW];
@@ -390,6 +403,7 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
   const uint32_t kBad = 0xffffffffu;
   uint32_t cq[CD + 1];                        // event codes, index i = event e+i
   uint32_t lq[FD + 1], pq[FD + 1], kq[FD + 1], mq[FD + 1][NPT];
+  float xq[FD + 1][NPT];  // s_eff / Bbot with self-contention over base scores
   int64_t tq[FD + 1];                         // arrival times (self-contention only)
   float4 ubpq[PD + 1];
   float ubdq[PD + 1][NPT];
@@ -458,15 +472,29 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
       if (lane == 0) dec_pref = *((volatile int32_t*)(dec + r));
       return;
     }
-    if (kBase || pr >= t.P || k >= n_snap) return;
+    if ((kBase && !kInfl) || pr >= t.P || k >= n_snap) return;
     const uint32_t pinst = __ldg(t.pre + pr);
     const uint4 lp = __ldg(t.links + pinst);
-    ubp = __ldg(reinterpret_cast<const float4*>(UB) + (uint64_t)k * N + pinst);
+    if (!kBase) ubp = __ldg(reinterpret_cast<const float4*>(UB) + (uint64_t)k * N + pinst);
     const float* ub_row = UB + (uint64_t)k * N * 4;
 #pragma unroll
     for (int j = 0; j < NPT; ++j) {
       tau[j] = tier_of(lp, ld[j]);
-      if (tid * NPT + j < D) ubd[j] = __ldg(ub_row + (uint64_t)ld[j].x * 4 + tau[j]);
+      if (!kBase && tid * NPT + j < D) ubd[j] = __ldg(ub_row + (uint64_t)ld[j].x * 4 + tau[j]);
+    }
+  };
+  // with self-contention over base scores: the arrival's s_eff / Bbot row
+  auto xrow = [&](uint32_t code, float* x) {
+#pragma unroll
+    for (int j = 0; j < NPT; ++j) x[j] = 0.0f;
+    if (!(kBase && kInfl) || code == kBad || (code >> 31)) return;
+    const uint32_t r = code & 0x7fffffffu;
+    if (r >= R) return;
+    const float* x_row = xf + (uint64_t)r * D;
+#pragma unroll
+    for (int j = 0; j < NPT; ++j) {
+      const uint32_t d = tid * NPT + j;
+      if (d < D) x[j] = __ldg(x_row + d);
     }
   };
 
@@ -479,6 +507,7 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
 #pragma unroll
   for (int i = 0; i <= FD; ++i) {
     fields(cq[i], lq[i], pq[i], kq[i], mq[i]);
+    xrow(cq[i], xq[i]);
     tq[i] = time_of(cq[i]);
   }
 #pragma unroll
@@ -492,11 +521,13 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
     float ubd[NPT];
     int tau[NPT];
     uint32_t m[NPT];
+    float xv[NPT];
 #pragma unroll
     for (int j = 0; j < NPT; ++j) {
       ubd[j] = ubdq[0][j];
       tau[j] = tauq[0][j];
       m[j] = mq[0][j];
+      xv[j] = xq[0][j];
     }
     const int32_t dec_pref = decq[0];
 #pragma unroll
@@ -508,7 +539,10 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
       kq[i] = kq[i + 1];
       tq[i] = tq[i + 1];
 #pragma unroll
-      for (int j = 0; j < NPT; ++j) mq[i][j] = mq[i + 1][j];
+      for (int j = 0; j < NPT; ++j) {
+        mq[i][j] = mq[i + 1][j];
+        xq[i][j] = xq[i + 1][j];
+      }
     }
 #pragma unroll
     for (int i = 0; i < PD; ++i) {
@@ -522,6 +556,7 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
     }
     cq[CD] = (e + 1 + CD < e1) ? __ldg(events + e + 1 + CD) : kBad;
     fields(cq[FD], lq[FD], pq[FD], kq[FD], mq[FD]);
+    xrow(cq[FD], xq[FD]);
     tq[FD] = time_of(cq[FD]);
     operands(cq[PD], pq[PD], kq[PD], ubpq[PD], ubdq[PD], tauq[PD], decq[PD]);
 
@@ -599,6 +634,11 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
           const float t_decode = lm.t_a + lm.t_b * (float)(beta + 1);
           sc = base_score(w, l, m[j], pick4(ubp, tau[j]), ubd[j], pick4(lat, tau[j]), status) +
                w.w_load * (t_queue + t_decode);
+        } else if (kBase && kInfl) {  // base + w_net (s_eff / Bbot) n: Eq. 4's 1 + n
+          const uint32_t n = (cw >> (8 * tau[j])) & 0xffu;
+          sc = (__uint_as_float(m[j]) + w.w_net * (xv[j] * (float)n)) +
+               w.w_load * (w.theta_s_per_token * (float)load[j]);
+          tj = xv[j] * (float)(1u + n) + pick4(lat, tau[j]);
         } else if (kBase) {
           sc = __uint_as_float(m[j]) + w.w_load * (w.theta_s_per_token * (float)load[j]);
         } else if (kInfl) {
@@ -659,16 +699,22 @@ __global__ void __launch_bounds__(BLOCK) schedule_kernel(
       }
     }
     if constexpr (kInfl) {
+      // the winner's tier: packed streams own one decode a lane, so its lane has it
+      uint32_t ts_lane = 0;
+      if (LPS < 32) ts_lane = (uint32_t)__shfl_sync(smask, tau[0], dstar < 0 ? 0 : dstar, LPS);
       if (lead_thread) {
         if (dstar < 0) {
           xfer_us[r] = -1;
         } else {  // the dispatch's tier counter (Algorithm 1 line 14) and its completion
-          const double us = (double)bt * 1e6;
-          const int64_t dt = us < 2147483647.0 ? (int64_t)llrint(us) : 2147483647ll;
+          const float us = bt * 1.0e6f;
+          const int64_t dt = us < 2147483520.0f ? __float2ll_rn(us) : 2147483647ll;
           xfer_us[r] = (int32_t)dt;
-          const uint4 lp = __ldg(t.links + __ldg(t.pre + pr));
-          const uint4 lo = __ldg(t.links + __ldg(t.dec + (uint32_t)dstar));
-          const uint32_t ts = (uint32_t)tier_of(lp, lo);
+          uint32_t ts = ts_lane;
+          if (LPS == 32) {
+            const uint4 lp = __ldg(t.links + __ldg(t.pre + pr));
+            const uint4 lo = __ldg(t.links + __ldg(t.dec + (uint32_t)dstar));
+            ts = (uint32_t)tier_of(lp, lo);
+          }
           uint32_t* c = cnt + pr;
           const uint32_t sh = 8u * ts;
           if (((*c >> sh) & 0xffu) < inflight_cap) *c += 1u << sh;
@@ -1021,28 +1067,25 @@ netkv_status launch_staged(const TopoArgs& t, uint32_t n_streams, const netkv_we
   return netkv_launch_status();
 }
 
-template <int NPT, int BLOCK, int LPS>
-netkv_status launch(const TopoArgs& t, uint32_t n_streams, const netkv_weights* d_w, uint32_t R,
-                    const uint32_t* d_len, const uint32_t* d_prefill, const uint32_t* d_snap,
-                    const uint16_t* d_M, const float* d_UB, uint32_t n_snap,
-                    const uint32_t* d_events, const uint64_t* d_event_off,
-                    const int64_t* d_load_init, int32_t* d_dec, float* d_best, float* d_second,
-                    int64_t* d_load_final, float* d_base, int* d_status, cudaStream_t s) {
-  const uint32_t per_cta = LPS == 32 ? 1u : 32u / LPS;
-  const unsigned grid = (n_streams + per_cta - 1) / per_cta;
-  if (d_base) {
+// The base-score pre-pass over every arrival (and, with d_X, the factor s_eff / Bbot that
+// self-contention scales).
+netkv_status launch_base(const TopoArgs& t, uint32_t n_streams, const netkv_weights* d_w,
+                         uint32_t R, const uint32_t* d_len, const uint32_t* d_prefill,
+                         const uint32_t* d_snap, const uint16_t* d_M, const float* d_UB,
+                         uint32_t n_snap, const uint32_t* d_events, const uint64_t* d_event_off,
+                         float* d_base, float* d_X, int* d_status, cudaStream_t s) {
     const uint32_t D = t.D;
     const unsigned gy = n_streams >= 1024u ? 1u : (1024u + n_streams - 1) / n_streams;
     const dim3 bgrid(n_streams < (1u << 20) ? n_streams : (1u << 20), gy);
     if (D <= 8)
       base_kernel<8><<<bgrid, 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,
-                                           d_UB, n_snap, d_events, d_event_off, d_base, d_status);
+                                           d_UB, n_snap, d_events, d_event_off, d_base, d_status, d_X);
     else if (D <= 16)
       base_kernel<16><<<bgrid, 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,
-                                            d_UB, n_snap, d_events, d_event_off, d_base, d_status);
+                                            d_UB, n_snap, d_events, d_event_off, d_base, d_status, d_X);
     else if (D <= 32)
       base_kernel<32><<<bgrid, 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,
-                                            d_UB, n_snap, d_events, d_event_off, d_base, d_status);
+                                            d_UB, n_snap, d_events, d_event_off, d_base, d_status, d_X);
     else {
       // one block per (stream, chunk of decodes) and arrival segment, ~32 blocks per SM
       int dev = 0, sms = 0;
@@ -1056,13 +1099,28 @@ netkv_status launch(const TopoArgs& t, uint32_t n_streams, const netkv_weights* 
       if (D <= 256)
         base_wide_kernel<1><<<dim3(wx, wy), 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill,
                                                          d_snap, d_M, d_UB, n_snap, d_events,
-                                                         d_event_off, d_base, d_status);
+                                                         d_event_off, d_base, d_status, d_X);
       else
         base_wide_kernel<4><<<dim3(wx, wy), 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill,
                                                          d_snap, d_M, d_UB, n_snap, d_events,
-                                                         d_event_off, d_base, d_status);
+                                                         d_event_off, d_base, d_status, d_X);
     }
-    if (netkv_launch_status() != NETKV_OK) return NETKV_ECUDA;
+  return netkv_launch_status();
+}
+
+template <int NPT, int BLOCK, int LPS>
+netkv_status launch(const TopoArgs& t, uint32_t n_streams, const netkv_weights* d_w, uint32_t R,
+                    const uint32_t* d_len, const uint32_t* d_prefill, const uint32_t* d_snap,
+                    const uint16_t* d_M, const float* d_UB, uint32_t n_snap,
+                    const uint32_t* d_events, const uint64_t* d_event_off,
+                    const int64_t* d_load_init, int32_t* d_dec, float* d_best, float* d_second,
+                    int64_t* d_load_final, float* d_base, int* d_status, cudaStream_t s) {
+  const uint32_t per_cta = LPS == 32 ? 1u : 32u / LPS;
+  const unsigned grid = (n_streams + per_cta - 1) / per_cta;
+  if (d_base) {
+    if (launch_base(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events,
+                    d_event_off, d_base, nullptr, d_status, s) != NETKV_OK)
+      return NETKV_ECUDA;
     if (LPS == 32) {
       // one CTA per stream: the walk is bound by each warp's chain of dependent
       // instructions per event; 16 warps (4 per scheduler) measured best on 4,096 decodes
@@ -1105,13 +1163,34 @@ netkv_status launch_inflight(const TopoArgs& t, uint32_t n_streams, const netkv_
                              const uint32_t* d_events, const uint64_t* d_event_off,
                              uint32_t inflight_cap, const int64_t* d_load_init, int32_t* d_dec,
                              float* d_best, float* d_second, int32_t* d_xfer_us,
-                             int64_t* d_load_final, int* d_status, cudaStream_t s) {
+                             int64_t* d_load_final, float* d_base, float* d_X, int* d_status,
+                             cudaStream_t s) {
   const uint32_t per_cta = LPS == 32 ? 1u : 32u / LPS;
   const unsigned grid = (n_streams + per_cta - 1) / per_cta;
   const uint32_t heap_cap = LPS == 32 ? kHeapPerStream : kHeapPerPackedStream;
   const uint32_t infl_bytes = ((t.P * 4u + 15u) & ~15u) + heap_cap * 8u;
   const size_t smem = (size_t)per_cta * infl_bytes;
   if (smem > kInflightSmemMax) return NETKV_EINVAL;
+  if (d_base) {  // base scores and s_eff / Bbot of every arrival first, in parallel
+    if (launch_base(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events,
+                    d_event_off, d_base, d_X, d_status, s) != NETKV_OK)
+      return NETKV_ECUDA;
+    if (smem > 48u * 1024u) {
+      static bool raised = false;  // the same value every time: a benign race
+      if (!raised) {
+        NETKV_CUDA_TRY(cudaFuncSetAttribute(schedule_kernel<NPT, BLOCK, LPS, true, true>,
+                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                            (int)kInflightSmemMax));
+        raised = true;
+      }
+    }
+    schedule_kernel<NPT, BLOCK, LPS, true, true><<<grid, BLOCK, smem, s>>>(
+        t, n_streams, d_w, R, d_base, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events,
+        d_event_off, d_load_init, d_dec, d_best, d_second, d_load_final, d_status, d_arrival_us,
+        inflight_cap, d_xfer_us, infl_bytes, heap_cap, LoadModel{0.f, 0.f, 0, 0, 0}, nullptr,
+        nullptr, d_X);
+    return netkv_launch_status();
+  }
   if (smem > 48u * 1024u) {
     static bool raised = false;  // the same value every time: a benign race
     if (!raised) {
@@ -1172,13 +1251,18 @@ extern "C" netkv_status netkv_schedule_streams(
   return NETKV_EINVAL;
 }
 
+extern "C" size_t netkv_schedule_inflight_workspace_size(uint32_t R, uint32_t D) {
+  return 2 * netkv_schedule_workspace_size(R, D);
+}
+
 extern "C" netkv_status netkv_schedule_streams_inflight(
     netkv_topology_t topo, uint32_t n_streams, const netkv_weights* d_w, uint32_t R,
     const uint32_t* d_len, const uint32_t* d_prefill, const uint32_t* d_snap,
     const int64_t* d_arrival_us, const uint16_t* d_M, const float* d_UB, uint32_t n_snap,
     const uint32_t* d_events, const uint64_t* d_event_off, uint32_t inflight_cap,
     const int64_t* d_load_init, int32_t* d_dec, float* d_best, float* d_second,
-    int32_t* d_xfer_us, int64_t* d_load_final, int* d_status, netkv_stream_t stream) {
+    int32_t* d_xfer_us, int64_t* d_load_final, void* d_workspace, size_t workspace_bytes,
+    int* d_status, netkv_stream_t stream) {
   if (!topo || !d_w || !d_event_off || !d_load_final) return NETKV_EINVAL;
   if (inflight_cap > 255) return NETKV_EINVAL;
   if (n_streams == 0) return NETKV_OK;
@@ -1194,11 +1278,19 @@ extern "C" netkv_status netkv_schedule_streams_inflight(
   if (t.P >= (1u << 14)) return NETKV_EINVAL;  // prefill rank in a completion key
   const uint32_t D = t.D;
   cudaStream_t s = (cudaStream_t)stream;
+  if (d_workspace && (!aligned_to(d_workspace, 256) ||
+                      workspace_bytes < netkv_schedule_inflight_workspace_size(R, D)))
+    return NETKV_EINVAL;
+  float* d_base = (d_workspace && R > 0) ? reinterpret_cast<float*>(d_workspace) : nullptr;
+  float* d_X = d_base ? reinterpret_cast<float*>(reinterpret_cast<char*>(d_workspace) +
+                                                 netkv_schedule_workspace_size(R, D))
+                      : nullptr;
 #define NETKV_INFL(NPT, BLOCK, LPS)                                                             \
   return launch_inflight<NPT, BLOCK, LPS>(t, n_streams, d_w, R, d_len, d_prefill, d_snap,      \
                                           d_arrival_us, d_M, d_UB, n_snap, d_events,           \
                                           d_event_off, inflight_cap, d_load_init, d_dec,       \
-                                          d_best, d_second, d_xfer_us, d_load_final, d_status, s)
+                                          d_best, d_second, d_xfer_us, d_load_final, d_base,   \
+                                          d_X, d_status, s)
   if (D <= 8) NETKV_INFL(1, 32, 8);
   if (D <= 16) NETKV_INFL(1, 32, 16);
   if (D <= 32) NETKV_INFL(1, 32, 32);

@@ -36,6 +36,7 @@ EXPORTS = ("netkv_topology_create", "netkv_topology_destroy", "netkv_topology_qu
            "netkv_prefix_match_workspace_size",
            "netkv_prefix_match", "netkv_prefix_match_static", "netkv_schedule_workspace_size",
            "netkv_schedule_streams", "netkv_schedule_streams_inflight",
+           "netkv_schedule_inflight_workspace_size",
            "netkv_schedule_streams_load",
            "netkv_copy_async", "netkv_version")
 
@@ -80,7 +81,9 @@ _lib.netkv_schedule_streams.argtypes = [_P, _U32, _P, _U32, _P, _P, _P, _P, _P, 
                                         _P, _P, _P, _P, _P, _P, C.c_size_t, _P, _P]
 _lib.netkv_schedule_streams_inflight.argtypes = [_P, _U32, _P, _U32, _P, _P, _P, _P, _P, _P,
                                                  _U32, _P, _P, _U32, _P, _P, _P, _P, _P, _P,
-                                                 _P, _P]
+                                                 _P, C.c_size_t, _P, _P]
+_lib.netkv_schedule_inflight_workspace_size.argtypes = [_U32, _U32]
+_lib.netkv_schedule_inflight_workspace_size.restype = C.c_size_t
 class LoadModel(C.Structure):
     """netkv_load_model: the paper's compute-load model constants (Sec. III-C, IV-B)."""
     _fields_ = [("t_a_s", C.c_float), ("t_b_s", C.c_float), ("beta_max", C.c_int32),
@@ -93,7 +96,7 @@ _lib.netkv_schedule_streams_load.argtypes = [_P, _U32, _P, C.POINTER(LoadModel),
 _lib.netkv_copy_async.argtypes = [_P, _P, C.c_size_t, _P]
 for _f in EXPORTS:
     if _f not in ("netkv_version", "netkv_prefix_match_workspace_size", "netkv_cache_index_bytes",
-                  "netkv_schedule_workspace_size"):
+                  "netkv_schedule_workspace_size", "netkv_schedule_inflight_workspace_size"):
         getattr(_lib, _f).restype = C.c_int
 
 
@@ -226,13 +229,20 @@ def netkv_schedule_streams(topo: Topology, n_streams: int, weights, R: int, leng
 def netkv_schedule_streams_inflight(topo: Topology, n_streams: int, weights, R: int, length,
                                     prefill, snap, arrival_us, M, UB, n_snap: int, events,
                                     event_off, inflight_cap: int, load_init, dec, best, second,
-                                    xfer_us, load_final, status=None, stream=None) -> None:
+                                    xfer_us, load_final, status=None, stream=None,
+                                    workspace=None) -> None:
     """Algorithm 1 with self-contention; see include/netkv.h."""
+    ws_bytes = 0 if workspace is None else int(workspace.numel() * workspace.element_size())
     _check("netkv_schedule_streams_inflight", _lib.netkv_schedule_streams_inflight(
         topo.handle, int(n_streams), _ptr(weights), int(R), _ptr(length), _ptr(prefill),
         _ptr(snap), _ptr(arrival_us), _ptr(M), _ptr(UB), int(n_snap), _ptr(events),
         _ptr(event_off), int(inflight_cap), _ptr(load_init), _ptr(dec), _ptr(best),
-        _ptr(second), _ptr(xfer_us), _ptr(load_final), _ptr(status), _stream(stream)))
+        _ptr(second), _ptr(xfer_us), _ptr(load_final), _ptr(workspace), ws_bytes, _ptr(status),
+        _stream(stream)))
+
+
+def netkv_schedule_inflight_workspace_size(R: int, D: int) -> int:
+    return int(_lib.netkv_schedule_inflight_workspace_size(int(R), int(D)))
 
 
 def netkv_oracle_build_directed(topo: Topology, util_up, util_down, n_snap: int, kv_bytes: float,

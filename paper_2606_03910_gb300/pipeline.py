@@ -169,7 +169,7 @@ class Scorer:
                 self.topo, x.n_streams, x.weights, x.R, x.length, x.prefill, x.snap,
                 x.arrival_us, out.M, out.UB, x.n_snap, x.events, x.event_off, self.inflight_cap,
                 x.load_init, out.dec, out.best, out.second, out.xfer_us, out.load_final,
-                out.status, stream)
+                out.status, stream)  # the walk, not its scoring, bounds this form
             return
         netkv.netkv_schedule_streams(self.topo, x.n_streams, x.weights, x.R, x.length, x.prefill,
                                      x.snap, out.M, out.UB, x.n_snap, x.events, x.event_off,

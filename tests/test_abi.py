@@ -68,7 +68,8 @@ def test_version_and_host_validation(lib):
     assert so.netkv_schedule_workspace_size(10, 8) == 512
     assert so.netkv_schedule_streams_inflight(None, 1, None, 0, None, None, None, None, None,
                                               None, 0, None, None, 16, None, None, None, None,
-                                              None, None, None, None) == lib.NETKV_EINVAL
+                                              None, None, None, 0, None, None) == lib.NETKV_EINVAL
+    assert so.netkv_schedule_inflight_workspace_size(10, 8) == 1024
     assert so.netkv_topology_destroy(None) == lib.NETKV_EINVAL
 
 

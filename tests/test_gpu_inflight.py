@@ -37,7 +37,8 @@ def nk():
     return netkv
 
 
-def run_inflight(sc, x, out, inflight_cap, arrival):
+def run_inflight(sc, x, out, inflight_cap, arrival, workspace=False):
+    """workspace: the form with base scores and s_eff / Bbot computed first."""
     netkv = nk()
     R, S, D = x.R, x.n_streams, sc.D
     dev = out.M.device
@@ -50,7 +51,10 @@ def run_inflight(sc, x, out, inflight_cap, arrival):
     netkv.netkv_schedule_streams_inflight(sc.topo, S, x.weights, R, x.length, x.prefill, x.snap,
                                           arrival, out.M, out.UB, x.n_snap, x.events, x.event_off,
                                           inflight_cap, x.load_init, o["dec"], o["best"],
-                                          o["second"], o["xfer"], o["load"], o["status"])
+                                          o["second"], o["xfer"], o["load"], o["status"],
+                                          workspace=torch.empty(
+                                              netkv.netkv_schedule_inflight_workspace_size(R, D),
+                                              dtype=torch.uint8, device=dev) if workspace else None)
     torch.cuda.synchronize()
     return o
 
@@ -82,17 +86,22 @@ def _spec(fanout, rule, rate=2000.0, rps=120, n_streams=2):
 
 
 @pytest.mark.parametrize("fanout,rule,D", SHAPES)
-def test_inflight_cap0_is_the_plain_greedy(fanout, rule, D):
+@pytest.mark.parametrize("ws", [False, True])
+def test_inflight_cap0_is_the_plain_greedy(fanout, rule, D, ws):
+    """Without workspaces and with them, on each side."""
     netkv = nk()
     w, sc, x, out, arrival = _workload(_spec(fanout, rule))
     assert w.D == D
-    o = run_inflight(sc, x, out, 0, arrival)
+    o = run_inflight(sc, x, out, 0, arrival, workspace=ws)
     assert int(o["status"].item()) == 0
     plain = sc.alloc_outputs(x.n_snap, x.R, x.n_streams)
     netkv.netkv_schedule_streams(sc.topo, x.n_streams, x.weights, x.R, x.length, x.prefill,
                                  x.snap, out.M, out.UB, x.n_snap, x.events, x.event_off,
                                  x.load_init, plain.dec, plain.best, plain.second,
-                                 plain.load_final, plain.status)
+                                 plain.load_final, plain.status,
+                                 workspace=torch.empty(netkv.netkv_schedule_workspace_size(x.R, D),
+                                                       dtype=torch.uint8, device="cuda")
+                                 if ws else None)
     torch.cuda.synchronize()
     assert torch.equal(o["dec"], plain.dec)
     assert torch.equal(o["best"], plain.best) and torch.equal(o["second"], plain.second)
@@ -101,11 +110,11 @@ def test_inflight_cap0_is_the_plain_greedy(fanout, rule, D):
 
 
 @pytest.mark.parametrize("fanout,rule,D", SHAPES)
-@pytest.mark.parametrize("icap", [1, 2, 16])
-def test_inflight_streams_vs_oracle(fanout, rule, D, icap):
+@pytest.mark.parametrize("icap,ws", [(1, False), (2, False), (16, False), (2, True), (16, True)])
+def test_inflight_streams_vs_oracle(fanout, rule, D, icap, ws):
     from oracle.workload import run_stream_inflight
     w, sc, x, out, arrival = _workload(_spec(fanout, rule), n_prefills=4)
-    o = run_inflight(sc, x, out, icap, arrival)
+    o = run_inflight(sc, x, out, icap, arrival, workspace=ws)
     assert int(o["status"].item()) == 0
     dec, best, second = host(o["dec"]), host(o["best"]), host(o["second"])
     xfer, load = host(o["xfer"]), host(o["load"])
