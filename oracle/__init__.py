@@ -76,6 +76,10 @@ def _declare(l):
     l.oracle_schedule_stream_load.argtypes = [P, P, P, P, P, U64, P, P, P, P, P, U64, F64, F64,
                                               F64, U64, F64, F64, I64, I64, I64, P, P, P, F64,
                                               P, P, P, P, P, P]
+    l.oracle_schedule_stream_evolving.restype = None
+    l.oracle_schedule_stream_evolving.argtypes = [P, P, P, P, P, U64, P, P, P, P, P, P, P, P, U64,
+                                                  F64, F64, F64, F64, I64, U64, P, F64, P, P, P,
+                                                  P, P, P]
     l.oracle_cost_matrix_tiers.restype = None
     l.oracle_cost_matrix_tiers.argtypes = [P, P, P, P, P, U64, F64, P]
     l.oracle_cost_matrix_directed.restype = None
@@ -336,3 +340,40 @@ def schedule_stream_load(fanout, role, bw, lat, util, length, prefill, snap, M, 
         _p(dec), _p(best), _p(second), _p(n_out), _p(m_out), _p(counts))
     return LoadResult(dec, best, second, n_out, m_out, int(counts[0]), int(counts[1]),
                       int(counts[2]))
+
+
+class EvolvingResult(StreamResult):
+    def __init__(self, dec, best, second, load, M, near_ties, mismatches, rejects):
+        super().__init__(dec, best, second, load, near_ties, mismatches, rejects)
+        self.M = M
+
+
+def schedule_stream_evolving(fanout, role, bw, lat, util, length, prefill, snap, keys, key_off,
+                             chains, chain_off, events, w_net, w_prefix, w_load, theta, cap,
+                             bytes_per_token, hint=None, rel_tol=1e-5) -> EvolvingResult:
+    """Algorithm 1 with evolving caches (the simulator's cache update, without eviction):
+    keys/key_off [D+1] are the decodes' caches at the stream's start; a dispatch adds the
+    request's chain to its decode's cache; M is taken per arrival against the caches of
+    that moment and returned (.M)."""
+    f, ro = _c(fanout, np.uint32), _c(role, np.uint8)
+    b, la = _c(bw, np.float64), _c(lat, np.float64)
+    u = _c(util, np.float32)
+    ln, pf, sn = _c(length, np.uint32), _c(prefill, np.uint32), _c(snap, np.uint32)
+    k, ko = _c(keys, np.uint64), _c(key_off, np.uint64)
+    ch, co = _c(chains, np.uint64), _c(chain_off, np.uint64)
+    ev = _c(events, np.uint32)
+    R = len(ln)
+    D = int((ro == 1).sum())
+    assert len(ko) == D + 1 and len(co) == R + 1
+    dec = np.full(R, -1, np.int32)
+    best = np.full(R, np.inf); second = np.full(R, np.inf)
+    M = np.zeros((R, D), np.uint16)
+    load = np.zeros(D, np.int64)
+    counts = np.zeros(3, np.int64)
+    h = None if hint is None else _c(hint, np.int32)
+    lib().oracle_schedule_stream_evolving(
+        _p(f), _p(ro), _p(b), _p(la), _p(u), u.shape[1], _p(ln), _p(pf), _p(sn), _p(k), _p(ko),
+        _p(ch), _p(co), _p(ev), len(ev), float(w_net), float(w_prefix), float(w_load),
+        float(theta), int(cap), int(bytes_per_token), _p(h), float(rel_tol), _p(dec), _p(best),
+        _p(second), _p(M), _p(load), _p(counts))
+    return EvolvingResult(dec, best, second, load, M, int(counts[0]), int(counts[1]), int(counts[2]))

@@ -28,6 +28,9 @@
 //   * Algorithm 1 (Sec. IV-A) as a weighted score: filter by capacity (line 1), reject
 //     when nothing is feasible (line 2), score every candidate (lines 3-11), take the
 //     argmin with the lowest index among equal scores (line 13), then update load.
+//   * Evolving caches (the simulator's cache update, Sec. V-B, without LRU eviction), in
+//     oracle_schedule_stream_evolving: a dispatch adds the request's blocks to its
+//     decode's cache and later arrivals match against the grown caches.
 //   * The compute-load model (Sec. III-C, IV-B, the feasible set of Sec. IV-A), in
 //     oracle_schedule_stream_load: T_queue + T_decode from each decode's request count
 //     and t_iter(beta) = a + b beta, memory feasibility m_d >= s_eff + m_min.
@@ -621,6 +624,86 @@ void oracle_schedule_stream_load(
     n_out[d] = (int32_t)n[d];
     m_out[d] = m[d];
   }
+}
+
+// Algorithm 1 with evolving caches (the simulator's cache update of Sec. V-B, without its
+// LRU eviction): a stream starts from its decodes' cache contents (key lists keys,
+// key_off [D+1]); every arrival's prefix hits are taken against the caches as they are
+// at that arrival (first-miss scan, Sec. III-B), and a dispatch to d* adds every block of
+// the request's chain (chains, chain_off [R+1]) to K_{d*}.  Scores, feasibility and load
+// as oracle_schedule_stream.  M_out [R][D]: the hits each arrival was scored with.
+void oracle_schedule_stream_evolving(
+    const uint32_t* fanout, const uint8_t* role, const double* bw, const double* lat,
+    const float* util, uint64_t n_links, const uint32_t* len, const uint32_t* prefill,
+    const uint32_t* snap, const uint64_t* keys, const uint64_t* key_off,
+    const uint64_t* chains, const uint64_t* chain_off, const uint32_t* events,
+    uint64_t n_events, double w_net, double w_prefix, double w_load, double theta, int64_t cap,
+    uint64_t bytes_per_token, const int32_t* hint, double rel_tol, int32_t* dec, double* best,
+    double* second, uint16_t* M_out, int64_t* load_out, int64_t* counts) {
+  const Tree t = make_tree(fanout);
+  std::vector<uint64_t> pre, decs;
+  ranks(role, t.n, pre, decs);
+  const uint64_t D = decs.size();
+  std::vector<std::unordered_set<uint64_t>> K(D);
+  for (uint64_t d = 0; d < D; ++d)
+    for (uint64_t j = key_off[d]; j < key_off[d + 1]; ++j) K[d].insert(keys[j]);
+  std::vector<int64_t> load(D, 0);
+  std::vector<double> score(D);
+  const double inf = std::numeric_limits<double>::infinity();
+  for (uint64_t e = 0; e < n_events; ++e) {
+    const uint32_t code = events[e];
+    const uint32_t r = code & 0x7fffffffu;
+    const int64_t l = len[r];
+    if (code >> 31) {
+      if (dec[r] >= 0) load[dec[r]] -= l;
+      continue;
+    }
+    for (uint64_t d = 0; d < D; ++d) {  // hits against the caches as they are now
+      uint64_t m = 0;
+      for (uint64_t j = chain_off[r]; j < chain_off[r + 1]; ++j) {
+        if (K[d].count(chains[j]) == 0) break;
+        ++m;
+      }
+      M_out[(uint64_t)r * D + d] = (uint16_t)m;
+    }
+    const float* u_row = util + (uint64_t)snap[r] * n_links;
+    const uint64_t p = pre[prefill[r]];
+    int32_t arg = -1;
+    for (uint64_t d = 0; d < D; ++d) {
+      if (load[d] + l > cap) { score[d] = inf; continue; }
+      int tau = 0;
+      const double b = path_bottleneck(t, bw, u_row, p, decs[d], &tau);
+      const int64_t lam = 16 * (int64_t)M_out[(uint64_t)r * D + d];
+      const double s_eff = (double)((l - lam) * (int64_t)bytes_per_token);
+      const double T = s_eff / b + lat[tau];
+      const double miss = (double)(l - lam) / (double)l;
+      score[d] = w_net * T + w_prefix * miss + w_load * (theta * (double)load[d]);
+      if (arg < 0 || score[d] < score[arg]) arg = (int32_t)d;
+    }
+    double b1 = inf, b2 = inf;
+    if (arg >= 0) {
+      b1 = score[arg];
+      for (uint64_t d = 0; d < D; ++d)
+        if ((int32_t)d != arg && score[d] < b2) b2 = score[d];
+    }
+    int32_t chosen = arg;
+    if (hint && hint[r] != arg) {
+      const int32_t h = hint[r];
+      const bool near = (arg >= 0 && h >= 0 && (uint64_t)h < D && score[h] != inf &&
+                         score[h] - b1 <= rel_tol * std::fabs(b1));
+      counts[near ? 0 : 1] += 1;
+      chosen = (h >= 0 && (uint64_t)h < D) ? h : -1;
+    }
+    if (chosen < 0) counts[2] += 1;
+    dec[r] = chosen;
+    best[r] = b1;
+    second[r] = b2;
+    if (chosen >= 0) {
+      load[chosen] += l;
+      for (uint64_t j = chain_off[r]; j < chain_off[r + 1]; ++j) K[chosen].insert(chains[j]);
+    }
+  }
+  for (uint64_t d = 0; d < D; ++d) load_out[d] = load[d];
 }
 
 }  // extern "C"

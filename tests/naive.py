@@ -279,3 +279,47 @@ def greedy_exact_load(tree, role, bw, lat, util, length, prefill, snap, M, event
             n[d] += 1
             m[d] -= (l - 16 * int(M[r][d])) * bpt
     return dec, best, n, m
+
+
+def greedy_exact_evolving(tree, role, bw, lat, util, length, prefill, snap, keys_per_decode,
+                          chains, events, w, theta, cap, bpt):
+    """Exact-rational Algorithm 1 with evolving caches: hits per arrival against the caches
+    of that moment (a list scan to the first miss), and a dispatch adds the request's whole
+    chain to its decode's cache.  Returns (dec, best, load, M)."""
+    pre = [i for i in range(tree.n) if role[i] == 0]
+    dec_inst = [i for i in range(tree.n) if role[i] == 1]
+    D = len(dec_inst)
+    caches = [set(int(k) for k in keys_per_decode[d]) for d in range(D)]
+    load = [0] * D
+    R = len(length)
+    dec, best = [-1] * R, [None] * R
+    M = [[0] * D for _ in range(R)]
+    wn, wp, wl = (frac(x) for x in w)
+    th = frac(theta)
+    for code in events:
+        code = int(code)
+        r = code & 0x7FFFFFFF
+        l = int(length[r])
+        if code >> 31:
+            if dec[r] >= 0:
+                load[dec[r]] -= l
+            continue
+        chain = [int(x) for x in chains[r]]
+        for d in range(D):
+            M[r][d] = lcp_blocks(chain, caches[d])
+        p = pre[int(prefill[r])]
+        u_row = util[int(snap[r])]
+        cands = []
+        for d in range(D):
+            if load[d] + l > cap:
+                continue
+            miss_tok = l - 16 * M[r][d]
+            T = Fraction(miss_tok * bpt) / bottleneck(tree, bw, u_row, p, dec_inst[d]) \
+                + frac(lat[tree.tier(p, dec_inst[d])])
+            cands.append((wn * T + wp * Fraction(miss_tok, l) + wl * th * load[d], d))
+        if cands:
+            s, d = min(cands)
+            dec[r], best[r] = d, s
+            load[d] += l
+            caches[d].update(chain)
+    return dec, best, load, M

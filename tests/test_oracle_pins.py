@@ -896,3 +896,101 @@ def test_load_model_memory_filter():
     pb["events"] = np.array([0, 1, 0 | (1 << 31), 2], np.uint32)
     res = _run_load(pb, (1.0, 1.0, 1.0), beta_max=64, m0=2 * per + 5, m_min=5)
     assert list(res.dec) == [0, 0, 0] and list(res.n) == [2] and list(res.m) == [5]
+
+
+# ------------------------------------------ evolving caches (NEXT: cache update on dispatch)
+def _evolving_problem(seed, R=10, span=1000):
+    """A tiny tree (P = D = 4) whose requests share three roots (random depths, tails of
+    their own) and whose caches hold root prefixes with holes."""
+    pb = _tiny_problem(seed, R=R, span=span)
+    rng = np.random.default_rng(2000 + seed)
+    roots = [rng.integers(1, 2 ** 63, 80, dtype=np.int64).astype(np.uint64) for _ in range(3)]
+    chains = []
+    for r in range(R):
+        n = int(pb["length"][r]) // 16
+        k = int(rng.integers(0, min(n, 80) + 1))
+        c = np.concatenate([roots[int(rng.integers(0, 3))][:k],
+                            rng.integers(1, 2 ** 63, n - k, dtype=np.int64).astype(np.uint64)])
+        if r >= 2 and rng.random() < 0.3:              # a repeat of an earlier prefix
+            prev = chains[int(rng.integers(0, r))]
+            c = np.concatenate([prev[:min(len(prev), n)],
+                                rng.integers(1, 2 ** 63, max(0, n - len(prev)), dtype=np.int64).astype(np.uint64)])
+        chains.append(c.astype(np.uint64))
+    D = int(pb["role"].sum())
+    keys = []
+    for d in range(D):
+        ks = []
+        for root in roots:
+            depth = int(rng.integers(0, 81))
+            keep = list(root[:depth])
+            if depth > 5 and rng.random() < 0.3:
+                keep.pop(int(rng.integers(0, depth)))
+            ks += keep
+        keys.append(np.array(ks, np.uint64))
+    pb["chains"], pb["keys"] = chains, keys
+    return pb
+
+
+def _run_evolving(pb, w, theta=float(np.float32(1e-6)), bpt=81920, cap=None):
+    keys = np.concatenate(pb["keys"])
+    key_off = np.concatenate([[0], np.cumsum([len(k) for k in pb["keys"]])]).astype(np.uint64)
+    chains = np.concatenate(pb["chains"])
+    chain_off = np.concatenate([[0], np.cumsum([len(c) for c in pb["chains"]])]).astype(np.uint64)
+    return oracle.schedule_stream_evolving(pb["fanout"], pb["role"], pb["bw"], pb["lat"], pb["u"],
+                                           pb["length"], pb["prefill"], pb["snap"], keys, key_off,
+                                           chains, chain_off, pb["events"], w[0], w[1], w[2],
+                                           theta, pb["cap"] if cap is None else cap, bpt)
+
+
+def test_evolving_matches_exact_rational_bruteforce():
+    theta = float(np.float32(1e-6))
+    grew = 0
+    for seed in range(30):
+        pb = _evolving_problem(seed)
+        w = tuple(float(np.float32(x)) for x in np.random.default_rng(1400 + seed).uniform(0, 2, 3))
+        res = _run_evolving(pb, w)
+        dec, best, load, M = naive.greedy_exact_evolving(
+            pb["tree"], pb["role"], pb["bw"], pb["lat"], pb["u"], pb["length"], pb["prefill"],
+            pb["snap"], pb["keys"], pb["chains"], pb["events"], w, theta, pb["cap"], 81920)
+        assert list(res.dec) == dec and list(res.load) == load
+        np.testing.assert_array_equal(res.M, np.array(M, np.uint16))
+        for r in range(len(dec)):
+            if dec[r] >= 0:
+                assert res.best[r] == pytest.approx(float(best[r]), rel=1e-14)
+        # the static match of the same caches: evolving hits are never below it
+        keys = np.concatenate(pb["keys"])
+        key_off = np.concatenate([[0], np.cumsum([len(k) for k in pb["keys"]])]).astype(np.uint64)
+        chains = np.concatenate(pb["chains"])
+        chain_off = np.concatenate([[0], np.cumsum([len(c) for c in pb["chains"]])]).astype(np.uint64)
+        static = oracle.prefix_match(keys, key_off, len(pb["keys"]), chains, chain_off,
+                                     np.array([0, len(pb["chains"])], np.uint32))
+        assert (res.M >= static).all()
+        grew += int((res.M > static).sum())
+    assert grew > 10
+
+
+def test_evolving_without_dispatches_is_the_static_match():
+    """Nothing fits (cap 0): no cache grows, every arrival sees the static hits."""
+    pb = _evolving_problem(3)
+    res = _run_evolving(pb, (1.0, 1.0, 1.0), cap=0)
+    assert (res.dec == -1).all()
+    keys = np.concatenate(pb["keys"])
+    key_off = np.concatenate([[0], np.cumsum([len(k) for k in pb["keys"]])]).astype(np.uint64)
+    chains = np.concatenate(pb["chains"])
+    chain_off = np.concatenate([[0], np.cumsum([len(c) for c in pb["chains"]])]).astype(np.uint64)
+    np.testing.assert_array_equal(res.M, oracle.prefix_match(keys, key_off, 4, chains, chain_off,
+                                                             np.array([0, len(pb["chains"])], np.uint32)))
+
+
+def test_evolving_dispatch_warms_its_decode():
+    """Request 1 repeats request 0's chain: after request 0 goes to some decode, that
+    decode holds the whole chain and request 1 hits all of it there, and only there."""
+    pb = _evolving_problem(5, R=2)
+    pb["chains"][1] = pb["chains"][0].copy()
+    pb["length"][1] = pb["length"][0]
+    pb["events"] = np.array([0, 1, 1 << 31, 1 | (1 << 31)], np.uint32)
+    res = _run_evolving(pb, (1.0, 1.0, 0.0), cap=10 ** 9)
+    d0 = int(res.dec[0])
+    n = len(pb["chains"][0])
+    assert d0 >= 0 and res.M[1, d0] == n
+    assert all(res.M[1, d] == res.M[0, d] for d in range(4) if d != d0)
