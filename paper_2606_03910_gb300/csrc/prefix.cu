@@ -40,34 +40,12 @@
 //     warp per member: the common prefix is read once, the member's row is
 //     min(M_L, lcp) elementwise, and block lcp is probed only in the groups where a
 //     leader hit reaches lcp, up to 32 groups at a time.
-#include "netkv_internal.cuh"
+#include "cache_index.cuh"
 
 namespace {
 
 constexpr int kBuildBlock = 1024;
 constexpr int kMatchBlock = 256;
-constexpr uint32_t kGroup = 64;  // decodes per index (bits of the mask)
-constexpr unsigned long long kNotFound = ~0ull;
-
-struct __align__(16) IndexSlot {
-  unsigned long long key;
-  unsigned long long pos;  // position of the key in the run array
-};
-
-struct __align__(16) RunEntry {
-  unsigned long long key;
-  unsigned long long mask;  // decodes of the group that cache the key
-};
-
-// Hash table and run array of index (set g, decode group q): 2^L slots then 2^L entries.
-__device__ __forceinline__ IndexSlot* index_hash(void* index, uint64_t idx, uint32_t L) {
-  return reinterpret_cast<IndexSlot*>(index) + (idx << (L + 1));
-}
-__device__ __forceinline__ const IndexSlot* index_hash(const void* index, uint64_t idx,
-                                                       uint32_t L) {
-  return reinterpret_cast<const IndexSlot*>(index) + (idx << (L + 1));
-}
-
 // Exclusive scan of one flag per thread over a 1024-thread block; returns the prefix and
 // writes the block total to *total (shared).
 __device__ __forceinline__ uint32_t block_scan(uint32_t flag, uint32_t* warp_sums,
@@ -150,22 +128,6 @@ __global__ void __launch_bounds__(kBuildBlock) cache_build_kernel(
       }
     }
   }
-}
-
-// Run position of `key` (non-zero) in one index, or kNotFound.
-__device__ __forceinline__ unsigned long long lookup(const IndexSlot* __restrict__ hash,
-                                                     uint64_t key, uint32_t log2_cap,
-                                                     int* status) {
-  const uint64_t mask = (1ull << log2_cap) - 1;
-  uint64_t slot = home_slot(key, log2_cap);
-  for (uint64_t seen = 0; seen <= mask; ++seen) {
-    const ulonglong2 s = __ldg(reinterpret_cast<const ulonglong2*>(hash + slot));
-    if (s.x == key) return s.y;
-    if (s.x == 0ull) return kNotFound;
-    slot = (slot + 1) & mask;
-  }
-  flag_status(status, NETKV_DEV_EFULL);
-  return kNotFound;
 }
 
 __device__ __forceinline__ int32_t find_set(const uint32_t* __restrict__ set_off, uint32_t n_sets,
