@@ -12,7 +12,8 @@
  *                           snapshots, and the per-instance level bottlenecks UB
  *                           (netkv_oracle_build_directed: per link and direction;
  *                           netkv_oracle_build_tiers: the paper's per-tier maps)
- *   netkv_cache_build       decode caches K_d as open-addressing hash tables
+ *   netkv_cache_build       decode caches K_d as an inverted index (block hash -> the
+ *                           decodes of a 64-decode group that cache it)
  *   netkv_prefix_match      block-level prefix hit M[r][d] (Sec. III-B)
  *   netkv_schedule_streams  the greedy of Algorithm 1 over independent streams
  *   netkv_schedule_streams_inflight  the same with self-contention (Eq. 4's n_inflight)
@@ -215,8 +216,10 @@ netkv_status netkv_prefix_match(const void* d_index, uint32_t D, uint32_t log2_c
  * until the process exits).
  *   - Arguments are those of netkv_prefix_match without the workspace.
  *   - R above NETKV_PREFIX_MATCH_STATIC_MAX_R returns NETKV_ELIMIT and enqueues nothing.
- *   - The first call on a device looks up the array's device address with that device
- *     current; make that first call before any stream capture.
+ *   - Every call made outside a stream capture looks up the array's device address
+ *     with the device current (so a device reset, which may move the array, is
+ *     followed); a call inside a capture uses the last address looked up on that
+ *     device.  Make the first call on a device before any stream capture.
  *   - Allocates nothing: no cudaMalloc, no cudaFree, no allocating library routine.
  *     The array is cleared where it must start at zero on every call.
  *   - All calls on a device share the one array: calls that overlap on the GPU (on
@@ -291,7 +294,7 @@ netkv_status netkv_schedule_streams(netkv_topology_t topo, uint32_t n_streams,
                                     size_t workspace_bytes, int* d_status, netkv_stream_t stream);
 
 /* Algorithm 1 with self-contention (Eq. 4's n_inflight term, Algorithm 1 lines 5 and 14,
- * Sec. IV-C).  As netkv_schedule_streams without a workspace, and in addition each
+ * Sec. V-C).  As netkv_schedule_streams without a workspace, and in addition each
  * stream keeps a counter n[p][tau] per prefill rank and tier (zero at the start of the
  * call) of its own transfers in flight:
  *     B_eff  = min(UB[k_r][p][tau], UB[k_r][d][tau]) / (1 + n[p_r][tau])  (Eq. 4)

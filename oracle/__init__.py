@@ -45,6 +45,8 @@ U32, U64, I64, F64, INT = C.c_uint32, C.c_uint64, C.c_int64, C.c_double, C.c_int
 
 
 def _declare(l):
+    l.oracle_set_threads.restype = None
+    l.oracle_set_threads.argtypes = [INT]
     l.oracle_kv_bytes_per_token.restype = F64
     l.oracle_kv_bytes_per_token.argtypes = [U32, U32, U32, U32]
     l.oracle_beff_tier.restype = F64
@@ -98,6 +100,11 @@ def _p(a: Optional[np.ndarray]):
 
 def _c(a, dt):
     return np.ascontiguousarray(np.asarray(a, dtype=dt))
+
+
+def set_threads(n: int) -> None:
+    """OpenMP threads of the calling thread's later oracle calls (timing only)."""
+    lib().oracle_set_threads(int(n))
 
 
 # ------------------------------------------------------------------ closed forms
@@ -275,7 +282,7 @@ def schedule_stream_inflight(fanout, role, bw, lat, util, length, prefill, snap,
                              inflight_cap, load_init=None, hint=None, xfer_hint=None,
                              rel_tol=1e-5) -> StreamResult:
     """Algorithm 1 with self-contention (Eq. 4's n_inflight, Algorithm 1 lines 5 and 14,
-    Sec. IV-C): arrays are indexed by request; arrival_us are the arrival times in
+    Sec. V-C): arrays are indexed by request; arrival_us are the arrival times in
     microseconds; inflight_cap = 0 turns self-contention off.  xfer_hint: another
     implementation's transfer times (whole microseconds) to adopt where they differ by at
     most one.  Returns a StreamResult with xfer_us set."""

@@ -25,16 +25,16 @@
 //   * Block-level prefix hit (Sec. III-B): lambda = 16 * |LCP_block(h_r, K_d)|, the number
 //     of leading blocks of the request's hash chain that are all in decode d's cache.
 //   * Effective transfer size, Eq. 2: s_eff = s * (1 - lambda / l).
-//   * Algorithm 1 (Sec. IV-A) as a weighted score: filter by capacity (line 1), reject
+//   * Algorithm 1 (Sec. V-A) as a weighted score: filter by capacity (line 1), reject
 //     when nothing is feasible (line 2), score every candidate (lines 3-11), take the
 //     argmin with the lowest index among equal scores (line 13), then update load.
-//   * Evolving caches (the simulator's cache update, Sec. V-B, without LRU eviction), in
+//   * Evolving caches (the simulator's cache update, Sec. VI-B, without LRU eviction), in
 //     oracle_schedule_stream_evolving: a dispatch adds the request's blocks to its
 //     decode's cache and later arrivals match against the grown caches.
 //   * The compute-load model (Sec. III-C, IV-B, the feasible set of Sec. IV-A), in
 //     oracle_schedule_stream_load: T_queue + T_decode from each decode's request count
 //     and t_iter(beta) = a + b beta, memory feasibility m_d >= s_eff + m_min.
-//   * Self-contention (Eq. 4's n_inflight, Algorithm 1 lines 5 and 14, Sec. IV-C), in
+//   * Self-contention (Eq. 4's n_inflight, Algorithm 1 lines 5 and 14, Sec. V-C), in
 //     oracle_schedule_stream_inflight: a per-(prefill, tier) counter divides the
 //     effective bandwidth by 1 + n; a dispatch raises the counter of its tier (saturating
 //     at the cap) and its transfer completes, lowering it again (never below zero), at
@@ -44,6 +44,8 @@
 // Parity: pinned by the not-gpu tests (worked example of Sec. III-D, closed forms of
 // Eq. 1, the per-tier special case of Eq. 4, brute force on tiny instances,
 // Propositions 1 and 2, first-miss LCP semantics).
+#include <omp.h>
+
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -137,6 +139,10 @@ void ranks(const uint8_t* role, uint64_t n, std::vector<uint64_t>& pre, std::vec
 }  // namespace
 
 extern "C" {
+
+// OpenMP threads of the calling thread's later parallel regions (timing only: results do
+// not depend on it).
+void oracle_set_threads(int n) { omp_set_num_threads(n > 0 ? n : 1); }
 
 // ---------------------------------------------------------------- closed forms
 // Eq. 1: bytes of KV cache per token, s_r / l_r.
@@ -626,7 +632,7 @@ void oracle_schedule_stream_load(
   }
 }
 
-// Algorithm 1 with evolving caches (the simulator's cache update of Sec. V-B, without its
+// Algorithm 1 with evolving caches (the simulator's cache update of Sec. VI-B, without its
 // LRU eviction): a stream starts from its decodes' cache contents (key lists keys,
 // key_off [D+1]); every arrival's prefix hits are taken against the caches as they are
 // at that arrival (first-miss scan, Sec. III-B), and a dispatch to d* adds every block of

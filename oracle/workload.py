@@ -3,9 +3,12 @@
 TEST INFRASTRUCTURE ONLY (tests, smoke check, benchmark CPU baseline).
 
 A stream is made self-contained: its requests are renumbered from 0, its events
-re-encoded, its telemetry rows gathered; the oracle then computes the level
-bottlenecks, the prefix hits (by set membership over the generator's key
-lists) and the greedy, all in double precision.
+re-encoded, its telemetry rows gathered.  ``stream_inputs`` does that gathering (the
+generator's output, no arithmetic of the method); the oracle then computes the prefix
+hits (by set membership over the generator's key lists), the greedy and, for the
+tests, the level bottlenecks, all in double precision.  The benchmark times the
+oracle alone by preparing the inputs first (``stream_inputs``) and timing
+``solve_stream``.
 """
 from __future__ import annotations
 
@@ -34,6 +37,24 @@ class OracleStream:
     UB: np.ndarray         # [len(snaps), N, 4] oracle level bottlenecks of those snapshots
 
 
+@dataclasses.dataclass
+class StreamInputs:
+    """One stream's inputs, gathered from the generator (requests renumbered from 0)."""
+    s: int
+    r0: int
+    r1: int
+    ev_local: np.ndarray           # u32 events with local request indices
+    snaps: np.ndarray              # global snapshot indices used by the stream's arrivals
+    snap_local: np.ndarray         # u32 [R_s] index into util
+    util: np.ndarray               # f32 [len(snaps), L] (or [len(snaps), 4] per tier)
+    util_down: Optional[np.ndarray]
+    keys: Optional[np.ndarray]     # the stream's caches: key lists of its table set
+    key_off: Optional[np.ndarray]
+    chains: Optional[np.ndarray]   # the stream's chains, offsets from 0
+    chain_off: Optional[np.ndarray]
+    M: Optional[np.ndarray]        # given prefix hits (then no keys or chains)
+
+
 def stream_problem(w, s: int):
     r0, r1 = int(w.req_off[s]), int(w.req_off[s + 1])
     e0, e1 = int(w.event_off[s]), int(w.event_off[s + 1])
@@ -56,6 +77,59 @@ def _rows(w, snaps, direction):
     return np.stack([w.util(int(k), int(k) + 1, direction)[0] for k in snaps])
 
 
+def stream_inputs(w, s: int, M: Optional[np.ndarray] = None, directed: bool = False,
+                  tiers: bool = False) -> StreamInputs:
+    """Gather stream s's inputs from the generator: events, telemetry rows, and either the
+    given prefix hits M or the key lists and chains the oracle matches itself."""
+    from synth import request_set, utilisation
+    r0, r1, ev_local, snaps, snap_local = stream_problem(w, s)
+    util = utilisation(w, snaps, "tiers") if tiers else _rows(w, snaps, "up")
+    util_down = _rows(w, snaps, "down") if directed else None
+    keys = key_off = chains = chain_off = None
+    if M is None:
+        g = int(request_set(w)[r0]) if r1 > r0 else 0
+        keys, key_off = stream_cache_keys(w, g)
+        chains = w.chains(r0, r1)
+        chain_off = (w.chain_off[r0:r1 + 1] - w.chain_off[r0]).astype(np.uint64)
+    return StreamInputs(s, r0, r1, ev_local, snaps, snap_local, util, util_down, keys, key_off,
+                        chains, chain_off, M)
+
+
+def stream_hits(w, x: StreamInputs) -> np.ndarray:
+    """The oracle's prefix hits of the stream (or the given ones)."""
+    if x.M is not None:
+        return x.M
+    return prefix_match(x.keys, x.key_off, w.D, x.chains, x.chain_off,
+                        np.array([0, x.r1 - x.r0], np.uint32))
+
+
+def solve_stream(w, x: StreamInputs, theta: float, cap: int, bytes_per_token: int,
+                 inflight_cap: int = 0, load_model=None, tiers: bool = False):
+    """The oracle's work for one prepared stream: its prefix match and its greedy (with
+    self-contention when inflight_cap > 0, with the compute-load model when load_model =
+    (t_a, t_b, beta_max, m_min, m0) is given).  Returns (M, greedy result)."""
+    M = stream_hits(w, x)
+    wn, wp, wl = (float(v) for v in w.weights[x.s])
+    spec = w.spec
+    r0, r1 = x.r0, x.r1
+    if load_model is not None:
+        a, b, bmax, m_min, m0 = load_model
+        res = schedule_stream_load(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, x.util,
+                                   w.length[r0:r1], w.prefill[r0:r1], x.snap_local, M, x.ev_local,
+                                   wn, wp, wl, bytes_per_token, a, b, bmax, m_min, m0)
+    elif inflight_cap > 0:
+        res = schedule_stream_inflight(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, x.util,
+                                       w.length[r0:r1], w.prefill[r0:r1], x.snap_local,
+                                       w.arrival_us[r0:r1], M, x.ev_local, wn, wp, wl, theta, cap,
+                                       bytes_per_token, inflight_cap)
+    else:
+        res = schedule_stream(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, x.util,
+                              w.length[r0:r1], w.prefill[r0:r1], x.snap_local, M, x.ev_local,
+                              wn, wp, wl, theta, cap, bytes_per_token, util_down=x.util_down,
+                              tier_mode=tiers)
+    return M, res
+
+
 def run_stream(w, s: int, theta: float, cap: int, bytes_per_token: int,
                hint: Optional[np.ndarray] = None, rel_tol: float = 1e-5,
                M: Optional[np.ndarray] = None, directed: bool = False,
@@ -68,32 +142,24 @@ def run_stream(w, s: int, theta: float, cap: int, bytes_per_token: int,
     tiers: the paper's per-tier maps (the generator's "tiers" rows, four congestion
     values per snapshot); UB[s][i][k] is then B_k (1 - c[s][k]) for every instance.
     """
-    from synth import request_set, utilisation
-    r0, r1, ev_local, snaps, snap_local = stream_problem(w, s)
-    util = utilisation(w, snaps, "tiers") if tiers else _rows(w, snaps, "up")
-    util_down = _rows(w, snaps, "down") if directed else None
-    if M is None:
-        g = int(request_set(w)[r0]) if r1 > r0 else 0
-        keys, key_off = stream_cache_keys(w, g)
-        chains = w.chains(r0, r1)
-        chain_off = (w.chain_off[r0:r1 + 1] - w.chain_off[r0]).astype(np.uint64)
-        M = prefix_match(keys, key_off, w.D, chains, chain_off,
-                         np.array([0, r1 - r0], np.uint32))
-    wn, wp, wl = (float(x) for x in w.weights[s])
+    x = stream_inputs(w, s, M=M, directed=directed, tiers=tiers)
+    M = stream_hits(w, x)
+    r0, r1 = x.r0, x.r1
+    wn, wp, wl = (float(v) for v in w.weights[s])
     spec = w.spec
-    res = schedule_stream(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, util,
-                          w.length[r0:r1], w.prefill[r0:r1], snap_local, M, ev_local,
+    res = schedule_stream(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, x.util,
+                          w.length[r0:r1], w.prefill[r0:r1], x.snap_local, M, x.ev_local,
                           wn, wp, wl, theta, cap, bytes_per_token, hint=hint, rel_tol=rel_tol,
-                          util_down=util_down, tier_mode=tiers)
+                          util_down=x.util_down, tier_mode=tiers)
     if tiers:
-        per_tier = np.asarray(spec.tier_bw, np.float64) * (1.0 - util.astype(np.float64))
+        per_tier = np.asarray(spec.tier_bw, np.float64) * (1.0 - x.util.astype(np.float64))
         UB = np.repeat(per_tier[:, None, :], len(w.role), axis=1)
     elif directed:
-        UB = level_bottleneck_directed(spec.fanout, w.role, spec.tier_bw, util, util_down)
+        UB = level_bottleneck_directed(spec.fanout, w.role, spec.tier_bw, x.util, x.util_down)
     else:
-        UB = up_bottleneck(spec.fanout, spec.tier_bw, util)
+        UB = up_bottleneck(spec.fanout, spec.tier_bw, x.util)
     return OracleStream(r0, r1, M, res.dec, res.best, res.second, res.load, res.near_ties,
-                        res.mismatches, res.rejects, snaps, UB)
+                        res.mismatches, res.rejects, x.snaps, UB)
 
 
 def run_stream_inflight(w, s: int, theta: float, cap: int, bytes_per_token: int,
@@ -103,26 +169,19 @@ def run_stream_inflight(w, s: int, theta: float, cap: int, bytes_per_token: int,
     """Oracle for stream s with self-contention (Eq. 4's n_inflight, Algorithm 1 lines 5
     and 14).  hint / xfer_hint: another implementation's decisions and transfer times
     for the stream's requests (local order).  The result carries xfer_us."""
-    from synth import request_set, utilisation
-    r0, r1, ev_local, snaps, snap_local = stream_problem(w, s)
-    util = _rows(w, snaps, "up")
-    if M is None:
-        g = int(request_set(w)[r0]) if r1 > r0 else 0
-        keys, key_off = stream_cache_keys(w, g)
-        chains = w.chains(r0, r1)
-        chain_off = (w.chain_off[r0:r1 + 1] - w.chain_off[r0]).astype(np.uint64)
-        M = prefix_match(keys, key_off, w.D, chains, chain_off,
-                         np.array([0, r1 - r0], np.uint32))
-    wn, wp, wl = (float(x) for x in w.weights[s])
+    x = stream_inputs(w, s, M=M)
+    M = stream_hits(w, x)
+    r0, r1 = x.r0, x.r1
+    wn, wp, wl = (float(v) for v in w.weights[s])
     spec = w.spec
-    res = schedule_stream_inflight(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, util,
-                                   w.length[r0:r1], w.prefill[r0:r1], snap_local,
-                                   w.arrival_us[r0:r1], M, ev_local, wn, wp, wl, theta, cap,
+    res = schedule_stream_inflight(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, x.util,
+                                   w.length[r0:r1], w.prefill[r0:r1], x.snap_local,
+                                   w.arrival_us[r0:r1], M, x.ev_local, wn, wp, wl, theta, cap,
                                    bytes_per_token, inflight_cap, hint=hint, xfer_hint=xfer_hint,
                                    rel_tol=rel_tol)
-    UB = up_bottleneck(spec.fanout, spec.tier_bw, util)
+    UB = up_bottleneck(spec.fanout, spec.tier_bw, x.util)
     out = OracleStream(r0, r1, M, res.dec, res.best, res.second, res.load, res.near_ties,
-                       res.mismatches, res.rejects, snaps, UB)
+                       res.mismatches, res.rejects, x.snaps, UB)
     out.xfer_us, out.xfer_adopted, out.xfer_mismatches = res.xfer_us, res.xfer_adopted, res.xfer_mismatches
     return out
 
@@ -133,21 +192,14 @@ def run_stream_load(w, s: int, t_a: float, t_b: float, beta_max: int, m_min: int
     """Oracle for stream s with the paper's compute-load model (Sec. III-C, IV-B); hint: another
     implementation's decisions for the stream's requests (local order).  Returns the
     oracle's LoadResult with its prefix hits attached (.M)."""
-    from synth import request_set
-    r0, r1, ev_local, snaps, snap_local = stream_problem(w, s)
-    util = _rows(w, snaps, "up")
-    if M is None:
-        g = int(request_set(w)[r0]) if r1 > r0 else 0
-        keys, key_off = stream_cache_keys(w, g)
-        chains = w.chains(r0, r1)
-        chain_off = (w.chain_off[r0:r1 + 1] - w.chain_off[r0]).astype(np.uint64)
-        M = prefix_match(keys, key_off, w.D, chains, chain_off,
-                         np.array([0, r1 - r0], np.uint32))
-    wn, wp, wl = (float(x) for x in w.weights[s])
+    x = stream_inputs(w, s, M=M)
+    M = stream_hits(w, x)
+    r0, r1 = x.r0, x.r1
+    wn, wp, wl = (float(v) for v in w.weights[s])
     spec = w.spec
-    res = schedule_stream_load(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, util,
-                               w.length[r0:r1], w.prefill[r0:r1], snap_local, M, ev_local, wn, wp,
-                               wl, bytes_per_token, t_a, t_b, beta_max, m_min, m0, hint=hint,
+    res = schedule_stream_load(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, x.util,
+                               w.length[r0:r1], w.prefill[r0:r1], x.snap_local, M, x.ev_local, wn,
+                               wp, wl, bytes_per_token, t_a, t_b, beta_max, m_min, m0, hint=hint,
                                rel_tol=rel_tol)
     res.M = M
     return res

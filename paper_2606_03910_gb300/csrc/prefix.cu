@@ -727,7 +727,10 @@ extern "C" netkv_status netkv_prefix_match(const void* d_index, uint32_t D,
 // ---------------------------------------------------------------------------------
 // netkv_prefix_match_static: the prefix match for callers that cannot allocate device
 // memory (see include/netkv.h).  Its workspace is this fixed device array, shared by
-// every call on a device; the device address is looked up once per device.
+// every call on a device.  Host code cannot use the array's name as a device address, so
+// the address is looked up with the device current: on every call made outside a stream
+// capture (a device reset reloads the module and may move the array), and from the
+// last lookup on that device during a capture.
 // ---------------------------------------------------------------------------------
 #include <mutex>
 
@@ -740,12 +743,17 @@ constexpr int kMaxDevices = 64;
 std::mutex g_scratch_mutex;
 void* g_scratch_addr[kMaxDevices] = {};
 
-// Device address of g_prefix_scratch on the current device (looked up on first use).
-netkv_status static_scratch(void** out) {
+// Device address of g_prefix_scratch on the current device.
+netkv_status static_scratch(cudaStream_t stream, void** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return NETKV_ECUDA;
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(stream, &cap) != cudaSuccess) {
+    cudaGetLastError();
+    return NETKV_ECUDA;
+  }
   std::lock_guard<std::mutex> lock(g_scratch_mutex);
-  if (!g_scratch_addr[dev]) {
+  if (cap == cudaStreamCaptureStatusNone || !g_scratch_addr[dev]) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_prefix_scratch) != cudaSuccess || !p) {
       cudaGetLastError();
@@ -771,7 +779,7 @@ extern "C" netkv_status netkv_prefix_match_static(const void* d_index, uint32_t 
       netkv_prefix_match_workspace_size(R) > kStaticScratchBytes)
     return NETKV_ELIMIT;
   void* scratch = nullptr;
-  const netkv_status st = static_scratch(&scratch);
+  const netkv_status st = static_scratch((cudaStream_t)stream, &scratch);
   if (st != NETKV_OK) return st;
   return netkv_prefix_match(d_index, D, log2_capacity, n_sets, d_chains, d_chain_off, R,
                             d_set_off, scratch, kStaticScratchBytes, d_M, d_status, stream);

@@ -73,7 +73,7 @@ struct LoadModel {
   int64_t m_min, m0;
 };
 
-// Self-contention (Eq. 4's n_inflight, Algorithm 1 lines 5 and 14, Sec. IV-C): the
+// Self-contention (Eq. 4's n_inflight, Algorithm 1 lines 5 and 14, Sec. V-C): the
 // candidate's bandwidth is divided by 1 + n; T is returned for the completion time.
 __device__ __forceinline__ float contended_score(const netkv_weights& w, uint32_t l, uint32_t m,
                                                  float ub_p, float ub_d, float lat_tau,
@@ -1053,14 +1053,10 @@ netkv_status launch_staged(const TopoArgs& t, uint32_t n_streams, const netkv_we
                            int64_t* d_load_final, const float* d_base, int* d_status,
                            cudaStream_t s) {
   const size_t smem = sizeof(float) * (size_t)kStages * BLOCK * NPT;
-  if (smem > 48u * 1024u) {
-    static bool raised = false;  // the same value every time: a benign race
-    if (!raised) {
-      NETKV_CUDA_TRY(cudaFuncSetAttribute(schedule_staged_kernel<NPT, BLOCK, kStages>,
-                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-      raised = true;
-    }
-  }
+  // the attribute is per device: set it before every launch that needs it (cheap)
+  if (smem > 48u * 1024u)
+    NETKV_CUDA_TRY(cudaFuncSetAttribute(schedule_staged_kernel<NPT, BLOCK, kStages>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   schedule_staged_kernel<NPT, BLOCK, kStages><<<n_streams, BLOCK, smem, s>>>(
       t, n_streams, d_w, R, d_base, d_len, d_prefill, d_snap, n_snap, d_events, d_event_off,
       d_load_init, d_dec, d_best, d_second, d_load_final, d_status);
@@ -1175,15 +1171,10 @@ netkv_status launch_inflight(const TopoArgs& t, uint32_t n_streams, const netkv_
     if (launch_base(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events,
                     d_event_off, d_base, d_X, d_status, s) != NETKV_OK)
       return NETKV_ECUDA;
-    if (smem > 48u * 1024u) {
-      static bool raised = false;  // the same value every time: a benign race
-      if (!raised) {
-        NETKV_CUDA_TRY(cudaFuncSetAttribute(schedule_kernel<NPT, BLOCK, LPS, true, true>,
-                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                            (int)kInflightSmemMax));
-        raised = true;
-      }
-    }
+    if (smem > 48u * 1024u)  // per device: set before every launch that needs it
+      NETKV_CUDA_TRY(cudaFuncSetAttribute(schedule_kernel<NPT, BLOCK, LPS, true, true>,
+                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                          (int)kInflightSmemMax));
     schedule_kernel<NPT, BLOCK, LPS, true, true><<<grid, BLOCK, smem, s>>>(
         t, n_streams, d_w, R, d_base, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events,
         d_event_off, d_load_init, d_dec, d_best, d_second, d_load_final, d_status, d_arrival_us,
@@ -1191,15 +1182,10 @@ netkv_status launch_inflight(const TopoArgs& t, uint32_t n_streams, const netkv_
         nullptr, d_X);
     return netkv_launch_status();
   }
-  if (smem > 48u * 1024u) {
-    static bool raised = false;  // the same value every time: a benign race
-    if (!raised) {
-      NETKV_CUDA_TRY(cudaFuncSetAttribute(schedule_kernel<NPT, BLOCK, LPS, false, true>,
-                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                          (int)kInflightSmemMax));
-      raised = true;
-    }
-  }
+  if (smem > 48u * 1024u)  // per device: set before every launch that needs it
+    NETKV_CUDA_TRY(cudaFuncSetAttribute(schedule_kernel<NPT, BLOCK, LPS, false, true>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        (int)kInflightSmemMax));
   schedule_kernel<NPT, BLOCK, LPS, false, true><<<grid, BLOCK, smem, s>>>(
       t, n_streams, d_w, R, nullptr, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events,
       d_event_off, d_load_init, d_dec, d_best, d_second, d_load_final, d_status, d_arrival_us,

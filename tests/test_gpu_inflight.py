@@ -1,5 +1,5 @@
 """GPU parity of the greedy with self-contention (netkv_schedule_streams_inflight;
-Eq. 4's n_inflight, Algorithm 1 lines 5 and 14, Sec. IV-C) against the oracle.
+Eq. 4's n_inflight, Algorithm 1 lines 5 and 14, Sec. V-C) against the oracle.
 
 * cap 0 is the plain greedy: bit for bit the no-workspace netkv_schedule_streams.
 * The worked example of Sec. III-D end to end: one transfer in flight on tier 2 makes
