@@ -68,9 +68,9 @@ def parse():
                     help="self-contention counter cap (Eq. 4's n_inflight; the paper uses 16); "
                          "0 = the plain greedy")
     ap.add_argument("--streams", type=int, default=4096)
-    ap.add_argument("--cpu-streams", type=int, default=32,
+    ap.add_argument("--cpu-streams", type=int, default=256,
                     help="streams of the multi-core CPU-oracle sample (one per core at a time)")
-    ap.add_argument("--cpu-streams-1t", type=int, default=4,
+    ap.add_argument("--cpu-streams-1t", type=int, default=12,
                     help="streams of the one-thread CPU-oracle sample")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
@@ -215,6 +215,10 @@ KERNEL_CODE = {
 #   prefix_match: bytes per request, from the 64-replica case of the bench workload
 #   oracle_build: bytes per snapshot of the oracle-build sweep
 MEASURED_TRAFFIC = {
+    # 64 replicas (64,000 requests): group_insert 8.97 MB, group_resolve 9.11 MB,
+    # match_leaders 129.29 MB, match_kernel<members> 243.36 MB (read + write)
+    "prefix_match": {"code_sha256_16": "5bb5552e2265ced6", "bytes_per_unit": 390_734_080 / 64_000,
+                     "unit": "request", "captured": "64-replica case, one launch per kernel"},
     "oracle_build": {"code_sha256_16": "ed437e71560780e2", "bytes_per_unit": 67_155_930,
                      "unit": "snapshot", "captured": "1,000-snapshot sweep, one launch"},
 }
@@ -273,7 +277,9 @@ def cpu_oracle_sample(w, streams, theta, cap, bpt, inflight=0, directed=False, t
     import concurrent.futures as cf
     import oracle
     from oracle.workload import solve_stream, stream_inputs
-    xs = [stream_inputs(w, int(s), directed=directed, tiers=tiers) for s in streams]
+    with cf.ThreadPoolExecutor(cpu_cores()) as ex:  # generator output, before the clock
+        xs = list(ex.map(lambda s: stream_inputs(w, int(s), directed=directed, tiers=tiers),
+                         streams))
     lm = None
     if load_model:
         a, b, bmax, _, m_min, m0 = LOAD_MODEL

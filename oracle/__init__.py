@@ -79,9 +79,9 @@ def _declare(l):
                                               F64, U64, F64, F64, I64, I64, I64, P, P, P, F64,
                                               P, P, P, P, P, P]
     l.oracle_schedule_stream_evolving.restype = None
-    l.oracle_schedule_stream_evolving.argtypes = [P, P, P, P, P, U64, P, P, P, P, P, P, P, P, U64,
-                                                  F64, F64, F64, F64, I64, U64, P, F64, P, P, P,
-                                                  P, P, P]
+    l.oracle_schedule_stream_evolving.argtypes = [P, P, P, P, P, U64, P, P, P, P, P, U64, P, P, P,
+                                                  U64, F64, F64, F64, F64, I64, U64, P, F64, P, P,
+                                                  P, P, P, P, P, U64, P]
     l.oracle_cost_matrix_tiers.restype = None
     l.oracle_cost_matrix_tiers.argtypes = [P, P, P, P, P, U64, F64, P]
     l.oracle_cost_matrix_directed.restype = None
@@ -349,19 +349,26 @@ def schedule_stream_load(fanout, role, bw, lat, util, length, prefill, snap, M, 
                       int(counts[2]))
 
 
+UNBOUNDED = (1 << 64) - 1  # cache capacity that never evicts
+
+
 class EvolvingResult(StreamResult):
-    def __init__(self, dec, best, second, load, M, near_ties, mismatches, rejects):
+    def __init__(self, dec, best, second, load, M, near_ties, mismatches, rejects, caches):
         super().__init__(dec, best, second, load, near_ties, mismatches, rejects)
         self.M = M
+        self.caches = caches  # per decode: final cache, most recently used block first
 
 
 def schedule_stream_evolving(fanout, role, bw, lat, util, length, prefill, snap, keys, key_off,
                              chains, chain_off, events, w_net, w_prefix, w_load, theta, cap,
-                             bytes_per_token, hint=None, rel_tol=1e-5) -> EvolvingResult:
-    """Algorithm 1 with evolving caches (the simulator's cache update, without eviction):
-    keys/key_off [D+1] are the decodes' caches at the stream's start; a dispatch adds the
-    request's chain to its decode's cache; M is taken per arrival against the caches of
-    that moment and returned (.M)."""
+                             bytes_per_token, hint=None, rel_tol=1e-5,
+                             cap_blocks=UNBOUNDED) -> EvolvingResult:
+    """Algorithm 1 with evolving caches, the simulator's LRU-managed block caches (Sec. VI-B):
+    keys/key_off [D+1] are the decodes' caches at the stream's start, each list most
+    recently used block first; a dispatch makes the request's chain the most recently used
+    blocks of its decode's cache (block 0 the most recent) and evicts least recently used
+    blocks beyond cap_blocks; M is taken per arrival against the caches of that moment and
+    returned (.M), the final caches as lists (.caches)."""
     f, ro = _c(fanout, np.uint32), _c(role, np.uint8)
     b, la = _c(bw, np.float64), _c(lat, np.float64)
     u = _c(util, np.float32)
@@ -378,9 +385,17 @@ def schedule_stream_evolving(fanout, role, bw, lat, util, length, prefill, snap,
     load = np.zeros(D, np.int64)
     counts = np.zeros(3, np.int64)
     h = None if hint is None else _c(hint, np.int32)
+    # room for the final caches: at most cap_blocks, or every key the stream ever saw
+    stride = int(min(int(cap_blocks), len(k) + len(ch))) if D else 0
+    stride = max(stride, 1)
+    cache_out = np.zeros((D, stride), np.uint64)
+    cache_len = np.zeros(D, np.uint64)
     lib().oracle_schedule_stream_evolving(
         _p(f), _p(ro), _p(b), _p(la), _p(u), u.shape[1], _p(ln), _p(pf), _p(sn), _p(k), _p(ko),
-        _p(ch), _p(co), _p(ev), len(ev), float(w_net), float(w_prefix), float(w_load),
-        float(theta), int(cap), int(bytes_per_token), _p(h), float(rel_tol), _p(dec), _p(best),
-        _p(second), _p(M), _p(load), _p(counts))
-    return EvolvingResult(dec, best, second, load, M, int(counts[0]), int(counts[1]), int(counts[2]))
+        int(cap_blocks), _p(ch), _p(co), _p(ev), len(ev), float(w_net), float(w_prefix),
+        float(w_load), float(theta), int(cap), int(bytes_per_token), _p(h), float(rel_tol),
+        _p(dec), _p(best), _p(second), _p(M), _p(load), _p(counts), _p(cache_out), stride,
+        _p(cache_len))
+    caches = [cache_out[d, :int(cache_len[d])].copy() for d in range(D)]
+    return EvolvingResult(dec, best, second, load, M, int(counts[0]), int(counts[1]),
+                          int(counts[2]), caches)

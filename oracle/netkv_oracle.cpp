@@ -28,9 +28,11 @@
 //   * Algorithm 1 (Sec. V-A) as a weighted score: filter by capacity (line 1), reject
 //     when nothing is feasible (line 2), score every candidate (lines 3-11), take the
 //     argmin with the lowest index among equal scores (line 13), then update load.
-//   * Evolving caches (the simulator's cache update, Sec. VI-B, without LRU eviction), in
-//     oracle_schedule_stream_evolving: a dispatch adds the request's blocks to its
-//     decode's cache and later arrivals match against the grown caches.
+//   * Evolving caches (the simulator's LRU-managed block cache, Sec. VI-B), in
+//     oracle_schedule_stream_evolving: a dispatch makes the request's blocks the most
+//     recently used ones of its decode's cache (block 0 last, so the most recent), the
+//     least recently used blocks beyond the decode's capacity are evicted, and later
+//     arrivals match against the caches of their moment.
 //   * The compute-load model (Sec. III-C, IV-B, the feasible set of Sec. IV-A), in
 //     oracle_schedule_stream_load: T_queue + T_decode from each decode's request count
 //     and t_iter(beta) = a + b beta, memory feasibility m_d >= s_eff + m_min.
@@ -50,7 +52,9 @@
 #include <cstdint>
 #include <cstring>
 #include <limits>
+#include <list>
 #include <queue>
+#include <unordered_map>
 #include <unordered_set>
 #include <vector>
 
@@ -135,6 +139,39 @@ void ranks(const uint8_t* role, uint64_t n, std::vector<uint64_t>& pre, std::vec
   dec.clear();
   for (uint64_t i = 0; i < n; ++i) (role[i] ? dec : pre).push_back(i);
 }
+
+// One decode's block cache as the simulator keeps it (Sec. VI-B: an LRU-managed KV-block
+// cache): block hashes in recency order, most recent first, at most `cap` of them.
+struct LruCache {
+  std::list<uint64_t> order;  // most recent first
+  std::unordered_map<uint64_t, std::list<uint64_t>::iterator> where;
+  uint64_t cap = 0;
+
+  bool contains(uint64_t h) const { return where.count(h) != 0; }
+  // h becomes the most recently used block
+  void touch(uint64_t h) {
+    auto it = where.find(h);
+    if (it != where.end()) {
+      order.splice(order.begin(), order, it->second);
+    } else {
+      order.push_front(h);
+      where[h] = order.begin();
+    }
+  }
+  // drop least recently used blocks until at most cap remain
+  void evict() {
+    while (order.size() > cap) {
+      where.erase(order.back());
+      order.pop_back();
+    }
+  }
+  // a request's chain enters the cache: its blocks are used from the last to the first,
+  // so that block 0 ends up the most recent and a cached prefix loses its tail first
+  void use_chain(const uint64_t* h, uint64_t n) {
+    for (uint64_t j = n; j-- > 0;) touch(h[j]);
+    evict();
+  }
+};
 
 }  // namespace
 
@@ -632,27 +669,37 @@ void oracle_schedule_stream_load(
   }
 }
 
-// Algorithm 1 with evolving caches (the simulator's cache update of Sec. VI-B, without its
-// LRU eviction): a stream starts from its decodes' cache contents (key lists keys,
-// key_off [D+1]); every arrival's prefix hits are taken against the caches as they are
-// at that arrival (first-miss scan, Sec. III-B), and a dispatch to d* adds every block of
-// the request's chain (chains, chain_off [R+1]) to K_{d*}.  Scores, feasibility and load
-// as oracle_schedule_stream.  M_out [R][D]: the hits each arrival was scored with.
+// Algorithm 1 with evolving caches: the simulator's LRU-managed block cache of Sec. VI-B.
+// A stream starts from its decodes' caches, given as key lists keys, key_off [D+1], each
+// list from the most to the least recently used block.  Every arrival's prefix hits are
+// taken against the caches as they are at that arrival (first-miss scan, Sec. III-B).  A
+// dispatch to d* uses every block of the request's chain (chains, chain_off [R+1]) on
+// K_{d*}: the blocks from the last to the first become the most recently used ones
+// (present blocks are refreshed, absent ones inserted), then least recently used blocks
+// are evicted until at most cap_blocks remain.  A list longer than cap_blocks is cut to
+// its cap_blocks most recent blocks at the start.  Departures leave the caches as they
+// are.  Scores, feasibility and load as oracle_schedule_stream.
+//   M_out [R][D]: the hits each arrival was scored with.
+//   cache_out (nullable) [D][cache_stride], cache_len [D]: each decode's cache after the
+//   last event, most recent first (cache_stride >= cap_blocks when cache_out is given).
 void oracle_schedule_stream_evolving(
     const uint32_t* fanout, const uint8_t* role, const double* bw, const double* lat,
     const float* util, uint64_t n_links, const uint32_t* len, const uint32_t* prefill,
-    const uint32_t* snap, const uint64_t* keys, const uint64_t* key_off,
+    const uint32_t* snap, const uint64_t* keys, const uint64_t* key_off, uint64_t cap_blocks,
     const uint64_t* chains, const uint64_t* chain_off, const uint32_t* events,
     uint64_t n_events, double w_net, double w_prefix, double w_load, double theta, int64_t cap,
     uint64_t bytes_per_token, const int32_t* hint, double rel_tol, int32_t* dec, double* best,
-    double* second, uint16_t* M_out, int64_t* load_out, int64_t* counts) {
+    double* second, uint16_t* M_out, int64_t* load_out, int64_t* counts, uint64_t* cache_out,
+    uint64_t cache_stride, uint64_t* cache_len) {
   const Tree t = make_tree(fanout);
   std::vector<uint64_t> pre, decs;
   ranks(role, t.n, pre, decs);
   const uint64_t D = decs.size();
-  std::vector<std::unordered_set<uint64_t>> K(D);
-  for (uint64_t d = 0; d < D; ++d)
-    for (uint64_t j = key_off[d]; j < key_off[d + 1]; ++j) K[d].insert(keys[j]);
+  std::vector<LruCache> K(D);
+  for (uint64_t d = 0; d < D; ++d) {
+    K[d].cap = cap_blocks;
+    K[d].use_chain(keys + key_off[d], key_off[d + 1] - key_off[d]);
+  }
   std::vector<int64_t> load(D, 0);
   std::vector<double> score(D);
   const double inf = std::numeric_limits<double>::infinity();
@@ -667,7 +714,7 @@ void oracle_schedule_stream_evolving(
     for (uint64_t d = 0; d < D; ++d) {  // hits against the caches as they are now
       uint64_t m = 0;
       for (uint64_t j = chain_off[r]; j < chain_off[r + 1]; ++j) {
-        if (K[d].count(chains[j]) == 0) break;
+        if (!K[d].contains(chains[j])) break;
         ++m;
       }
       M_out[(uint64_t)r * D + d] = (uint16_t)m;
@@ -706,10 +753,17 @@ void oracle_schedule_stream_evolving(
     second[r] = b2;
     if (chosen >= 0) {
       load[chosen] += l;
-      for (uint64_t j = chain_off[r]; j < chain_off[r + 1]; ++j) K[chosen].insert(chains[j]);
+      K[chosen].use_chain(chains + chain_off[r], chain_off[r + 1] - chain_off[r]);
     }
   }
-  for (uint64_t d = 0; d < D; ++d) load_out[d] = load[d];
+  for (uint64_t d = 0; d < D; ++d) {
+    load_out[d] = load[d];
+    if (cache_len) cache_len[d] = K[d].order.size();
+    if (cache_out) {
+      uint64_t i = 0;
+      for (uint64_t h : K[d].order) cache_out[d * cache_stride + i++] = h;
+    }
+  }
 }
 
 }  // extern "C"

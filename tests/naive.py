@@ -281,15 +281,27 @@ def greedy_exact_load(tree, role, bw, lat, util, length, prefill, snap, M, event
     return dec, best, n, m
 
 
+def lru_front(blocks, cache, cap):
+    """A recency list (most recent first) after `blocks` are used: the distinct blocks in
+    order of first appearance go to the front, the rest of the list keeps its order, and
+    the list is cut to its `cap` most recent entries."""
+    front = list(dict.fromkeys(int(b) for b in blocks))
+    seen = set(front)
+    merged = front + [k for k in cache if k not in seen]
+    return merged if cap is None else merged[:cap]
+
+
 def greedy_exact_evolving(tree, role, bw, lat, util, length, prefill, snap, keys_per_decode,
-                          chains, events, w, theta, cap, bpt):
+                          chains, events, w, theta, cap, bpt, cap_blocks=None):
     """Exact-rational Algorithm 1 with evolving caches: hits per arrival against the caches
-    of that moment (a list scan to the first miss), and a dispatch adds the request's whole
-    chain to its decode's cache.  Returns (dec, best, load, M)."""
+    of that moment (a list scan to the first miss), and a dispatch brings the request's
+    whole chain to the front of its decode's recency list, which keeps at most cap_blocks
+    entries (None: no limit).  Returns (dec, best, load, M, caches), caches most recent
+    first."""
     pre = [i for i in range(tree.n) if role[i] == 0]
     dec_inst = [i for i in range(tree.n) if role[i] == 1]
     D = len(dec_inst)
-    caches = [set(int(k) for k in keys_per_decode[d]) for d in range(D)]
+    caches = [lru_front(keys_per_decode[d], [], cap_blocks) for d in range(D)]
     load = [0] * D
     R = len(length)
     dec, best = [-1] * R, [None] * R
@@ -306,7 +318,7 @@ def greedy_exact_evolving(tree, role, bw, lat, util, length, prefill, snap, keys
             continue
         chain = [int(x) for x in chains[r]]
         for d in range(D):
-            M[r][d] = lcp_blocks(chain, caches[d])
+            M[r][d] = lcp_blocks(chain, set(caches[d]))
         p = pre[int(prefill[r])]
         u_row = util[int(snap[r])]
         cands = []
@@ -321,5 +333,5 @@ def greedy_exact_evolving(tree, role, bw, lat, util, length, prefill, snap, keys
             s, d = min(cands)
             dec[r], best[r] = d, s
             load[d] += l
-            caches[d].update(chain)
-    return dec, best, load, M
+            caches[d] = lru_front(chain, caches[d], cap_blocks)
+    return dec, best, load, M, caches

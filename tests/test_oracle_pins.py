@@ -931,15 +931,17 @@ def _evolving_problem(seed, R=10, span=1000):
     return pb
 
 
-def _run_evolving(pb, w, theta=float(np.float32(1e-6)), bpt=81920, cap=None):
-    keys = np.concatenate(pb["keys"])
+def _run_evolving(pb, w, theta=float(np.float32(1e-6)), bpt=81920, cap=None,
+                  cap_blocks=oracle.UNBOUNDED):
+    keys = np.concatenate([np.asarray(k, np.uint64) for k in pb["keys"]])
     key_off = np.concatenate([[0], np.cumsum([len(k) for k in pb["keys"]])]).astype(np.uint64)
-    chains = np.concatenate(pb["chains"])
+    chains = np.concatenate([np.asarray(c, np.uint64) for c in pb["chains"]])
     chain_off = np.concatenate([[0], np.cumsum([len(c) for c in pb["chains"]])]).astype(np.uint64)
     return oracle.schedule_stream_evolving(pb["fanout"], pb["role"], pb["bw"], pb["lat"], pb["u"],
                                            pb["length"], pb["prefill"], pb["snap"], keys, key_off,
                                            chains, chain_off, pb["events"], w[0], w[1], w[2],
-                                           theta, pb["cap"] if cap is None else cap, bpt)
+                                           theta, pb["cap"] if cap is None else cap, bpt,
+                                           cap_blocks=cap_blocks)
 
 
 def test_evolving_matches_exact_rational_bruteforce():
@@ -949,7 +951,7 @@ def test_evolving_matches_exact_rational_bruteforce():
         pb = _evolving_problem(seed)
         w = tuple(float(np.float32(x)) for x in np.random.default_rng(1400 + seed).uniform(0, 2, 3))
         res = _run_evolving(pb, w)
-        dec, best, load, M = naive.greedy_exact_evolving(
+        dec, best, load, M, _ = naive.greedy_exact_evolving(
             pb["tree"], pb["role"], pb["bw"], pb["lat"], pb["u"], pb["length"], pb["prefill"],
             pb["snap"], pb["keys"], pb["chains"], pb["events"], w, theta, pb["cap"], 81920)
         assert list(res.dec) == dec and list(res.load) == load
@@ -994,3 +996,103 @@ def test_evolving_dispatch_warms_its_decode():
     n = len(pb["chains"][0])
     assert d0 >= 0 and res.M[1, d0] == n
     assert all(res.M[1, d] == res.M[0, d] for d in range(4) if d != d0)
+
+
+# ------------------------------------------ LRU-managed caches (Sec. VI-B simulator)
+def test_evolving_lru_matches_exact_rational_bruteforce():
+    """Caches of a few dozen to a few hundred blocks, so that dispatches evict: decisions,
+    hits, final loads and the final recency lists equal the exact-rational evaluator's,
+    which keeps each cache as a plain list (most recent first) rebuilt on every dispatch."""
+    theta = float(np.float32(1e-6))
+    changed = 0
+    for seed in range(30):
+        pb = _evolving_problem(seed, R=14)
+        w = tuple(float(np.float32(x)) for x in np.random.default_rng(2400 + seed).uniform(0, 2, 3))
+        cap_blocks = (40, 120, 300)[seed % 3]
+        res = _run_evolving(pb, w, cap_blocks=cap_blocks)
+        dec, best, load, M, caches = naive.greedy_exact_evolving(
+            pb["tree"], pb["role"], pb["bw"], pb["lat"], pb["u"], pb["length"], pb["prefill"],
+            pb["snap"], pb["keys"], pb["chains"], pb["events"], w, theta, pb["cap"], 81920,
+            cap_blocks=cap_blocks)
+        assert list(res.dec) == dec and list(res.load) == load
+        np.testing.assert_array_equal(res.M, np.array(M, np.uint16))
+        for d in range(len(caches)):
+            assert [int(x) for x in res.caches[d]] == caches[d]
+            assert len(caches[d]) <= cap_blocks
+        for r in range(len(dec)):
+            if dec[r] >= 0:
+                assert res.best[r] == pytest.approx(float(best[r]), rel=1e-14)
+        free = _run_evolving(pb, w)
+        changed += int((free.M != res.M).sum() + (free.dec != res.dec).sum())
+    assert changed > 20  # eviction changed hits or decisions
+
+
+def _lru_case(keys, chains, lengths, cap_blocks, w=(0.0, 1.0, 0.0)):
+    """Arrivals only, one per chain, on the 4-decode tiny tree; prefix-only weights make
+    every candidate's score its missed fraction (ties to the lowest decode)."""
+    pb = _tiny_problem(7, R=len(chains))
+    pb["keys"] = [np.asarray(k, np.uint64) for k in keys]
+    pb["chains"] = [np.asarray(c, np.uint64) for c in chains]
+    pb["length"] = np.asarray(lengths, np.uint32)
+    pb["events"] = np.arange(len(chains), dtype=np.uint32)
+    pb["cap"] = 10 ** 9
+    return _run_evolving(pb, w, cap_blocks=cap_blocks)
+
+
+X = [1000 + i for i in range(10)]
+Y = [2000 + i for i in range(8)]
+
+
+def test_lru_eviction_changes_a_later_decision():
+    """d0 holds X0..X9, d1 holds X0..X5, each decode keeps 12 blocks.  A (8 new blocks,
+    no hits) goes to d0 (all tie); its blocks become d0's most recent and the 6 least
+    recent, X4..X9, are evicted.  B = X0..X9 then hits 4 blocks on d0 and 6 on d1 and goes
+    to d1, while without eviction it would hit all 10 on d0 and go there."""
+    keys = [X, X[:6], [], []]
+    res = _lru_case(keys, [Y, X], [128, 160], 12)
+    assert list(res.dec) == [0, 1]
+    assert list(res.M[1]) == [4, 6, 0, 0]
+    assert [int(h) for h in res.caches[0]] == Y + X[:4]
+    assert [int(h) for h in res.caches[1]] == X           # B's chain, X6..X9 inserted
+    free = _lru_case(keys, [Y, X], [128, 160], oracle.UNBOUNDED)
+    assert list(free.dec) == [0, 0] and list(free.M[1]) == [10, 6, 0, 0]
+
+
+def test_lru_chain_tail_is_evicted_first():
+    """A (C0..C9) to an empty d0, then B (4 new blocks) to d0 as well: d0 keeps 12 blocks,
+    so C8 and C9, the least recent (a chain's blocks are used from its last block to its
+    first), go; E = C0..C9 then hits 8 blocks on d0."""
+    C = [3000 + i for i in range(10)]
+    Dn = [4000 + i for i in range(4)]
+    res = _lru_case([[], [], [], []], [C, Dn, C], [160, 64, 160], 12)
+    assert list(res.dec[:2]) == [0, 0]
+    assert int(res.M[2, 0]) == 8
+    # E goes to d0 (8 hits) and refreshes the whole chain: C0..C9, then Dn0, Dn1
+    assert [int(h) for h in res.caches[0]] == C + Dn[:2]
+
+
+def test_lru_refresh_keeps_reused_blocks():
+    """d0 holds Z0..Z5 (most recent) then X0..X5.  A = X0 X1 X2 W0 W1 W2 hits 3 blocks on
+    d0 and goes there; its blocks become the most recent, so the 12-block cache evicts
+    X3..X5 and keeps the refreshed X0..X2: B = X0..X5 then hits 3 blocks on d0."""
+    Z = [5000 + i for i in range(6)]
+    W = [6000 + i for i in range(3)]
+    res = _lru_case([Z + X[:6], [], [], []], [X[:3] + W, X[:6]], [96, 96], 12)
+    assert int(res.dec[0]) == 0 and int(res.M[0, 0]) == 3
+    assert int(res.M[1, 0]) == 3
+    assert [int(h) for h in res.caches[0]][:12] == X[:6] + W + Z[:3]
+
+
+def test_lru_initial_list_cut_to_capacity():
+    """A key list longer than the capacity keeps its most recent (first) entries; with no
+    dispatch (nothing fits) the hits are the static match against those entries."""
+    K = [7000 + i for i in range(20)]
+    pb = _tiny_problem(11, R=1)
+    pb["keys"] = [np.asarray(K, np.uint64)] * 4
+    pb["chains"] = [np.asarray(K, np.uint64)]
+    pb["length"] = np.array([320], np.uint32)
+    pb["events"] = np.array([0], np.uint32)
+    res = _run_evolving(pb, (1.0, 1.0, 1.0), cap=0, cap_blocks=12)
+    assert int(res.dec[0]) == -1
+    assert list(res.M[0]) == [12] * 4
+    assert all([int(h) for h in c] == K[:12] for c in res.caches)
