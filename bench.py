@@ -67,6 +67,13 @@ def parse():
     ap.add_argument("--inflight", type=int, default=0,
                     help="self-contention counter cap (Eq. 4's n_inflight; the paper uses 16); "
                          "0 = the plain greedy")
+    ap.add_argument("--evolving", type=int, default=0,
+                    help="evolving LRU decode caches of this many blocks (the simulator's "
+                         "caches, Sec. VI-B; 200000 = the configs' cache size); 0 = static "
+                         "caches")
+    ap.add_argument("--evolving-batch", type=int, default=1024,
+                    help="streams whose caches are held at once (the state of a 200,000-block "
+                         "cache is 12 MiB)")
     ap.add_argument("--streams", type=int, default=4096)
     ap.add_argument("--cpu-streams", type=int, default=256,
                     help="streams of the multi-core CPU-oracle sample (one per core at a time)")
@@ -77,6 +84,9 @@ def parse():
     ap.add_argument("--table-batch", type=int, default=256)
     ap.add_argument("--e2e-copy-chains", action="store_true",
                     help="e2e: copy the chains to the device instead of reading them in place")
+    ap.add_argument("--no-fuse", action="store_true",
+                    help="build the level bottlenecks UB in their own pass (netkv_oracle_build) "
+                         "instead of from the utilisation rows inside the base-score pass")
     ap.add_argument("--no-share", action="store_true",
                     help="prefix match without the workspace (no grouping of shared prefixes)")
     return ap.parse_args()
@@ -559,6 +569,7 @@ def run_netkv(args):
                                    directed=args.directed, tiers=args.tiers)
     sc.share_prefixes = not args.no_share
     sc.inflight_cap = args.inflight
+    sc.fuse_level_bottlenecks = not args.no_fuse
     if args.load_model:
         from paper_2606_03910_gb300 import netkv
         sc.load_model = netkv.LoadModel(*LOAD_MODEL)
@@ -573,7 +584,10 @@ def run_netkv(args):
         raise RuntimeError(f"device status {int(out.status.item())} after warm-up")
 
     # ---- timed region: device-resident inputs
-    names = ("oracle_build", "prefix_match", "schedule")
+    fused = sc.fused(x)
+    names = ("prefix_match", "schedule") if fused else ("oracle_build", "prefix_match", "schedule")
+    calls = ((sc.prefix_match, sc.schedule) if fused
+             else (sc.oracle_build, sc.prefix_match, sc.schedule))
     ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
            for _ in names] for _ in range(args.steps)]
     t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -584,7 +598,7 @@ def run_netkv(args):
     clocks.start()
     t0.record(stream)
     for k in range(args.steps):
-        for j, fn in enumerate((sc.oracle_build, sc.prefix_match, sc.schedule)):
+        for j, fn in enumerate(calls):
             ev[k][j][0].record(stream)
             fn(x, out, stream)
             ev[k][j][1].record(stream)
@@ -604,7 +618,7 @@ def run_netkv(args):
     R, D = x.R, sc.D
     # level bottlenecks 1; prefix match 4 (group insert, group resolve, leaders, members)
     # with a workspace or 1 without; greedy 2 (base scores + walk) with a workspace or 1
-    launches_per_step = 1 + (4 if sc.share_prefixes else 1) + (
+    launches_per_step = (0 if fused else 1) + (4 if sc.share_prefixes else 1) + (
         1 if (sc.inflight_cap > 0 or sc.load_model is not None)
         else (2 if sc.precompute_scores else 1))
     n_input_tensors = sum(1 for f in dataclasses.fields(StepInputs)
@@ -620,7 +634,7 @@ def run_netkv(args):
         # them over shared prefixes and L2 serves most of the rest)
         "prefix_match": 8 * examined + 2 * R * D,
         # per snapshot: the utilisation row (L floats), 16-byte UB of every instance
-        "oracle_build": x.n_snap * (16 + 16 * sc.N) if args.tiers else
+        "oracle_build": 0 if fused else x.n_snap * (16 + 16 * sc.N) if args.tiers else
                         x.n_snap * ((8 if x.util_down is not None else 4) * w.L + 16 * sc.N),
         # per arrival: event, len/prefill/snap, per candidate base score (4 B) + the
         # dec/best/second stores; per departure: event, len, dec
@@ -759,6 +773,7 @@ def run_single(args):
     theta = float(np.float32(synth.THETA_S_PER_TOKEN))
     bpt = synth.BYTES_PER_TOKEN_SHARD
     R, D = x.R, sc.D
+    sc.fuse_level_bottlenecks = not args.no_fuse
     stream = torch.cuda.Stream(dev)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
 
@@ -776,8 +791,9 @@ def run_single(args):
         return g
 
     # the stream's step: grouping, leaders and members (with the workspace), base scores
-    # and the walk: 7 launches
+    # (level bottlenecks from the utilisation rows) and the walk: 6 launches
     g_step = capture(lambda st: sc.step(x, out, st), True, True)
+    step_launches = 6 if sc.fused(x) else 7
     # one decision: one request against the 8 decodes, no workspaces: 3 launches
     r_one = int(w.req_off[0]) + R // 2
     x1 = one_decision_inputs(x, r_one)
@@ -866,13 +882,13 @@ def run_single(args):
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                 "dtype": "f32", "data": "synthetic",
                 "config": workload_config(1, world, kind="single"),
-                "scores_per_s": value * D, "gpu_launches": 10 * args.steps,
+                "scores_per_s": value * D, "gpu_launches": (step_launches + 3) * args.steps,
                 "latency": {"stream_step_ms": round(step_ms, 4),
                             "stream_step_ms_median": round(step_med, 4),
                             "per_decision_us_amortised": round(1e3 * step_ms / R, 3),
                             "one_decision_ms": round(one_ms, 4),
                             "one_decision_ms_median": round(one_med, 4),
-                            "launches": {"stream_step": 7, "one_decision": 3},
+                            "launches": {"stream_step": step_launches, "one_decision": 3},
                             "paper": "decision latency below 1.5 ms at up to 1,024 GPUs "
                                      "(Sec. VI-I, Experiment 7), candidate pool of at most 12 "
                                      "after memory filtering (Sec. V-B); the paper's scheduler "
@@ -883,6 +899,158 @@ def run_single(args):
                                      "8 MB: launch- and dependency-bound, so no HBM "
                                      "roofline; the replicas workload carries it"},
                 "cpu_baseline": cpu, "e2e": e2e, "clocks": clk}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def run_evolving(args):
+    """The replicas workload with evolving LRU caches: one step is the level bottlenecks
+    of every snapshot, then, per batch of streams, their caches set from the key lists
+    (netkv_lru_init) and hits plus greedy in one walk (netkv_schedule_streams_evolving)."""
+    import torch
+    import synth
+    import synth.device as sdev
+    from synth import stage
+    import __graft_entry__
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    __graft_entry__.build()
+    from paper_2606_03910_gb300 import netkv
+    from paper_2606_03910_gb300.pipeline import Scorer, StepInputs, weights_tensor
+    spec = workload_spec("replicas", args.streams, rank, args.requests)
+    w = synth.make_workload(spec)
+    theta = float(np.float32(synth.THETA_S_PER_TOKEN))
+    bpt = synth.BYTES_PER_TOKEN_SHARD
+    sc = Scorer(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, w.L, w.n_sets, 1, device=dev,
+                index=False)
+    S, D = w.n_streams, sc.D
+    batch = max(1, min(args.evolving_batch, S))
+    sc.lru_setup(batch, args.evolving)
+    keys = sdev.keys(w, 0, w.n_sets, device=dev)       # every stream's initial caches
+    key_off = stage.key_offsets(w, w.n_sets * D, device=dev)
+    ra = stage.request_arrays(w, device=dev)
+    chains, _ = sdev.chains(w, device=dev)
+    x = StepInputs(util=sdev.util(w, device=dev), chains=chains, chain_off=ra["chain_off"],
+                   set_off=ra["set_off"], length=ra["length"], prefill=ra["prefill"],
+                   snap=ra["snap"], events=ra["events"], event_off=ra["event_off"],
+                   weights=weights_tensor(w.weights, theta, spec.cap_tokens, bpt, device=dev))
+    out = sc.alloc_outputs(x.n_snap, x.R, x.n_streams)
+    stream = torch.cuda.current_stream(dev)
+    batches = [(j0, min(S, j0 + batch)) for j0 in range(0, S, batch)]
+
+    def step(ev=None):
+        if ev:
+            ev[0].record(stream)
+        sc.oracle_build(x, out, stream)
+        if ev:
+            ev[1].record(stream)
+        for k, (j0, j1) in enumerate(batches):
+            netkv.netkv_lru_init(sc.lru_state, (j1 - j0) * D, sc.lru_cfg, keys, key_off[j0 * D:],
+                                 out.status, stream)
+            if ev:
+                ev[2 + 2 * k].record(stream)
+            sc.schedule_evolving(x, out, stream, streams=(j0, j1))
+            if ev:
+                ev[3 + 2 * k].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if int(out.status.item()) != 0:
+        raise RuntimeError(f"device status {int(out.status.item())} after warm-up")
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2 + 2 * len(batches))]
+           for _ in range(args.steps)]
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = Clocks(local)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    t0.record(stream)
+    for k in range(args.steps):
+        step(evs[k])
+    t1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, dev)
+    if int(out.status.item()) != 0:
+        raise RuntimeError(f"device status {int(out.status.item())} in the timed region")
+    nb = len(batches)
+    t_build = sum(e[0].elapsed_time(e[1]) for e in evs) / args.steps
+    t_init = sum(sum((e[1] if b == 0 else e[1 + 2 * b]).elapsed_time(e[2 + 2 * b]) for b in range(nb))
+                 for e in evs) / args.steps
+    t_walk = sum(sum(e[2 + 2 * b].elapsed_time(e[3 + 2 * b]) for b in range(nb))
+                 for e in evs) / args.steps
+    R = x.R
+    value = R * world / (ms / 1e3)
+    # algorithmic bytes of the walk: per (arrival, decode) probe up to the first miss a chain
+    # block (8 B) and a table slot (16 B); per block a dispatch uses, its log entry (8 B) and
+    # slot (16 B); per evicted block, as many again (taken as the blocks a dispatch adds
+    # beyond its hits on the chosen decode)
+    M = out.M.to(torch.int64) & 0xFFFF
+    nblk = (x.chain_off[1:] - x.chain_off[:-1]).to(torch.int64)
+    probes = int(torch.minimum(M + 1, nblk[:, None]).sum().item())
+    dsel = out.dec.to(torch.int64)
+    ok = dsel >= 0
+    used = int(nblk[ok].sum().item())
+    hits_sel = int(M[ok].gather(1, dsel[ok][:, None]).sum().item())
+    algo = 24 * probes + 24 * used + 24 * max(0, used - hits_sel)
+    peak, peak_src = measured_peaks()
+    achieved = algo / (t_walk / 1e3) / 1e9
+    roofline = {"kernel": "evolving_kernel (netkv_schedule_streams_evolving)", "bound": "hbm",
+                "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "traffic": None, "peak_source": peak_src,
+                "algorithmic_bytes_per_launch": algo,
+                "per_unit": "24 B per (arrival, decode) probe up to the first miss, 24 B per "
+                            "block used by a dispatch, 24 B per block it adds (evictions)",
+                "note": "a sequential walk per stream: bound by each arrival's chain of "
+                        "dependent probes, not by bandwidth",
+                "kernel_ms": {"oracle_build": round(t_build, 4), "lru_init": round(t_init, 4),
+                              "evolving_walk": round(t_walk, 4)}}
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        from oracle.workload import run_stream_evolving
+        import concurrent.futures as cf
+        import oracle
+        sample = np.random.default_rng(0).choice(S, size=min(args.cpu_streams_1t, S),
+                                                 replace=False)
+        oracle.lib()
+
+        def one(s):
+            oracle.set_threads(1)
+            t = time.perf_counter()
+            res = run_stream_evolving(w, int(s), theta, spec.cap_tokens, bpt, args.evolving)
+            return int(res.dec.shape[0]), time.perf_counter() - t
+
+        with cf.ThreadPoolExecutor(cpu_cores()) as ex:
+            t0w = time.perf_counter()
+            got = list(ex.map(one, sample))
+            wall = time.perf_counter() - t0w
+        d = sum(g[0] for g in got)
+        cpu = {"value": d / wall, "unit": UNIT, "cores": min(cpu_cores(), len(sample)),
+               "kind": "oracle",
+               "sample": f"{len(sample)} whole streams ({d} decisions in {wall:.1f} s), one per "
+                         "core; each includes gathering its key lists and chains from the "
+                         "generator (about a tenth of its time)",
+               "one_thread": {"value": d / sum(g[1] for g in got), "unit": UNIT, "cores": 1,
+                              "sample": "the same streams, per-thread time"}}
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 4),
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": "f32", "data": "synthetic",
+                "config": workload_config(args.streams, world, kind="replicas",
+                                          extra={"caches": f"evolving, LRU of {args.evolving} "
+                                                           "blocks per decode (Sec. VI-B)",
+                                                 "streams_per_batch": batch}),
+                "scores_per_s": value * D, "gpu_launches": (1 + 2 * nb) * args.steps,
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": None, "clocks": clk}
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
@@ -995,15 +1163,19 @@ def run_sweep(args):
 
 def main():
     args = parse()
-    if (args.inflight > 0) + args.directed + args.tiers + args.load_model > 1:
-        raise SystemExit("--inflight, --directed, --tiers and --load-model are measured one "
-                         "at a time")
+    if (args.inflight > 0) + args.directed + args.tiers + args.load_model + (args.evolving > 0) > 1:
+        raise SystemExit("--inflight, --directed, --tiers, --load-model and --evolving are "
+                         "measured one at a time")
+    if args.evolving and args.workload != "replicas":
+        raise SystemExit("--evolving runs on the replicas workload (one table set per stream)")
     if args.impl == "reference":
         return run_reference(args)
     if args.workload == "sweep":
         return run_sweep(args)
     if args.workload == "single":
         return run_single(args)
+    if args.evolving:
+        return run_evolving(args)
     return run_netkv(args)
 
 

@@ -18,6 +18,8 @@
  *   netkv_schedule_streams  the greedy of Algorithm 1 over independent streams
  *   netkv_schedule_streams_inflight  the same with self-contention (Eq. 4's n_inflight)
  *   netkv_schedule_streams_load      the same with the paper's queue/decode-step model
+ *   netkv_schedule_streams_evolving  the same with LRU-managed caches that change with
+ *                                    every dispatch (Sec. VI-B), set by netkv_lru_init
  *
  * Conventions for every call:
  *   - Pointers named d_* are device pointers owned by the caller; the library never
@@ -293,6 +295,22 @@ netkv_status netkv_schedule_streams(netkv_topology_t topo, uint32_t n_streams,
                                     float* d_second, int64_t* d_load_final, void* d_workspace,
                                     size_t workspace_bytes, int* d_status, netkv_stream_t stream);
 
+/* netkv_schedule_streams with the level bottlenecks taken from the telemetry itself: d_util
+ * [n_snap][n_links] fp32 utilisation rows (as for netkv_oracle_build) replace d_UB, and the
+ * base-score pass computes each candidate's min(UB[k][p][tau], UB[k][d][tau]) from the
+ * utilisations of the links of p and d in row k, with the arithmetic of netkv_oracle_build.
+ * So the results equal those of netkv_oracle_build(d_UB) followed by
+ * netkv_schedule_streams with a workspace, without writing UB.  The workspace is required
+ * (EINVAL when NULL or smaller than netkv_schedule_workspace_size(R, D)); other arguments
+ * and errors as netkv_schedule_streams, plus EDOMAIN for a utilisation outside [0, 1). */
+netkv_status netkv_schedule_streams_util(
+    netkv_topology_t topo, uint32_t n_streams, const netkv_weights* d_w, uint32_t R,
+    const uint32_t* d_len, const uint32_t* d_prefill, const uint32_t* d_snap, const uint16_t* d_M,
+    const float* d_util, uint32_t n_snap, const uint32_t* d_events, const uint64_t* d_event_off,
+    const int64_t* d_load_init, int32_t* d_dec, float* d_best, float* d_second,
+    int64_t* d_load_final, void* d_workspace, size_t workspace_bytes, int* d_status,
+    netkv_stream_t stream);
+
 /* Algorithm 1 with self-contention (Eq. 4's n_inflight term, Algorithm 1 lines 5 and 14,
  * Sec. V-C).  As netkv_schedule_streams without a workspace, and in addition each
  * stream keeps a counter n[p][tau] per prefill rank and tier (zero at the start of the
@@ -370,6 +388,75 @@ netkv_status netkv_schedule_streams_load(
     const uint32_t* d_events, const uint64_t* d_event_off, const int64_t* d_m_init,
     const int32_t* d_n_init, int32_t* d_dec, float* d_best, float* d_second, int64_t* d_m_final,
     int32_t* d_n_final, int* d_status, netkv_stream_t stream);
+
+/* ------------------------------------------------------------------ evolving caches
+ * The decode caches of the simulator of Sec. VI-B, LRU-managed KV-block caches that change
+ * with every dispatch.  Each (stream, decode) pair has its own cache, number
+ * c = stream * D + d, holding at most cap_blocks block hashes in recency order:
+ *   - netkv_lru_init sets every cache from a key list given from the most to the least
+ *     recently used block;
+ *   - in netkv_schedule_streams_evolving, a dispatch of request r to d* uses every block
+ *     of r's chain on cache (stream, d*), from the last block to the first, so that
+ *     block 0 becomes the most recently used one (a cached prefix loses its tail first);
+ *     present blocks are refreshed, absent ones inserted, and then the least recently
+ *     used blocks beyond cap_blocks are evicted.  Departures leave the caches unchanged.
+ * The caches live in a caller-owned state buffer of netkv_lru_state_bytes(n_caches, cfg)
+ * bytes (16-byte aligned) that the greedy updates in place, so a later call continues
+ * from the caches an earlier call left.  Per cache it holds a hash table of
+ * 2^log2_slots 16-byte slots and a recency log of 2^log2_ring 8-byte entries: 12 MiB for
+ * 2^19 of each, enough for caches of 200,000 blocks.
+ */
+typedef struct {
+  uint64_t cap_blocks; /* blocks a cache keeps (>= 1); the least recently used beyond go */
+  uint32_t log2_slots; /* hash slots per cache: (3/4) 2^log2_slots >= cap_blocks + 65535 */
+  uint32_t log2_ring;  /* recency-log entries per cache: 2^log2_ring >= cap_blocks + 65536 */
+} netkv_lru_config;   /* 16 bytes */
+
+/* Bytes of state for n_caches caches; 0 for an invalid configuration. */
+size_t netkv_lru_state_bytes(uint64_t n_caches, const netkv_lru_config* cfg);
+
+/* Sets caches [0, n_caches) of d_state (state_bytes bytes, at least
+ * netkv_lru_state_bytes(n_caches, cfg)) from key lists: cache c holds
+ * d_keys[d_key_off[c] .. d_key_off[c+1]), most recently used first (d_key_off has
+ * n_caches + 1 uint64 entries).  d_keys = NULL sets every cache empty.  A list longer than
+ * cap_blocks sets ERANGE and keeps its first cap_blocks entries; a zero key sets EDOMAIN
+ * and is skipped; repeated keys count once, at their first (most recent) entry.
+ * Host errors: EINVAL for a bad configuration or buffer. */
+netkv_status netkv_lru_init(void* d_state, size_t state_bytes, uint64_t n_caches,
+                            const netkv_lru_config* cfg, const uint64_t* d_keys,
+                            const uint64_t* d_key_off, int* d_status, netkv_stream_t stream);
+
+/* Every cache's blocks from the most to the least recently used:
+ * d_keys_out [n_caches][cap_blocks] (cache c's list starts at c * cap_blocks) and
+ * d_len_out [n_caches] its length.  Reads the state only. */
+netkv_status netkv_lru_export(const void* d_state, size_t state_bytes, uint64_t n_caches,
+                              const netkv_lru_config* cfg, uint64_t* d_keys_out,
+                              uint64_t* d_len_out, int* d_status, netkv_stream_t stream);
+
+/* Algorithm 1 (Sec. V-A) with evolving caches.  As netkv_schedule_streams without a
+ * workspace (scores, feasibility, argmin, loads, departures), except that the prefix hits
+ * are not an input: each arrival's hits on every decode are taken against the stream's
+ * caches in d_state as they are at that arrival (the first-miss scan of Sec. III-B), and
+ * a dispatch updates the chosen decode's cache as described above.
+ *
+ *   d_chains, d_chain_off  request chains as for netkv_prefix_match ([R+1] offsets;
+ *                          a chain longer than 65535 blocks sets EDOMAIN and is cut)
+ *   d_state                caches of n_streams * D decodes from netkv_lru_init (or an
+ *                          earlier call), with the same cfg; updated in place
+ *   state_bytes            size of d_state, at least netkv_lru_state_bytes(n_streams * D,
+ *                          cfg) (EINVAL otherwise)
+ *   d_M                    [R][D] uint16 output: the hits each arrival was scored with
+ * Other arguments as netkv_schedule_streams.  A zero hash in a chain sets EDOMAIN, counts as
+ * a miss and is not cached.  The decode pool may have at most 1024 instances.  Calls that
+ * overlap on the GPU need distinct state buffers.
+ */
+netkv_status netkv_schedule_streams_evolving(
+    netkv_topology_t topo, uint32_t n_streams, const netkv_weights* d_w, uint32_t R,
+    const uint32_t* d_len, const uint32_t* d_prefill, const uint32_t* d_snap, const float* d_UB,
+    uint32_t n_snap, const uint64_t* d_chains, const uint64_t* d_chain_off,
+    const uint32_t* d_events, const uint64_t* d_event_off, void* d_state, size_t state_bytes,
+    const netkv_lru_config* cfg, const int64_t* d_load_init, int32_t* d_dec, float* d_best,
+    float* d_second, uint16_t* d_M, int64_t* d_load_final, int* d_status, netkv_stream_t stream);
 
 /* ------------------------------------------------------------------ transfers
  * Asynchronous copy of `bytes` bytes by a kernel (SM loads and stores).  Either side may

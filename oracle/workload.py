@@ -17,8 +17,8 @@ from typing import Optional
 
 import numpy as np
 
-from . import (level_bottleneck_directed, prefix_match, schedule_stream, schedule_stream_inflight,
-               schedule_stream_load, up_bottleneck)
+from . import (level_bottleneck_directed, prefix_match, schedule_stream, schedule_stream_evolving,
+               schedule_stream_inflight, schedule_stream_load, up_bottleneck)
 
 
 @dataclasses.dataclass
@@ -203,3 +203,20 @@ def run_stream_load(w, s: int, t_a: float, t_b: float, beta_max: int, m_min: int
                                rel_tol=rel_tol)
     res.M = M
     return res
+
+
+def run_stream_evolving(w, s: int, theta: float, cap: int, bytes_per_token: int, cap_blocks: int,
+                        hint: Optional[np.ndarray] = None, rel_tol: float = 1e-5):
+    """Oracle for stream s with evolving LRU caches of cap_blocks blocks (Sec. VI-B): the
+    stream's decodes start from its table set's key lists, most recently used first.
+    hint: another implementation's decisions (local order).  Returns the oracle's
+    EvolvingResult (hits per arrival .M, final caches .caches)."""
+    x = stream_inputs(w, s)
+    r0, r1 = x.r0, x.r1
+    wn, wp, wl = (float(v) for v in w.weights[s])
+    spec = w.spec
+    return schedule_stream_evolving(spec.fanout, w.role, spec.tier_bw, spec.tier_lat, x.util,
+                                    w.length[r0:r1], w.prefill[r0:r1], x.snap_local, x.keys,
+                                    x.key_off, x.chains, x.chain_off, x.ev_local, wn, wp, wl,
+                                    theta, cap, bytes_per_token, hint=hint, rel_tol=rel_tol,
+                                    cap_blocks=cap_blocks)

@@ -19,7 +19,7 @@
 // shrinks to a load, a capacity test, one multiply-add and the argmin per candidate.
 #include <math.h>
 
-#include "netkv_internal.cuh"
+#include "score.cuh"
 
 namespace {
 
@@ -47,23 +47,6 @@ __device__ __forceinline__ void seg_argmin(float& b, uint32_t& i, float& s, uint
     const float s2 = __shfl_xor_sync(mask, s, o, LPS);
     combine(b, i, s, b2, i2, s2);
   }
-}
-
-// Decision-independent part of a candidate's score (Algorithm 1 lines 5-8, Eq. 2, Eq. 3):
-// w_net * (s_eff / min(UB_p[tau], UB_d[tau]) + L_tau) + w_prefix * (l - 16 M) / l.
-__device__ __forceinline__ float base_score(const netkv_weights& w, uint32_t l, uint32_t m,
-                                            float ub_p, float ub_d, float lat_tau, int* status) {
-  uint32_t lam = 16u * m;
-  if (m > l / 16u) {
-    flag_status(status, NETKV_DEV_EDOMAIN);
-    lam = lam < l ? lam : l;
-  }
-  const uint32_t miss_tok = l - lam;
-  const float bb = fminf(ub_p, ub_d);
-  const float s_eff = (float)((int64_t)miss_tok * (int64_t)w.bytes_per_token);
-  const float T = s_eff / bb + lat_tau;
-  const float miss = (float)miss_tok / (float)l;
-  return w.w_net * T + w.w_prefix * miss;
 }
 
 // The paper's compute-load model (Sec. III-C, IV-B) as kernel parameters.
@@ -164,7 +147,9 @@ __device__ __forceinline__ float xfer_factor(const netkv_weights& w, uint32_t l,
 // No dependence between events, so the events of a stream are split into contiguous
 // ranges over the segments (LPS lanes each) of grid.y blocks; each segment strides over
 // one row's decodes.  Departures and invalid events are skipped (the greedy reports them).
-template <int LPS>
+// kUtil: `UB` holds the utilisation rows [n_snap][n_links] instead of the level
+// bottlenecks, and each candidate's bottlenecks are taken from its links' entries.
+template <int LPS, bool kUtil = false>
 __global__ void __launch_bounds__(256, 8) base_kernel(
     TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
     const uint32_t* __restrict__ len, const uint32_t* __restrict__ prefill,
@@ -195,12 +180,15 @@ __global__ void __launch_bounds__(256, 8) base_kernel(
       if (pr >= t.P || k >= n_snap || l == 0) continue;
       const uint32_t pinst = __ldg(t.pre + pr);
       const uint4 lp = __ldg(t.links + pinst);
-      const float4 ubp = __ldg(reinterpret_cast<const float4*>(UB) + (uint64_t)k * N + pinst);
+      const float* urow = UB + (uint64_t)k * t.n_links;
+      const float4 ubp = kUtil ? level_bottlenecks_of(t, urow, lp, status)
+                               : __ldg(reinterpret_cast<const float4*>(UB) + (uint64_t)k * N + pinst);
       const float* ub_row = UB + (uint64_t)k * N * 4;
       for (uint32_t d = sl; d < D; d += LPS) {
         const uint4 ld = __ldg(t.links + __ldg(t.dec + d));
         const int tau = tier_of(lp, ld);
-        const float ubd = __ldg(ub_row + (uint64_t)ld.x * 4 + tau);
+        const float ubd = kUtil ? pick4(level_bottlenecks_of(t, urow, ld, status), tau)
+                                : __ldg(ub_row + (uint64_t)ld.x * 4 + tau);
         const uint32_t m = __ldg(M + (uint64_t)r * D + d);
         base[(uint64_t)r * D + d] = base_score(w, l, m, pick4(ubp, tau), ubd, pick4(lat, tau), status);
         if (X) X[(uint64_t)r * D + d] = xfer_factor(w, l, m, pick4(ubp, tau), ubd);
@@ -215,8 +203,8 @@ __global__ void __launch_bounds__(256, 8) base_kernel(
 // An arrival's request fields and the thread's NPT prefix hits are loaded one arrival
 // ahead, so the per-arrival chain of dependent loads overlaps the previous arrival's
 // scoring; prefix hits are read 8 bytes and scores written 16 bytes at a time when the
-// rows allow it.
-template <int NPT>
+// rows allow it.  kUtil: as for base_kernel (UB holds the utilisation rows).
+template <int NPT, bool kUtil = false>
 __global__ void __launch_bounds__(256) base_wide_kernel(
     TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
     const uint32_t* __restrict__ len, const uint32_t* __restrict__ prefill,
@@ -288,13 +276,17 @@ __global__ void __launch_bounds__(256) base_wide_kernel(
       if (r == kBad) continue;
       const uint32_t pinst = __ldg(t.pre + pr);
       const uint4 lp = __ldg(t.links + pinst);
-      const float4 ubp = __ldg(reinterpret_cast<const float4*>(UB) + (uint64_t)k * N + pinst);
+      const float* urow = UB + (uint64_t)k * t.n_links;
+      const float4 ubp = kUtil ? level_bottlenecks_of(t, urow, lp, status)
+                               : __ldg(reinterpret_cast<const float4*>(UB) + (uint64_t)k * N + pinst);
       const float* ub_row = UB + (uint64_t)k * N * 4;
       float out[NPT];
 #pragma unroll
       for (int j = 0; j < NPT; ++j) {
         const int tau = tier_of(lp, ld[j]);
-        const float ubd = d0 + j < D ? __ldg(ub_row + (uint64_t)ld[j].x * 4 + tau) : 1.0f;
+        const float ubd = d0 + j >= D ? 1.0f
+                          : kUtil ? pick4(level_bottlenecks_of(t, urow, ld[j], status), tau)
+                                  : __ldg(ub_row + (uint64_t)ld[j].x * 4 + tau);
         out[j] = base_score(w, l, m[j], pick4(ubp, tau), ubd, pick4(lat, tau), status);
         if (X && d0 + j < D) X[(uint64_t)r * D + d0 + j] = xfer_factor(w, l, m[j], pick4(ubp, tau), ubd);
       }
@@ -1065,6 +1057,7 @@ netkv_status launch_staged(const TopoArgs& t, uint32_t n_streams, const netkv_we
 
 // The base-score pre-pass over every arrival (and, with d_X, the factor s_eff / Bbot that
 // self-contention scales).
+template <bool kUtil = false>
 netkv_status launch_base(const TopoArgs& t, uint32_t n_streams, const netkv_weights* d_w,
                          uint32_t R, const uint32_t* d_len, const uint32_t* d_prefill,
                          const uint32_t* d_snap, const uint16_t* d_M, const float* d_UB,
@@ -1074,13 +1067,13 @@ netkv_status launch_base(const TopoArgs& t, uint32_t n_streams, const netkv_weig
     const unsigned gy = n_streams >= 1024u ? 1u : (1024u + n_streams - 1) / n_streams;
     const dim3 bgrid(n_streams < (1u << 20) ? n_streams : (1u << 20), gy);
     if (D <= 8)
-      base_kernel<8><<<bgrid, 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,
+      base_kernel<8, kUtil><<<bgrid, 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,
                                            d_UB, n_snap, d_events, d_event_off, d_base, d_status, d_X);
     else if (D <= 16)
-      base_kernel<16><<<bgrid, 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,
+      base_kernel<16, kUtil><<<bgrid, 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,
                                             d_UB, n_snap, d_events, d_event_off, d_base, d_status, d_X);
     else if (D <= 32)
-      base_kernel<32><<<bgrid, 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,
+      base_kernel<32, kUtil><<<bgrid, 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,
                                             d_UB, n_snap, d_events, d_event_off, d_base, d_status, d_X);
     else {
       // one block per (stream, chunk of decodes) and arrival segment, ~32 blocks per SM
@@ -1093,18 +1086,18 @@ netkv_status launch_base(const TopoArgs& t, uint32_t n_streams, const netkv_weig
       const unsigned wx = (unsigned)(gx < (1u << 20) ? gx : (1u << 20));
       const unsigned wy = (unsigned)(gx >= want ? 1 : (want + gx - 1) / gx < 65535 ? (want + gx - 1) / gx : 65535);
       if (D <= 256)
-        base_wide_kernel<1><<<dim3(wx, wy), 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill,
+        base_wide_kernel<1, kUtil><<<dim3(wx, wy), 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill,
                                                          d_snap, d_M, d_UB, n_snap, d_events,
                                                          d_event_off, d_base, d_status, d_X);
       else
-        base_wide_kernel<4><<<dim3(wx, wy), 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill,
+        base_wide_kernel<4, kUtil><<<dim3(wx, wy), 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill,
                                                          d_snap, d_M, d_UB, n_snap, d_events,
                                                          d_event_off, d_base, d_status, d_X);
     }
   return netkv_launch_status();
 }
 
-template <int NPT, int BLOCK, int LPS>
+template <int NPT, int BLOCK, int LPS, bool kUtil = false>
 netkv_status launch(const TopoArgs& t, uint32_t n_streams, const netkv_weights* d_w, uint32_t R,
                     const uint32_t* d_len, const uint32_t* d_prefill, const uint32_t* d_snap,
                     const uint16_t* d_M, const float* d_UB, uint32_t n_snap,
@@ -1114,8 +1107,8 @@ netkv_status launch(const TopoArgs& t, uint32_t n_streams, const netkv_weights* 
   const uint32_t per_cta = LPS == 32 ? 1u : 32u / LPS;
   const unsigned grid = (n_streams + per_cta - 1) / per_cta;
   if (d_base) {
-    if (launch_base(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events,
-                    d_event_off, d_base, nullptr, d_status, s) != NETKV_OK)
+    if (launch_base<kUtil>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M, d_UB, n_snap,
+                           d_events, d_event_off, d_base, nullptr, d_status, s) != NETKV_OK)
       return NETKV_ECUDA;
     if (LPS == 32) {
       // one CTA per stream: the walk is bound by each warp's chain of dependent
@@ -1234,6 +1227,50 @@ extern "C" netkv_status netkv_schedule_streams(
   if (D <= 1024) NETKV_SCHED(4, 256, 32);
   if (D <= 4096) NETKV_SCHED(4, 1024, 32);
 #undef NETKV_SCHED
+  return NETKV_EINVAL;
+}
+
+// The same greedy with the level bottlenecks taken from the utilisation rows inside the
+// base-score pass (see include/netkv.h): the workspace is required, and every launch is
+// the workspace form of netkv_schedule_streams, whose walks never read UB.
+extern "C" netkv_status netkv_schedule_streams_util(
+    netkv_topology_t topo, uint32_t n_streams, const netkv_weights* d_w, uint32_t R,
+    const uint32_t* d_len, const uint32_t* d_prefill, const uint32_t* d_snap, const uint16_t* d_M,
+    const float* d_util, uint32_t n_snap, const uint32_t* d_events, const uint64_t* d_event_off,
+    const int64_t* d_load_init, int32_t* d_dec, float* d_best, float* d_second,
+    int64_t* d_load_final, void* d_workspace, size_t workspace_bytes, int* d_status,
+    netkv_stream_t stream) {
+  if (!topo || !d_w || !d_event_off || !d_load_final) return NETKV_EINVAL;
+  if (n_streams == 0) return NETKV_OK;
+  if (n_streams > 0x7fffffffu) return NETKV_EINVAL;
+  if (R > 0 && (!d_len || !d_prefill || !d_snap || !d_M || !d_util || !d_dec || !d_best ||
+                !d_second || !d_events))
+    return NETKV_EINVAL;
+  if (!aligned_to(d_w, 8) || !aligned_to(d_event_off, 8) || !aligned_to(d_load_final, 8) ||
+      (d_util && !aligned_to(d_util, 4)) || (d_load_init && !aligned_to(d_load_init, 8)))
+    return NETKV_EINVAL;
+  const TopoArgs t = topo_args(topo);
+  const uint32_t D = t.D;
+  cudaStream_t s = (cudaStream_t)stream;
+  if (!d_workspace || !aligned_to(d_workspace, 256) ||
+      workspace_bytes < netkv_schedule_workspace_size(R, D))
+    return NETKV_EINVAL;
+  if (R == 0)  // no request: the walk only reports out-of-range events and copies the loads
+    return netkv_schedule_streams(topo, n_streams, d_w, 0, d_len, d_prefill, d_snap, d_M,
+                                  nullptr, n_snap, d_events, d_event_off, d_load_init, d_dec,
+                                  d_best, d_second, d_load_final, nullptr, 0, d_status, stream);
+  float* d_base = reinterpret_cast<float*>(d_workspace);
+#define NETKV_SCHED_U(NPT, BLOCK, LPS)                                                           \
+  return launch<NPT, BLOCK, LPS, true>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,     \
+                                       d_util, n_snap, d_events, d_event_off, d_load_init,      \
+                                       d_dec, d_best, d_second, d_load_final, d_base, d_status, s)
+  if (D <= 8) NETKV_SCHED_U(1, 32, 8);
+  if (D <= 16) NETKV_SCHED_U(1, 32, 16);
+  if (D <= 32) NETKV_SCHED_U(1, 32, 32);
+  if (D <= 256) NETKV_SCHED_U(1, 256, 32);
+  if (D <= 1024) NETKV_SCHED_U(4, 256, 32);
+  if (D <= 4096) NETKV_SCHED_U(4, 1024, 32);
+#undef NETKV_SCHED_U
   return NETKV_EINVAL;
 }
 

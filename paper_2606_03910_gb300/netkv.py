@@ -35,9 +35,12 @@ EXPORTS = ("netkv_topology_create", "netkv_topology_destroy", "netkv_topology_qu
            "netkv_cache_build",
            "netkv_prefix_match_workspace_size",
            "netkv_prefix_match", "netkv_prefix_match_static", "netkv_schedule_workspace_size",
-           "netkv_schedule_streams", "netkv_schedule_streams_inflight",
+           "netkv_schedule_streams", "netkv_schedule_streams_util",
+           "netkv_schedule_streams_inflight",
            "netkv_schedule_inflight_workspace_size",
            "netkv_schedule_streams_load",
+           "netkv_lru_state_bytes", "netkv_lru_init", "netkv_lru_export",
+           "netkv_schedule_streams_evolving",
            "netkv_copy_async", "netkv_version")
 
 
@@ -79,6 +82,8 @@ _lib.netkv_schedule_workspace_size.argtypes = [_U32, _U32]
 _lib.netkv_schedule_workspace_size.restype = C.c_size_t
 _lib.netkv_schedule_streams.argtypes = [_P, _U32, _P, _U32, _P, _P, _P, _P, _P, _U32, _P, _P,
                                         _P, _P, _P, _P, _P, _P, C.c_size_t, _P, _P]
+_lib.netkv_schedule_streams_util.argtypes = [_P, _U32, _P, _U32, _P, _P, _P, _P, _P, _U32, _P,
+                                             _P, _P, _P, _P, _P, _P, _P, C.c_size_t, _P, _P]
 _lib.netkv_schedule_streams_inflight.argtypes = [_P, _U32, _P, _U32, _P, _P, _P, _P, _P, _P,
                                                  _U32, _P, _P, _U32, _P, _P, _P, _P, _P, _P,
                                                  _P, C.c_size_t, _P, _P]
@@ -93,10 +98,35 @@ class LoadModel(C.Structure):
 _lib.netkv_schedule_streams_load.argtypes = [_P, _U32, _P, C.POINTER(LoadModel), _U32, _P, _P,
                                              _P, _P, _P, _U32, _P, _P, _P, _P, _P, _P, _P, _P,
                                              _P, _P, _P]
+class LruConfig(C.Structure):
+    """netkv_lru_config: capacity and table sizes of the evolving (LRU) decode caches."""
+    _fields_ = [("cap_blocks", C.c_uint64), ("log2_slots", C.c_uint32), ("log2_ring", C.c_uint32)]
+
+
+def lru_config(cap_blocks: int) -> LruConfig:
+    """The smallest tables netkv.h allows for caches of cap_blocks blocks."""
+    need = int(cap_blocks) + 65536
+    ls = 4
+    while (3 << ls) // 4 < need - 1:
+        ls += 1
+    lr = 4
+    while (1 << lr) < need:
+        lr += 1
+    return LruConfig(int(cap_blocks), ls, lr)
+
+
+_lib.netkv_lru_state_bytes.argtypes = [_U64, C.POINTER(LruConfig)]
+_lib.netkv_lru_state_bytes.restype = C.c_size_t
+_lib.netkv_lru_init.argtypes = [_P, C.c_size_t, _U64, C.POINTER(LruConfig), _P, _P, _P, _P]
+_lib.netkv_lru_export.argtypes = [_P, C.c_size_t, _U64, C.POINTER(LruConfig), _P, _P, _P, _P]
+_lib.netkv_schedule_streams_evolving.argtypes = [_P, _U32, _P, _U32, _P, _P, _P, _P, _U32, _P, _P,
+                                                 _P, _P, _P, C.c_size_t, C.POINTER(LruConfig), _P,
+                                                 _P, _P, _P, _P, _P, _P, _P]
 _lib.netkv_copy_async.argtypes = [_P, _P, C.c_size_t, _P]
 for _f in EXPORTS:
     if _f not in ("netkv_version", "netkv_prefix_match_workspace_size", "netkv_cache_index_bytes",
-                  "netkv_schedule_workspace_size", "netkv_schedule_inflight_workspace_size"):
+                  "netkv_schedule_workspace_size", "netkv_schedule_inflight_workspace_size",
+                  "netkv_lru_state_bytes"):
         getattr(_lib, _f).restype = C.c_int
 
 
@@ -226,6 +256,19 @@ def netkv_schedule_streams(topo: Topology, n_streams: int, weights, R: int, leng
         ws_bytes, _ptr(status), _stream(stream)))
 
 
+def netkv_schedule_streams_util(topo: Topology, n_streams: int, weights, R: int, length, prefill,
+                                snap, M, util, n_snap: int, events, event_off, load_init, dec,
+                                best, second, load_final, status=None, stream=None,
+                                workspace=None) -> None:
+    """The greedy with level bottlenecks from the utilisation rows; see include/netkv.h."""
+    ws_bytes = 0 if workspace is None else int(workspace.numel() * workspace.element_size())
+    _check("netkv_schedule_streams_util", _lib.netkv_schedule_streams_util(
+        topo.handle, int(n_streams), _ptr(weights), int(R), _ptr(length), _ptr(prefill),
+        _ptr(snap), _ptr(M), _ptr(util), int(n_snap), _ptr(events), _ptr(event_off),
+        _ptr(load_init), _ptr(dec), _ptr(best), _ptr(second), _ptr(load_final), _ptr(workspace),
+        ws_bytes, _ptr(status), _stream(stream)))
+
+
 def netkv_schedule_streams_inflight(topo: Topology, n_streams: int, weights, R: int, length,
                                     prefill, snap, arrival_us, M, UB, n_snap: int, events,
                                     event_off, inflight_cap: int, load_init, dec, best, second,
@@ -271,6 +314,43 @@ def netkv_schedule_streams_load(topo: Topology, n_streams: int, weights, model: 
         _ptr(prefill), _ptr(snap), _ptr(M), _ptr(UB), int(n_snap), _ptr(events), _ptr(event_off),
         _ptr(m_init), _ptr(n_init), _ptr(dec), _ptr(best), _ptr(second), _ptr(m_final),
         _ptr(n_final), _ptr(status), _stream(stream)))
+
+
+def netkv_lru_state_bytes(n_caches: int, cfg: LruConfig) -> int:
+    return int(_lib.netkv_lru_state_bytes(int(n_caches), C.byref(cfg)))
+
+
+def _nbytes(t) -> int:
+    return int(t.numel() * t.element_size())
+
+
+def netkv_lru_init(state, n_caches: int, cfg: LruConfig, keys, key_off, status=None,
+                   stream=None) -> None:
+    """Evolving caches from key lists (most recently used first); see include/netkv.h."""
+    _check("netkv_lru_init", _lib.netkv_lru_init(_ptr(state), _nbytes(state), int(n_caches),
+                                                 C.byref(cfg), _ptr(keys), _ptr(key_off),
+                                                 _ptr(status), _stream(stream)))
+
+
+def netkv_lru_export(state, n_caches: int, cfg: LruConfig, keys_out, len_out, status=None,
+                     stream=None) -> None:
+    """Every evolving cache's blocks, most recently used first; see include/netkv.h."""
+    _check("netkv_lru_export", _lib.netkv_lru_export(_ptr(state), _nbytes(state), int(n_caches),
+                                                     C.byref(cfg), _ptr(keys_out), _ptr(len_out),
+                                                     _ptr(status), _stream(stream)))
+
+
+def netkv_schedule_streams_evolving(topo: Topology, n_streams: int, weights, R: int, length,
+                                    prefill, snap, UB, n_snap: int, chains, chain_off, events,
+                                    event_off, state, cfg: LruConfig, load_init, dec, best,
+                                    second, M, load_final, status=None, stream=None) -> None:
+    """Algorithm 1 with evolving LRU caches; see include/netkv.h."""
+    _check("netkv_schedule_streams_evolving", _lib.netkv_schedule_streams_evolving(
+        topo.handle, int(n_streams), _ptr(weights), int(R), _ptr(length), _ptr(prefill),
+        _ptr(snap), _ptr(UB), int(n_snap), _ptr(chains), _ptr(chain_off), _ptr(events),
+        _ptr(event_off), _ptr(state), _nbytes(state), C.byref(cfg), _ptr(load_init), _ptr(dec),
+        _ptr(best),
+        _ptr(second), _ptr(M), _ptr(load_final), _ptr(status), _stream(stream)))
 
 
 def netkv_copy_async(dst, src, nbytes: int, stream=None) -> None:

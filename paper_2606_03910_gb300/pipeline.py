@@ -10,6 +10,10 @@ CUDA stream:
 3. ``netkv_schedule_streams`` -> decisions, best/second scores, final loads
    (``netkv_schedule_streams_inflight`` when ``inflight_cap`` > 0: self-contention)
 
+With evolving caches (``lru_setup``), steps 2 and 3 are one call,
+``netkv_schedule_streams_evolving``: prefix hits are taken inside the greedy against
+LRU-managed caches that every dispatch updates (``lru_reset`` sets them from key lists).
+
 ``step_host`` is the same step from host buffers: it copies the step's inputs
 host->device (``netkv_copy_async``: SM-driven reads of pinned host memory), runs
 the step and copies the results back, all on the stream.
@@ -74,9 +78,11 @@ class StepOutputs:
 
 class Scorer:
     def __init__(self, fanout, role, tier_bw, tier_lat, n_links: int, n_sets: int,
-                 log2_capacity: int, device="cuda", share_prefixes: bool = True):
+                 log2_capacity: int, device="cuda", share_prefixes: bool = True,
+                 index: bool = True):
         """log2_capacity: slots per cache-index table (one table per table set and group
-        of 64 decodes); see netkv.index_log2_capacity."""
+        of 64 decodes); see netkv.index_log2_capacity.  index=False: no static cache index
+        (a scorer of evolving caches only)."""
         self.device = torch.device(device)
         self.topo = netkv.netkv_topology_create(fanout, role, tier_bw, tier_lat, n_links)
         self.N, self.P, self.D, self.used_links = netkv.netkv_topology_query(self.topo)
@@ -84,7 +90,8 @@ class Scorer:
         self.n_sets = int(n_sets)
         self.log2_capacity = int(log2_capacity)
         nbytes = netkv.netkv_cache_index_bytes(self.n_sets, self.D, self.log2_capacity)
-        self.index = torch.empty(nbytes // 8, dtype=torch.int64, device=self.device)
+        self.index = (torch.empty(nbytes // 8, dtype=torch.int64, device=self.device) if index
+                      else None)
         self.status = torch.zeros(1, dtype=torch.int32, device=self.device)
         self.share_prefixes = share_prefixes
         self.workspace = None
@@ -98,6 +105,39 @@ class Scorer:
         # the paper's compute-load model (netkv.LoadModel) instead of the token load;
         # out.load_final then holds free bytes and out.held_final request counts
         self.load_model = None
+        # level bottlenecks from the utilisation rows inside the base-score pass
+        # (netkv_schedule_streams_util): the step skips netkv_oracle_build and out.UB is
+        # not written.  Used by the plain greedy with the base-score workspace only.
+        self.fuse_level_bottlenecks = False
+        # evolving LRU caches (netkv.LruConfig) and their state, one cache per
+        # (stream, decode); None: the static caches of the index
+        self.lru_cfg = None
+        self.lru_state = None
+        self.lru_caches = 0
+
+    # ---- evolving caches
+    def lru_setup(self, n_streams: int, cap_blocks: int) -> None:
+        """State for the evolving caches of n_streams streams of cap_blocks blocks each."""
+        self.lru_cfg = netkv.lru_config(cap_blocks)
+        self.lru_caches = int(n_streams) * self.D
+        nbytes = netkv.netkv_lru_state_bytes(self.lru_caches, self.lru_cfg)
+        self.lru_state = torch.empty(nbytes // 8, dtype=torch.int64, device=self.device)
+
+    def lru_reset(self, keys: torch.Tensor, key_off: torch.Tensor, stream=None,
+                  n_caches: Optional[int] = None) -> None:
+        """Every (stream, decode) cache from its key list, cache c = stream * D + decode,
+        most recently used block first (the first n_caches caches when given)."""
+        netkv.netkv_lru_init(self.lru_state, self.lru_caches if n_caches is None else n_caches,
+                             self.lru_cfg, keys, key_off, self.status, stream)
+
+    def lru_export(self, stream=None):
+        """Each cache's blocks, most recently used first: (keys [caches, cap], lengths)."""
+        cap = int(self.lru_cfg.cap_blocks)
+        keys = torch.empty((self.lru_caches, cap), dtype=torch.int64, device=self.device)
+        lens = torch.empty(self.lru_caches, dtype=torch.int64, device=self.device)
+        netkv.netkv_lru_export(self.lru_state, self.lru_caches, self.lru_cfg, keys, lens,
+                               self.status, stream)
+        return keys, lens
 
     def _sched_workspace(self, R: int):
         """Greedy workspace (base scores of every arrival), grown on demand."""
@@ -152,6 +192,16 @@ class Scorer:
             return
         netkv.netkv_oracle_build(self.topo, x.util, x.n_snap, 1.0, None, out.UB, out.status, stream)
 
+    def schedule_evolving(self, x: StepInputs, out: StepOutputs, stream=None, streams=None) -> None:
+        """Prefix hits and the greedy in one call, against the evolving caches; streams =
+        (j0, j1) runs streams j0 .. j1-1 on the caches of the state's first j1 - j0 streams."""
+        j0, j1 = (0, x.n_streams) if streams is None else streams
+        netkv.netkv_schedule_streams_evolving(
+            self.topo, j1 - j0, x.weights[32 * j0:], x.R, x.length, x.prefill, x.snap, out.UB,
+            x.n_snap, x.chains, x.chain_off, x.events, x.event_off[j0:], self.lru_state,
+            self.lru_cfg, None if x.load_init is None else x.load_init[j0:], out.dec, out.best,
+            out.second, out.M, out.load_final[j0:], out.status, stream)
+
     def prefix_match(self, x: StepInputs, out: StepOutputs, stream=None) -> None:
         netkv.netkv_prefix_match(self.index, self.D, self.log2_capacity, self.n_sets, x.chains,
                                  x.chain_off, x.R, x.set_off if self.n_sets > 1 else None, out.M,
@@ -171,13 +221,33 @@ class Scorer:
                 x.load_init, out.dec, out.best, out.second, out.xfer_us, out.load_final,
                 out.status, stream)  # the walk, not its scoring, bounds this form
             return
+        if self.fused(x):
+            netkv.netkv_schedule_streams_util(
+                self.topo, x.n_streams, x.weights, x.R, x.length, x.prefill, x.snap, out.M,
+                x.util, x.n_snap, x.events, x.event_off, x.load_init, out.dec, out.best,
+                out.second, out.load_final, out.status, stream,
+                workspace=self._sched_workspace(x.R))
+            return
         netkv.netkv_schedule_streams(self.topo, x.n_streams, x.weights, x.R, x.length, x.prefill,
                                      x.snap, out.M, out.UB, x.n_snap, x.events, x.event_off,
                                      x.load_init, out.dec, out.best, out.second, out.load_final,
                                      out.status, stream, workspace=self._sched_workspace(x.R))
 
+    def fused(self, x: StepInputs) -> bool:
+        """Whether the step takes the level bottlenecks from the utilisation rows."""
+        return (self.fuse_level_bottlenecks and self.precompute_scores and
+                self.oracle_mode == "links" and x.util_down is None and self.inflight_cap == 0
+                and self.load_model is None and self.lru_cfg is None)
+
     def step(self, x: StepInputs, out: StepOutputs, stream=None) -> StepOutputs:
+        if self.fused(x):
+            self.prefix_match(x, out, stream)
+            self.schedule(x, out, stream)
+            return out
         self.oracle_build(x, out, stream)
+        if self.lru_cfg is not None:
+            self.schedule_evolving(x, out, stream)
+            return out
         self.prefix_match(x, out, stream)
         self.schedule(x, out, stream)
         return out

@@ -1,8 +1,8 @@
 """Parity at the benchmark's full size and launch configuration.
 
 The 4,096-replica workload is set up exactly as bench.py sets it up (same
-generator, cache index sizing, workspace and kernels); one step runs through the
-public pipeline, and whole sampled streams (first, last and three random ones)
+generator, cache index sizing, workspace and kernels, level bottlenecks taken from the
+utilisation rows in the base-score pass); one step runs through the public pipeline, and whole sampled streams (first, last and three random ones)
 are checked against the CPU oracle: prefix hits and decisions bit-exact (near-ties
 replayed and counted), scores within 1e-5 relative, final loads exact, level
 bottlenecks within 1e-5.  A second step must reproduce the first bit for bit.
@@ -25,7 +25,10 @@ def fullsize():
     import bench
     dev = torch.device("cuda", 0)
     w, sc, x, out = bench.setup_replicas(4096, 0, dev)
+    sc.fuse_level_bottlenecks = True   # the bench's step: level bottlenecks in the base pass
+    assert sc.fused(x)
     sc.step(x, out)
+    sc.oracle_build(x, out)            # UB as well, for the level-bottleneck check
     torch.cuda.synchronize()
     yield w, sc, x, out
     del sc, x, out
@@ -66,7 +69,7 @@ def test_bench_workload_with_self_contention(fullsize):
     w, sc, x, out = fullsize
     x2 = dataclasses.replace(x, arrival_us=torch.from_numpy(w.arrival_us.astype(np.int64)).cuda())
     o = sc.alloc_outputs(x.n_snap, x.R, x.n_streams)
-    sc.inflight_cap = 16
+    sc.inflight_cap = 16               # not fused: the step builds UB for this walk
     try:
         sc.step(x2, o)
         torch.cuda.synchronize()
