@@ -53,6 +53,9 @@ def parse():
                          "from CUDA graphs (latency); sweep: the oracle-build sweep (1,000 "
                          "snapshots x 2,048 x 8,192 pairs); longctx, cluster: the long-"
                          "context and large-cluster steps")
+    ap.add_argument("--keys", type=int, default=0,
+                    help="cached blocks per decode (0 = the workload's own; smaller values give "
+                         "reduced cases for ncu captures)")
     ap.add_argument("--requests", type=int, default=0,
                     help="requests per stream (0 = the workload's own; smaller values give "
                          "the reduced cases that ncu captures run on)")
@@ -466,9 +469,10 @@ def run_reference_sweep(args, world):
     return 0
 
 
-def workload_spec(kind: str, streams: int, rank: int, requests: int = 0):
+def workload_spec(kind: str, streams: int, rank: int, requests: int = 0, keys: int = 0):
     """Generator spec of a bench workload; rank k takes its own seeds (weak scaling).
-    requests > 0 sets the requests per stream (reduced cases)."""
+    requests > 0 sets the requests per stream, keys > 0 the cached blocks per decode
+    (reduced cases)."""
     import synth
     if kind == "replicas":
         spec = synth.config1(streams)
@@ -486,6 +490,8 @@ def workload_spec(kind: str, streams: int, rank: int, requests: int = 0):
         raise ValueError(f"unknown workload {kind!r}")
     if requests:
         spec.requests_per_stream = int(requests)
+    if keys:
+        spec.n_keys = int(keys)
     return spec
 
 
@@ -564,7 +570,8 @@ def run_netkv(args):
     __graft_entry__.build()
     from paper_2606_03910_gb300.pipeline import StepInputs
 
-    w, sc, x, out = setup_workload(workload_spec(args.workload, args.streams, rank, args.requests), dev,
+    w, sc, x, out = setup_workload(workload_spec(args.workload, args.streams, rank, args.requests,
+                                                 args.keys), dev,
                                    args.table_batch, inflight=args.inflight > 0,
                                    directed=args.directed, tiers=args.tiers)
     sc.share_prefixes = not args.no_share

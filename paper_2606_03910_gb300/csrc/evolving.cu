@@ -11,20 +11,22 @@
 //   hash table    2^log2_slots slots {hash, latest position of the hash in the log}
 //   header        head (the oldest position still in the cache), tail (the next
 //                 position), live blocks, occupied slots
-// A block is cached iff its latest position is at least head, so
+// A block is cached iff its latest position is at least head, and a use zeroes the log
+// entry it supersedes, so the non-zero entries of the window [head, tail) are exactly the
+// cached blocks at their latest uses:
 //   lookup    one probe of the table and a comparison with head;
-//   use       append at tail and raise the slot's position (atomicMax, so a hash that
-//             occurs twice in a chain keeps its later use);
-//   evict     advance head past the oldest log entries that are their hash's latest
-//             position (stale entries are skipped), one per evicted block.
+//   use       append at tail, raise the slot's position (atomicMax, so a hash that occurs
+//             twice in a chain keeps its later use) and zero the superseded entry;
+//   evict     advance head past as many non-zero entries as blocks to evict (a coalesced
+//             scan of the log, no lookups).
 // The table keeps evicted hashes (with old positions) until the log or the table fills;
-// then the cache is rebuilt in place: the live entries are packed in order from head and
-// the table is rebuilt from them.
+// then the cache is rebuilt in place: the non-zero entries are packed in order from head
+// and the table is rebuilt from them.
 //
 // One CTA per stream walks the stream's events in order:
 //   departure  the lead thread returns the request's tokens to its decode's load;
-//   arrival    warps take decodes and find the first miss of the chain, 128 blocks a
-//              step (coalesced chain loads, four independent probes per lane); threads
+//   arrival    warps take decodes and find the first miss of the chain by following the
+//              runs the chain's blocks form in the log (32 blocks a step); threads
 //              take decodes and score them exactly as netkv_schedule_streams does without
 //              a workspace (base score + w_load * theta * load), then a block-wide
 //              (score, index) argmin; every thread then uses its share of the chain's
@@ -144,28 +146,81 @@ __device__ __forceinline__ uint32_t block_count(bool flag, uint32_t* warp_buf, u
   return before + in_warp;
 }
 
+// Record that log position p (already holding `key`) is the latest use of the key: raise
+// the slot's position and zero the superseded log entry, which is p itself when a later
+// use of the key in the same pass got there first, else the key's previous entry when it
+// lies in the log window [head, tail).  So the non-zero entries of the window are exactly
+// the cached blocks, each at its latest use.  Counts claimed slots and keys that were not
+// cached before.
+__device__ __forceinline__ void lru_use(LruSlot* T, unsigned long long* ring, const LruGeom& g,
+                                        unsigned long long key, unsigned long long p,
+                                        unsigned long long head, unsigned int* fresh_cnt,
+                                        unsigned int* live_cnt, int* status) {
+  const unsigned long long qmask = (1ull << g.log2_ring) - 1;
+  bool fresh;
+  LruSlot* slot = lru_claim(T, g.log2_slots, key, fresh, status);
+  if (!slot) {  // not indexed (a full table, flagged): the entry does not count as cached
+    ring[p & qmask] = 0ull;
+    return;
+  }
+  const unsigned long long old = atomicMax(&slot->pos, p);
+  if (fresh) atomicAdd(fresh_cnt, 1u);
+  if (old > p) {
+    ring[p & qmask] = 0ull;
+  } else if (old >= head) {
+    ring[old & qmask] = 0ull;
+  } else {
+    atomicAdd(live_cnt, 1u);
+  }
+}
+
 // Leading chain blocks cached in one cache: the first miss among blocks [0, n), found by
-// one warp 128 blocks a step.
-__device__ __forceinline__ uint32_t lru_match(const LruSlot* T, uint32_t ls,
-                                              unsigned long long head,
+// one warp.  The blocks of a chain that entered the cache together sit in the log as one
+// run in reverse order (block j at the run's start position minus j), so the warp looks a
+// block up in the table once and then compares 32 chain blocks with the 32 log entries
+// below its position per step (coalesced), looking up again only where chain and log part.
+// A log entry in the window that holds the block's hash is its latest use (the others
+// are zero), so a match there is a cached block.
+__device__ __forceinline__ uint32_t lru_match(const LruSlot* T, const unsigned long long* ring,
+                                              const LruGeom& g, unsigned long long head,
                                               const uint64_t* __restrict__ chain, uint32_t n,
                                               uint32_t lane, int* status) {
-  for (uint32_t base = 0; base < n; base += 128) {
-    bool hit[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const uint32_t j = base + 32u * u + lane;
-      const unsigned long long key = j < n ? __ldg(chain + j) : 0ull;
-      const unsigned long long pos = key ? lru_find(T, ls, key, status) : 0ull;
-      hit[u] = pos != 0ull && pos >= head;
+  const unsigned long long qmask = (1ull << g.log2_ring) - 1;
+  uint32_t p = 0;
+  unsigned long long rp = 0;  // log position of block p within the current run
+  bool in_run = false;
+  while (p < n) {
+    const bool looked_up = !in_run;
+    if (!in_run) {  // look block p up in the table
+      unsigned long long pos = 0ull;
+      if (lane == 0) {
+        const unsigned long long key = __ldg(chain + p);
+        if (key != 0ull) pos = lru_find(T, g.log2_slots, key, status);
+      }
+      pos = __shfl_sync(0xffffffffu, pos, 0);
+      if (pos == 0ull || pos < head) return p;  // absent or evicted
+      rp = pos;
+      in_run = true;
     }
-    uint32_t first = 0xffffffffu;
-#pragma unroll
-    for (int u = 3; u >= 0; --u) {
-      const uint32_t bad = __ballot_sync(0xffffffffu, !hit[u]);
-      if (bad) first = base + 32u * u + (uint32_t)(__ffs(bad) - 1);
+    const uint32_t j = p + lane;
+    bool same = false;
+    if (j < n && rp >= head && (unsigned long long)lane <= rp - head) {
+      const unsigned long long ck = __ldg(chain + j);
+      same = ck != 0ull && vload(ring + ((rp - lane) & qmask)) == ck;
     }
-    if (first != 0xffffffffu) return first < n ? first : n;
+    const uint32_t ok = __ballot_sync(0xffffffffu, same);
+    const uint32_t lead = ~ok ? (uint32_t)(__ffs(~ok) - 1) : 32u;
+    if (lead == 0) {
+      if (looked_up) {  // the table's latest position does not hold the hash: inconsistent
+        if (lane == 0) flag_status(status, NETKV_DEV_EFULL);
+        return p;
+      }
+      in_run = false;  // the run ended with the last step: look block p up
+      continue;
+    }
+    p += lead;
+    rp -= lead;
+    if (lead < 32) in_run = false;
   }
   return n;
 }
@@ -193,25 +248,21 @@ __device__ __forceinline__ void warp_take(float& b, uint32_t& i, float& s) {
   }
 }
 
-// Evict the `excess` least recently used blocks of cache c: advance head past that many
-// log entries that are their hash's latest position.  CTA-wide.
-__device__ void lru_evict(const LruSlot* T, const unsigned long long* ring, const LruGeom& g,
+// Evict the `excess` least recently used blocks of a cache: advance head past that many
+// non-zero log entries (a coalesced scan of the log).  CTA-wide.
+__device__ void lru_evict(const unsigned long long* ring, const LruGeom& g,
                           unsigned long long& head, unsigned long long tail,
                           unsigned long long excess, uint32_t* warp_buf,
                           unsigned long long* s_newhead, int* status) {
   const unsigned long long qmask = (1ull << g.log2_ring) - 1;
   unsigned long long p = head;
   while (excess > 0) {
-    if (p >= tail) {  // fewer live entries than the header counts: an inconsistent state
+    if (p >= tail) {  // fewer cached blocks than the header counts: an inconsistent state
       if (threadIdx.x == 0) flag_status(status, NETKV_DEV_EFULL);
       break;
     }
     const unsigned long long i = p + threadIdx.x;
-    bool live = false;
-    if (i < tail) {
-      const unsigned long long key = vload(ring + (i & qmask));
-      live = key != 0ull && lru_find(T, g.log2_slots, key, status) == i;
-    }
+    const bool live = i < tail && vload(ring + (i & qmask)) != 0ull;
     uint32_t total;
     const uint32_t before = block_count<kEvoBlock>(live, warp_buf, total);
     if ((unsigned long long)total >= excess) {
@@ -228,8 +279,9 @@ __device__ void lru_evict(const LruSlot* T, const unsigned long long* ring, cons
   head = p;
 }
 
-// Rebuild cache c in place: pack the live log entries in order from head, then clear the
-// table and insert them at their new positions.  Returns the live count.  CTA-wide.
+// Rebuild a cache in place: pack the non-zero log entries of [head, tail) in order from
+// head, then clear the table and insert them at their new positions.  Returns the number
+// kept (the cached blocks).  CTA-wide.
 template <int BLOCK>
 __device__ unsigned long long lru_rebuild(LruSlot* T, unsigned long long* ring, const LruGeom& g,
                                           unsigned long long head, unsigned long long tail,
@@ -238,16 +290,11 @@ __device__ unsigned long long lru_rebuild(LruSlot* T, unsigned long long* ring, 
   unsigned long long kept = 0;
   for (unsigned long long p = head; p < tail; p += BLOCK) {
     const unsigned long long i = p + threadIdx.x;
-    unsigned long long key = 0ull;
-    bool live = false;
-    if (i < tail) {
-      key = vload(ring + (i & qmask));
-      live = key != 0ull && lru_find(T, g.log2_slots, key, status) == i;
-    }
+    const unsigned long long key = i < tail ? vload(ring + (i & qmask)) : 0ull;
     uint32_t total;
-    const uint32_t before = block_count<BLOCK>(live, warp_buf, total);  // reads done
+    const uint32_t before = block_count<BLOCK>(key != 0ull, warp_buf, total);  // reads done
     // the write position never passes the entry's own: entries are only moved down
-    if (live) ring[(head + kept + before) & qmask] = key;
+    if (key != 0ull) ring[(head + kept + before) & qmask] = key;
     kept += total;
     __syncthreads();
   }
@@ -273,7 +320,7 @@ __global__ void __launch_bounds__(kLruBlock) lru_init_kernel(void* state, LruGeo
                                                             const uint64_t* __restrict__ keys,
                                                             const uint64_t* __restrict__ key_off,
                                                             int* status) {
-  __shared__ unsigned int s_fresh;
+  __shared__ unsigned int s_fresh, s_live;
   const unsigned long long qmask = (1ull << g.log2_ring) - 1;
   const unsigned long long n_slots = 1ull << g.log2_slots;
   for (uint64_t c = blockIdx.x; c < n_caches; c += gridDim.x) {
@@ -281,7 +328,10 @@ __global__ void __launch_bounds__(kLruBlock) lru_init_kernel(void* state, LruGeo
     unsigned long long* ring = lru_ring(state, g, c);
     for (unsigned long long s = threadIdx.x; s < n_slots; s += kLruBlock)
       reinterpret_cast<ulonglong2*>(T)[s] = make_ulonglong2(0ull, 0ull);
-    if (threadIdx.x == 0) s_fresh = 0;
+    if (threadIdx.x == 0) {
+      s_fresh = 0;
+      s_live = 0;
+    }
     __syncthreads();
     uint64_t beg = 0, K = 0;
     if (keys) {
@@ -299,24 +349,20 @@ __global__ void __launch_bounds__(kLruBlock) lru_init_kernel(void* state, LruGeo
     }
     for (uint64_t j = threadIdx.x; j < K; j += kLruBlock) {
       const unsigned long long key = __ldg(keys + beg + j);
-      const unsigned long long p = K - j;
-      ring[p & qmask] = key;
-      if (key == 0ull) {
-        flag_status(status, NETKV_DEV_EDOMAIN);
-        continue;
-      }
-      bool fresh;
-      LruSlot* slot = lru_claim(T, g.log2_slots, key, fresh, status);
-      if (!slot) continue;
-      atomicMax(&slot->pos, p);
-      if (fresh) atomicAdd(&s_fresh, 1u);
+      ring[(K - j) & qmask] = key;
+      if (key == 0ull) flag_status(status, NETKV_DEV_EDOMAIN);
+    }
+    __syncthreads();  // every entry is written before any is zeroed as superseded
+    for (uint64_t j = threadIdx.x; j < K; j += kLruBlock) {
+      const unsigned long long key = __ldg(keys + beg + j);
+      if (key != 0ull) lru_use(T, ring, g, key, K - j, 1ull, &s_fresh, &s_live, status);
     }
     __syncthreads();
     if (threadIdx.x == 0) {
       LruHeader* h = lru_header(state, g, c);
       h->head = 1;
       h->tail = K + 1;
-      h->live = s_fresh;
+      h->live = s_live;
       h->n_keys = s_fresh;
     }
     __syncthreads();
@@ -346,7 +392,7 @@ __global__ void __launch_bounds__(kLruBlock) lru_export_kernel(const void* state
       if (threadIdx.x < chunk) {
         const unsigned long long i = top - 1 - threadIdx.x;  // newest first
         key = vload(ring + (i & qmask));
-        live = key != 0ull && lru_find(T, g.log2_slots, key, status) == i;
+        live = key != 0ull;  // the window's non-zero entries are the cached blocks
       }
       uint32_t total;
       const uint32_t before = block_count<kLruBlock>(live, warp_buf, total);
@@ -441,8 +487,8 @@ __global__ void __launch_bounds__(kEvoBlock) evolving_kernel(
 
     // hits against the caches as they are now (Sec. III-B first-miss scan)
     for (uint32_t d = wid; d < D; d += kEvoWarps) {
-      const uint32_t m = lru_match(lru_slots(state, g, c0_cache + d), g.log2_slots, s_head[d],
-                                   chain, (uint32_t)n, lane, status);
+      const uint32_t m = lru_match(lru_slots(state, g, c0_cache + d), lru_ring(state, g, c0_cache + d),
+                                   g, s_head[d], chain, (uint32_t)n, lane, status);
       if (lane == 0) {
         s_m[d] = m;
         M[(uint64_t)r * D + d] = (uint16_t)m;
@@ -512,27 +558,22 @@ __global__ void __launch_bounds__(kEvoBlock) evolving_kernel(
       __syncthreads();
     }
     const unsigned long long P0 = s_tail[dstar], head = s_head[dstar];
+    for (uint64_t j = tid; j < n; j += kEvoBlock) {  // block j is used at P0 + n - 1 - j
+      const unsigned long long key = __ldg(chain + j);
+      ring[(P0 + (n - 1 - j)) & qmask] = key;
+      if (key == 0ull) flag_status(status, NETKV_DEV_EDOMAIN);
+    }
+    __syncthreads();  // every entry is written before any is zeroed as superseded
     for (uint64_t j = tid; j < n; j += kEvoBlock) {
       const unsigned long long key = __ldg(chain + j);
-      const unsigned long long p = P0 + (n - 1 - j);
-      ring[p & qmask] = key;
-      if (key == 0ull) {
-        flag_status(status, NETKV_DEV_EDOMAIN);
-        continue;
-      }
-      bool fresh;
-      LruSlot* slot = lru_claim(T, g.log2_slots, key, fresh, status);
-      if (!slot) continue;
-      const unsigned long long old = atomicMax(&slot->pos, p);
-      if (fresh) atomicAdd(&s_cnt[0], 1u);
-      if (old < head) atomicAdd(&s_cnt[1], 1u);  // not cached before this use
+      if (key != 0ull) lru_use(T, ring, g, key, P0 + (n - 1 - j), head, &s_cnt[0], &s_cnt[1], status);
     }
     __syncthreads();
     const unsigned long long tail = P0 + n;
     const unsigned long long live = s_live[dstar] + s_cnt[1];
     if (live > g.cap_blocks) {
       unsigned long long hd = head;
-      lru_evict(T, ring, g, hd, tail, live - g.cap_blocks, warp_buf, &s_newhead, status);
+      lru_evict(ring, g, hd, tail, live - g.cap_blocks, warp_buf, &s_newhead, status);
       __syncthreads();
       if (tid == 0) {
         s_head[dstar] = hd;
