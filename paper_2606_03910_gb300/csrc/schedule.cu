@@ -143,12 +143,15 @@ __device__ __forceinline__ float xfer_factor(const netkv_weights& w, uint32_t l,
   return s_eff / fminf(ub_p, ub_d);
 }
 
-// Base scores of every arrival: base[r][d] = base_score(...) for the stream's weights.
-// No dependence between events, so the events of a stream are split into contiguous
-// ranges over the segments (LPS lanes each) of grid.y blocks; each segment strides over
-// one row's decodes.  Departures and invalid events are skipped (the greedy reports them).
-// kUtil: `UB` holds the utilisation rows [n_snap][n_links] instead of the level
-// bottlenecks, and each candidate's bottlenecks are taken from its links' entries.
+// Base scores of every arrival (pools of at most 32 decodes): the events of a stream are
+// split into contiguous ranges over the segments (LPS lanes each) of grid.y blocks, and
+// lane sl of a segment owns decode sl.  As in base_wide_kernel, a lane keeps its decode's
+// quotients bytes_per_token / UB_d[k] for the current snapshot and each arrival divides
+// once per level for its prefill and once for 1 / l:
+//     base = w_net * (miss_tok * max(qp[tau], qd[tau]) + L_tau) + w_prefix * miss_tok * (1/l)
+// Departures and invalid events are skipped (the greedy reports them).  kUtil: `UB` holds
+// the utilisation rows [n_snap][n_links] instead of the level bottlenecks, and the
+// bottlenecks are taken from the links' entries.  X (self-contention) gets s_eff / Bbot.
 template <int LPS, bool kUtil = false>
 __global__ void __launch_bounds__(256, 8) base_kernel(
     TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
@@ -160,16 +163,22 @@ __global__ void __launch_bounds__(256, 8) base_kernel(
   constexpr uint32_t kSegs = 256 / LPS;
   const uint32_t seg = threadIdx.x / LPS, sl = threadIdx.x % LPS;
   const uint32_t D = t.D, N = t.N;
+  const bool mine = sl < D;  // D <= LPS: lane sl owns decode sl
   const float4 lat = make_float4(t.lat[0], t.lat[1], t.lat[2], t.lat[3]);
+  const uint32_t inst = mine ? __ldg(t.dec + sl) : 0u;
+  const uint4 ld = __ldg(t.links + inst);
   for (uint32_t stream = blockIdx.x; stream < n_streams; stream += gridDim.x) {
-    const netkv_weights w = W[stream];
+    const float w_net = W[stream].w_net, w_prefix = W[stream].w_prefix;
+    const float bpt = (float)W[stream].bytes_per_token;
     // each segment takes a contiguous range of the stream's events, so consecutive
-    // arrivals share their snapshot's level-bottleneck row in L1
+    // arrivals share their snapshot
     const uint64_t e0 = event_off[stream], e1 = event_off[stream + 1];
     const uint64_t n_seg = (uint64_t)gridDim.y * kSegs;
     const uint64_t span = (e1 - e0 + n_seg - 1) / n_seg;
     const uint64_t eb = e0 + ((uint64_t)blockIdx.y * kSegs + seg) * span;
     const uint64_t ee = min(e1, eb + span);
+    uint32_t cur_k = 0xffffffffu;
+    float4 qd = make_float4(0.f, 0.f, 0.f, 0.f);
     uint32_t next = eb < ee ? __ldg(events + eb) : 0u;
     for (uint64_t e = eb; e < ee; ++e) {
       const uint32_t code = next;
@@ -177,35 +186,51 @@ __global__ void __launch_bounds__(256, 8) base_kernel(
       const uint32_t r = code & 0x7fffffffu;
       if ((code >> 31) || r >= R) continue;
       const uint32_t l = __ldg(len + r), pr = __ldg(prefill + r), k = __ldg(snap + r);
-      if (pr >= t.P || k >= n_snap || l == 0) continue;
+      if (pr >= t.P || k >= n_snap || l == 0 || !mine) continue;
+      const uint32_t m = __ldg(M + (uint64_t)r * D + sl);
+      if (k != cur_k) {  // the decode's level bottlenecks of a new snapshot
+        cur_k = k;
+        const float4 ub = kUtil ? level_bottlenecks_of(t, UB + (uint64_t)k * t.n_links, ld, status)
+                                : __ldg(reinterpret_cast<const float4*>(UB) + (uint64_t)k * N + inst);
+        qd = make_float4(bpt / ub.x, bpt / ub.y, bpt / ub.z, bpt / ub.w);
+      }
       const uint32_t pinst = __ldg(t.pre + pr);
       const uint4 lp = __ldg(t.links + pinst);
-      const float* urow = UB + (uint64_t)k * t.n_links;
-      const float4 ubp = kUtil ? level_bottlenecks_of(t, urow, lp, status)
-                               : __ldg(reinterpret_cast<const float4*>(UB) + (uint64_t)k * N + pinst);
-      const float* ub_row = UB + (uint64_t)k * N * 4;
-      for (uint32_t d = sl; d < D; d += LPS) {
-        const uint4 ld = __ldg(t.links + __ldg(t.dec + d));
-        const int tau = tier_of(lp, ld);
-        const float ubd = kUtil ? pick4(level_bottlenecks_of(t, urow, ld, status), tau)
-                                : __ldg(ub_row + (uint64_t)ld.x * 4 + tau);
-        const uint32_t m = __ldg(M + (uint64_t)r * D + d);
-        base[(uint64_t)r * D + d] = base_score(w, l, m, pick4(ubp, tau), ubd, pick4(lat, tau), status);
-        if (X) X[(uint64_t)r * D + d] = xfer_factor(w, l, m, pick4(ubp, tau), ubd);
+      const int tau = tier_of(lp, ld);
+      const float ubp = kUtil ? pick4(level_bottlenecks_of(t, UB + (uint64_t)k * t.n_links, lp,
+                                                           status), tau)
+                              : __ldg(UB + ((uint64_t)k * N + pinst) * 4 + tau);
+      uint32_t lam = 16u * m;
+      if (m > l / 16u) {
+        flag_status(status, NETKV_DEV_EDOMAIN);
+        lam = lam < l ? lam : l;
       }
+      const float miss_tok = (float)(l - lam);
+      const float q = fmaxf(bpt / ubp, pick4(qd, tau));
+      const float T = __fmaf_rn(miss_tok, q, pick4(lat, tau));
+      base[(uint64_t)r * D + sl] = __fmaf_rn(w_net, T, w_prefix * (miss_tok * (1.0f / (float)l)));
+      if (X) X[(uint64_t)r * D + sl] = miss_tok * q;
     }
   }
 }
 
 // Base scores for pools of more than 32 decodes.  A block takes one chunk of 256 * NPT
-// decodes of one stream; each thread owns NPT consecutive decodes, whose links it loads
-// once, and walks the arrivals given to the block (every grid.y-th event of the stream).
-// An arrival's request fields and the thread's NPT prefix hits are loaded one arrival
-// ahead, so the per-arrival chain of dependent loads overlaps the previous arrival's
-// scoring; prefix hits are read 8 bytes and scores written 16 bytes at a time when the
-// rows allow it.  kUtil: as for base_kernel (UB holds the utilisation rows).
+// decodes of one stream and a contiguous range of its events; each thread owns NPT
+// consecutive decodes.  Arrivals in a range mostly share their telemetry snapshot, so a
+// thread keeps, for its decodes and the current snapshot, the quotients
+// qd[k] = bytes_per_token / UB_d[k] of every level k, and recomputes them only when the
+// snapshot changes; per arrival it divides once per level for the prefill,
+// qp[k] = bytes_per_token / UB_p[k], and once for 1 / l.  Division of positive operands is
+// monotone, so bytes_per_token / min(UB_p, UB_d) = max(qp, qd) exactly, and a candidate
+// costs a tier test, a max and three multiply-adds:
+//     base = w_net * (miss_tok * max(qp[tau], qd[tau]) + L_tau) + w_prefix * miss_tok * (1/l)
+// (two roundings more than dividing per candidate: a relative difference below 3e-7).
+// The next arrival's request fields and prefix hits are loaded one arrival ahead; hits are
+// read 8 bytes and scores written 16 bytes at a time when the rows allow it.
+// kUtil: as for base_kernel (UB holds the utilisation rows).  X (self-contention) keeps
+// the per-candidate division s_eff / Bbot.
 template <int NPT, bool kUtil = false>
-__global__ void __launch_bounds__(256) base_wide_kernel(
+__global__ void __launch_bounds__(256, 4) base_wide_kernel(
     TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
     const uint32_t* __restrict__ len, const uint32_t* __restrict__ prefill,
     const uint32_t* __restrict__ snap, const uint16_t* __restrict__ M,
@@ -222,13 +247,17 @@ __global__ void __launch_bounds__(256) base_wide_kernel(
   for (uint64_t sc = blockIdx.x; sc < (uint64_t)n_streams * n_chunks; sc += gridDim.x) {
     const uint32_t stream = (uint32_t)(sc / n_chunks);
     const uint32_t d0 = (uint32_t)(sc % n_chunks) * kChunk + threadIdx.x * NPT;
-    uint4 ld[NPT];
+    uint3 lt[NPT];     // level-1..3 links of each decode: its tier against a prefill
+    uint32_t inst[NPT];
 #pragma unroll
-    for (int j = 0; j < NPT; ++j)
-      ld[j] = d0 + j < D ? __ldg(t.links + __ldg(t.dec + d0 + j)) : make_uint4(0, 0, 0, 0);
+    for (int j = 0; j < NPT; ++j) {
+      inst[j] = d0 + j < D ? __ldg(t.dec + d0 + j) : 0u;
+      const uint4 l = __ldg(t.links + inst[j]);
+      lt[j] = make_uint3(l.y, l.z, l.w);
+    }
     const netkv_weights w = W[stream];
-    // a contiguous range of the stream's events, so that consecutive arrivals share
-    // their snapshot's level-bottleneck row in L1
+    const float bpt = (float)w.bytes_per_token;
+    // a contiguous range of the stream's events
     const uint64_t e0 = event_off[stream], e1 = event_off[stream + 1];
     const uint64_t span = (e1 - e0 + gridDim.y - 1) / gridDim.y;
     const uint64_t eb = e0 + blockIdx.y * span;
@@ -262,9 +291,14 @@ __global__ void __launch_bounds__(256) base_wide_kernel(
       }
     };
 
+    float4 qd[NPT];  // bytes_per_token / UB_d[k] of the current snapshot
+    uint32_t cur_k = kBad;
     uint32_t nr, nl = 0, npr = 0, nk = 0, nm[NPT];
 #pragma unroll
-    for (int j = 0; j < NPT; ++j) nm[j] = 0;
+    for (int j = 0; j < NPT; ++j) {
+      nm[j] = 0;
+      qd[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
     uint64_t e = eb;
     fields(e, nr, nl, npr, nk, nm);
     for (; e < ee; ++e) {
@@ -274,21 +308,40 @@ __global__ void __launch_bounds__(256) base_wide_kernel(
       for (int j = 0; j < NPT; ++j) m[j] = nm[j];
       fields(e + 1, nr, nl, npr, nk, nm);
       if (r == kBad) continue;
+      if (k != cur_k) {  // the decodes' level bottlenecks of a new snapshot
+        cur_k = k;
+        const float* urow = UB + (uint64_t)k * t.n_links;
+#pragma unroll
+        for (int j = 0; j < NPT; ++j) {
+          if (d0 + j < D) {
+            const float4 ub = kUtil
+                ? level_bottlenecks_of(t, urow, __ldg(t.links + inst[j]), status)
+                : __ldg(reinterpret_cast<const float4*>(UB) + (uint64_t)k * N + inst[j]);
+            qd[j] = make_float4(bpt / ub.x, bpt / ub.y, bpt / ub.z, bpt / ub.w);
+          }
+        }
+      }
       const uint32_t pinst = __ldg(t.pre + pr);
       const uint4 lp = __ldg(t.links + pinst);
-      const float* urow = UB + (uint64_t)k * t.n_links;
-      const float4 ubp = kUtil ? level_bottlenecks_of(t, urow, lp, status)
-                               : __ldg(reinterpret_cast<const float4*>(UB) + (uint64_t)k * N + pinst);
-      const float* ub_row = UB + (uint64_t)k * N * 4;
+      const float4 ubp = kUtil
+          ? level_bottlenecks_of(t, UB + (uint64_t)k * t.n_links, lp, status)
+          : __ldg(reinterpret_cast<const float4*>(UB) + (uint64_t)k * N + pinst);
+      const float4 qp = make_float4(bpt / ubp.x, bpt / ubp.y, bpt / ubp.z, bpt / ubp.w);
+      const float rl = 1.0f / (float)l;
       float out[NPT];
 #pragma unroll
       for (int j = 0; j < NPT; ++j) {
-        const int tau = tier_of(lp, ld[j]);
-        const float ubd = d0 + j >= D ? 1.0f
-                          : kUtil ? pick4(level_bottlenecks_of(t, urow, ld[j], status), tau)
-                                  : __ldg(ub_row + (uint64_t)ld[j].x * 4 + tau);
-        out[j] = base_score(w, l, m[j], pick4(ubp, tau), ubd, pick4(lat, tau), status);
-        if (X && d0 + j < D) X[(uint64_t)r * D + d0 + j] = xfer_factor(w, l, m[j], pick4(ubp, tau), ubd);
+        const int tau = (lp.y == lt[j].x) ? 0 : (lp.z == lt[j].y) ? 1 : (lp.w == lt[j].z) ? 2 : 3;
+        uint32_t lam = 16u * m[j];
+        if (m[j] > l / 16u) {
+          flag_status(status, NETKV_DEV_EDOMAIN);
+          lam = lam < l ? lam : l;
+        }
+        const float miss_tok = (float)(l - lam);
+        const float q = fmaxf(pick4(qp, tau), pick4(qd[j], tau));
+        const float T = __fmaf_rn(miss_tok, q, pick4(lat, tau));
+        out[j] = __fmaf_rn(w.w_net, T, w.w_prefix * (miss_tok * rl));
+        if (X && d0 + j < D) X[(uint64_t)r * D + d0 + j] = miss_tok * q;
       }
       float* brow = base + (uint64_t)r * D + d0;
       if (vec) {
