@@ -1,6 +1,6 @@
 // Layout of the decode-cache index (the block-level prefix caches K_d of Sec. III-B) and
-// its lookup, shared by the prefix match that builds and walks it and by the greedy with
-// evolving caches that reads it.
+// its lookup, used by the cache build and the prefix match.  (The greedy with evolving
+// caches keeps its own per-decode state and does not read this index.)
 //
 // The caches of a table set are indexed per group of up to 64 decodes:
 //   hash table  2^L open-addressing slots {hash, position in the run array};
