@@ -229,8 +229,8 @@ KERNEL_CODE = {
 #   oracle_build: bytes per snapshot of the oracle-build sweep
 MEASURED_TRAFFIC = {
     # 64 replicas (64,000 requests): group_insert 8.97 MB, group_resolve 9.11 MB,
-    # match_leaders 129.29 MB, match_kernel<members> 243.36 MB (read + write)
-    "prefix_match": {"code_sha256_16": "5bb5552e2265ced6", "bytes_per_unit": 390_734_080 / 64_000,
+    # match_leaders 129.31 MB, match_kernel<members> 243.13 MB (read + write)
+    "prefix_match": {"code_sha256_16": "25b21a15533a1bcf", "bytes_per_unit": 390_518_016 / 64_000,
                      "unit": "request", "captured": "64-replica case, one launch per kernel"},
     "oracle_build": {"code_sha256_16": "ed437e71560780e2", "bytes_per_unit": 67_155_930,
                      "unit": "snapshot", "captured": "1,000-snapshot sweep, one launch"},
