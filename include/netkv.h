@@ -274,12 +274,18 @@ typedef struct {
  *   d_best       [R] fp32 output: minimum score (+inf when rejected)
  *   d_second     [R] fp32 output: minimum over the other feasible candidates (+inf if none)
  *   d_load_final [n_streams][D] int64 output: loads after the last event
- *   d_workspace  NULL, or a device buffer of at least netkv_schedule_workspace_size(R, D)
- *                bytes, 256-byte aligned, owned by the caller and overwritten by the call.
+ *   d_workspace  NULL, or a device buffer, 256-byte aligned, owned by the caller and
+ *                overwritten by the call, of at least R * D * 4 bytes rounded up to 256.
  *                With a workspace the decision-independent part of every arrival's scores
  *                (w_net * T_xfer + w_prefix * miss) is computed first for all arrivals in
  *                parallel and the sequential walk only adds the load term; without one
- *                the walk computes every term itself.  Overlapping calls need distinct
+ *                the walk computes every term itself.  For pools of 1,025 .. 4,096 decodes
+ *                a workspace of netkv_schedule_workspace_size(R, D) bytes also holds, per
+ *                arrival and chunk of 1,024 decodes, the 32 smallest (base score, rank)
+ *                pairs and a bound on the rest: the walk then rescores only those and falls
+ *                back to the arrival's full row when the bound does not certify the argmin
+ *                (the same decisions and scores, bit for bit).  A workspace of only the
+ *                rows runs the walk over every candidate.  Overlapping calls need distinct
  *                workspaces.
  * Every request index must occur in at most one stream, and its departure after its
  * arrival.  Out-of-range indices set ERANGE and the event is skipped.  The topology
@@ -301,7 +307,8 @@ netkv_status netkv_schedule_streams(netkv_topology_t topo, uint32_t n_streams,
  * utilisations of the links of p and d in row k, with the arithmetic of netkv_oracle_build.
  * So the results equal those of netkv_oracle_build(d_UB) followed by
  * netkv_schedule_streams with a workspace, without writing UB.  The workspace is required
- * (EINVAL when NULL or smaller than netkv_schedule_workspace_size(R, D)); other arguments
+ * (EINVAL when NULL or smaller than R * D * 4 bytes rounded up to 256; the candidate lists
+ * need netkv_schedule_workspace_size(R, D), as for netkv_schedule_streams); other arguments
  * and errors as netkv_schedule_streams, plus EDOMAIN for a utilisation outside [0, 1). */
 netkv_status netkv_schedule_streams_util(
     netkv_topology_t topo, uint32_t n_streams, const netkv_weights* d_w, uint32_t R,

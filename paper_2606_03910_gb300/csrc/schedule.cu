@@ -19,6 +19,8 @@
 // shrinks to a load, a capacity test, one multiply-add and the argmin per candidate.
 #include <math.h>
 
+#include <type_traits>
+
 #include "score.cuh"
 
 namespace {
@@ -47,6 +49,29 @@ __device__ __forceinline__ void seg_argmin(float& b, uint32_t& i, float& s, uint
     const float s2 = __shfl_xor_sync(mask, s, o, LPS);
     combine(b, i, s, b2, i2, s2);
   }
+}
+
+// Order-preserving 32-bit keys of fp32 scores, so that warp-wide redux minima give the
+// (score, rank) argmin; kNoKey (above every float's key) stands for "no candidate".
+constexpr uint32_t kNoKey = 0xffffffffu;
+__device__ __forceinline__ uint32_t score_key(float x) {
+  const uint32_t u = __float_as_uint(__fadd_rn(x, 0.0f));  // -0 and +0 tie, as compared
+  return u ^ ((uint32_t)((int32_t)u >> 31) | 0x80000000u);
+}
+__device__ __forceinline__ float key_score(uint32_t k) {
+  if (k == kNoKey) return __int_as_float(0x7f800000);
+  return __uint_as_float(k ^ ((k >> 31) ? 0x80000000u : 0xffffffffu));
+}
+// Block-free argmin over the 32 lanes of a warp: (best key, its lowest rank, second key),
+// where a lane offers (key, rank, key of its own runner-up).
+__device__ __forceinline__ void warp_argmin_keys(uint32_t& key, uint32_t& rank, uint32_t& key2) {
+  const uint32_t bk = __reduce_min_sync(0xffffffffu, key);
+  const uint32_t br = __reduce_min_sync(0xffffffffu, key == bk ? rank : kNone);
+  // the winning lane offers its runner-up; every other lane its best
+  const uint32_t sk = __reduce_min_sync(0xffffffffu, (key == bk && rank == br) ? key2 : key);
+  key = bk;
+  rank = br;
+  key2 = sk;
 }
 
 // The paper's compute-load model (Sec. III-C, IV-B) as kernel parameters.
@@ -214,6 +239,139 @@ __global__ void __launch_bounds__(256, 8) base_kernel(
   }
 }
 
+// ---- candidate lists: a bound on every decode a walk need not rescore ----------------
+// The load term of a score is w_load * theta * load >= 0, so a decode's score is never below
+// its base score, and the fp32 score fma(w_load, theta * load, base) is monotone in both the
+// load and the base.  For each arrival and chunk of kListChunk decodes the base pass lists the
+// kListLen smallest (base, rank) pairs in that order and a bound (tau, tau_rank): every decode
+// of the chunk not listed has (base, rank) >= (tau, tau_rank).  A walk that knows a lower bound
+// L on every decode's current load then has, for every unlisted decode d,
+//     score(d) >= fma(w_load, theta * L, base(d)) >= fma(w_load, theta * L, tau) =: LB,
+// so the best listed (score, rank) is the argmin of all decodes when its score is below LB, or
+// equal to tau with a rank below tau_rank (with L >= 0, an unlisted decode scores at least its
+// base); the second-best listed score is the second-best of all when it is <= LB.  Otherwise
+// the walk rescans the arrival's full row.  The result is the full argmin in every case.
+//
+// Bound keys: score_key(tau), or kNoKey when every decode of the chunk is listed, or
+// kBoundInvalid (below every float's key) when the chunk cannot bound anything (a NaN score).
+constexpr int kListLen = 32;             // (rank, base) pairs listed per chunk
+constexpr uint32_t kListChunk = 1024;    // decodes per chunk: base_wide_kernel<4>'s block
+constexpr uint32_t kListMaxChunks = 4;   // pools of up to 4,096 decodes
+constexpr int kListLevels = 8;           // distinct base scores a block walks up per arrival
+constexpr uint32_t kBoundInvalid = 0u;
+
+// Per-level exchange of a block's warps, double-buffered by barrier phase.
+struct ListShared {
+  uint32_t cnt[2][8];  // pairs of the warp at the current key
+  uint32_t nxt[2][8];  // the warp's smallest key above it
+};
+
+// The chunk's list and bound for one arrival, by the whole block: walking up the distinct
+// keys of the chunk (at most kListLevels of them), the pairs of each key are listed in rank
+// order until kListLen are listed; the next pair is the bound.  Every warp first finds its
+// smallest key and how many of its pairs hold it, so that after one block barrier the
+// chunk's smallest key and its pairs are placed: when there are more than kListLen of them
+// (ties, the common case) that barrier is the only one.  Each further level costs one
+// barrier: every warp counts its pairs at the key and finds its smallest key above it, and
+// after the barrier each thread places its own pairs by the counts of the warps before it.
+// When the levels run out first, the bound is (next key, rank 0) or, with no key left, the
+// chunk is listed entirely (kNoKey).  k: the thread's NPT = 4 keys (kNoKey past D) of
+// decodes d0 .. d0 + 3 (lane-major within a warp, warps in rank order).  `phase` counts the
+// block's barrier phases (uniform).  NaN scores make the chunk's bound kBoundInvalid.
+__device__ __forceinline__ void block_levels(ListShared& S, uint32_t& phase, const uint32_t (&k)[4],
+                                             bool nan, uint32_t d0, uint2* __restrict__ out,
+                                             uint2* __restrict__ bound) {
+  const uint32_t tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+  const uint32_t below = (1u << lane) - 1u;
+  // pairs of this thread at key v placed from position base_pos (in rank order)
+  auto place = [&](uint32_t v, uint32_t base_pos) {
+    uint32_t pos = base_pos;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) pos += __popc(__ballot_sync(0xffffffffu, k[j] == v) & below);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      if (k[j] == v) {
+        if (pos < (uint32_t)kListLen)
+          out[pos] = make_uint2(d0 + j, __float_as_uint(key_score(v)));
+        else if (pos == (uint32_t)kListLen)
+          *bound = make_uint2(d0 + j, v);
+        ++pos;
+      }
+    }
+  };
+  // level 0: each warp's smallest key, its pairs at that key, and whether a score is NaN
+  {
+    const uint32_t m = __reduce_min_sync(0xffffffffu, min(min(k[0], k[1]), min(k[2], k[3])));
+    uint32_t c = 0;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) c += __popc(__ballot_sync(0xffffffffu, k[j] == m));
+    const bool bad = __any_sync(0xffffffffu, nan);
+    if (lane == 0) {
+      S.nxt[phase & 1][wid] = m;
+      S.cnt[phase & 1][wid] = c | (bad ? 0x80000000u : 0u);
+    }
+  }
+  __syncthreads();
+  uint32_t v, cum;
+  {
+    const uint32_t b = phase & 1;
+    const uint32_t mw = lane < 8 ? S.nxt[b][lane] : kNoKey;
+    const uint32_t cw = lane < 8 ? S.cnt[b][lane] : 0u;
+    ++phase;
+    if (__reduce_or_sync(0xffffffffu, cw & 0x80000000u)) {
+      if (tid < (uint32_t)kListLen) out[tid] = make_uint2(kNone, 0x7f800000u);
+      if (tid == 0) *bound = make_uint2(0u, kBoundInvalid);
+      return;
+    }
+    v = __reduce_min_sync(0xffffffffu, mw);
+    if (v == kNoKey) {  // no decode in the chunk
+      if (tid < (uint32_t)kListLen) out[tid] = make_uint2(kNone, 0x7f800000u);
+      if (tid == 0) *bound = make_uint2(kNone, kNoKey);
+      return;
+    }
+    const uint32_t c = mw == v ? cw : 0u;  // a warp whose smallest key is above v has none at v
+    const uint32_t off = __reduce_add_sync(0xffffffffu, lane < wid ? c : 0u);
+    cum = __reduce_add_sync(0xffffffffu, c);
+    place(v, off);
+  }
+  for (int lev = 1; lev < kListLevels && cum <= (uint32_t)kListLen; ++lev) {
+    // each warp's smallest key above v and its pairs at that key, as at level 0
+    const uint32_t b = phase & 1;
+    uint32_t m = kNoKey;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) m = min(m, k[j] > v ? k[j] : kNoKey);
+    m = __reduce_min_sync(0xffffffffu, m);
+    uint32_t c = 0;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) c += __popc(__ballot_sync(0xffffffffu, k[j] == m));
+    if (lane == 0) {
+      S.nxt[b][wid] = m;
+      S.cnt[b][wid] = c;
+    }
+    __syncthreads();
+    const uint32_t mw = lane < 8 ? S.nxt[b][lane] : kNoKey;
+    const uint32_t cw = lane < 8 ? S.cnt[b][lane] : 0u;
+    ++phase;
+    v = __reduce_min_sync(0xffffffffu, mw);
+    if (v == kNoKey) break;  // every pair is listed
+    const uint32_t cv = mw == v ? cw : 0u;
+    const uint32_t off = __reduce_add_sync(0xffffffffu, lane < wid ? cv : 0u);
+    const uint32_t total = __reduce_add_sync(0xffffffffu, cv);
+    place(v, cum + off);
+    cum += total;
+  }
+  if (cum <= (uint32_t)kListLen) {  // as many pairs as the list holds, or fewer
+    if (tid >= cum && tid < (uint32_t)kListLen) out[tid] = make_uint2(kNone, 0x7f800000u);
+    if (tid == 0) {
+      if (v == kNoKey) {
+        *bound = make_uint2(kNone, kNoKey);
+      } else {  // the levels ran out: every pair not listed has a key above v
+        *bound = make_uint2(0u, v + 1u);
+      }
+    }
+  }
+}
+
 // Base scores for pools of more than 32 decodes.  A block takes one chunk of 256 * NPT
 // decodes of one stream and a contiguous range of its events; each thread owns NPT
 // consecutive decodes.  Arrivals in a range mostly share their telemetry snapshot, so a
@@ -229,14 +387,20 @@ __global__ void __launch_bounds__(256, 8) base_kernel(
 // read 8 bytes and scores written 16 bytes at a time when the rows allow it.
 // kUtil: as for base_kernel (UB holds the utilisation rows).  X (self-contention) keeps
 // the per-candidate division s_eff / Bbot.
-template <int NPT, bool kUtil = false>
-__global__ void __launch_bounds__(256, 4) base_wide_kernel(
+// kList: the block also writes each arrival's candidate list and bound for its chunk
+// (lists[r][chunk][kListLen], bounds[r][chunk]) with block_levels.
+template <int NPT, bool kUtil = false, bool kList = false>
+__global__ void __launch_bounds__(256, kList ? 3 : 4) base_wide_kernel(
     TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
     const uint32_t* __restrict__ len, const uint32_t* __restrict__ prefill,
     const uint32_t* __restrict__ snap, const uint16_t* __restrict__ M,
     const float* __restrict__ UB, uint32_t n_snap, const uint32_t* __restrict__ events,
     const uint64_t* __restrict__ event_off, float* __restrict__ base, int* status,
-    float* __restrict__ X = nullptr) {
+    float* __restrict__ X = nullptr, uint2* __restrict__ lists = nullptr,
+    uint2* __restrict__ bounds = nullptr) {
+  static_assert(!kList || (NPT == 4 && 256u * NPT == kListChunk), "lists need 1,024-decode chunks");
+  __shared__ std::conditional_t<kList, ListShared, char> S;
+  uint32_t phase = 0;  // block barrier phases of the list selection (buffer parity)
   constexpr uint32_t kChunk = 256u * NPT;
   constexpr uint32_t kBad = 0xffffffffu;
   const uint32_t D = t.D, N = t.N;
@@ -350,6 +514,18 @@ __global__ void __launch_bounds__(256, 4) base_wide_kernel(
 #pragma unroll
         for (int j = 0; j < NPT; ++j)
           if (d0 + j < D) __stcs(brow + j, out[j]);
+      }
+      if constexpr (kList) {
+        uint32_t key[4];
+        bool nan = false;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const bool present = d0 + j < D;
+          key[j] = present ? score_key(out[j]) : kNoKey;
+          nan |= present && !(out[j] == out[j]);
+        }
+        const uint64_t slot = (uint64_t)r * n_chunks + (uint32_t)(sc % n_chunks);
+        block_levels(S, phase, key, nan, d0, lists + slot * kListLen, bounds + slot);
       }
     }
   }
@@ -815,6 +991,10 @@ __device__ __forceinline__ void cp_async4(void* smem, const void* gmem) {
   const unsigned sa = (unsigned)__cvta_generic_to_shared(smem);
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(sa), "l"(gmem) : "memory");
 }
+__device__ __forceinline__ void cp_async8(void* smem, const void* gmem) {
+  const unsigned sa = (unsigned)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;\n" ::"r"(sa), "l"(gmem) : "memory");
+}
 __device__ __forceinline__ void cp_async_commit() {
   asm volatile("cp.async.commit_group;\n" ::: "memory");
 }
@@ -824,29 +1004,6 @@ __device__ __forceinline__ void cp_async_wait() {
 }
 
 constexpr int kRing = 16;  // arrivals remembered per warp (>= STAGES + 1)
-
-// Order-preserving 32-bit keys of fp32 scores, so that warp-wide redux minima give the
-// (score, rank) argmin; kNoKey (above every float's key) stands for "no candidate".
-constexpr uint32_t kNoKey = 0xffffffffu;
-__device__ __forceinline__ uint32_t score_key(float x) {
-  const uint32_t u = __float_as_uint(__fadd_rn(x, 0.0f));  // -0 and +0 tie, as compared
-  return u ^ ((uint32_t)((int32_t)u >> 31) | 0x80000000u);
-}
-__device__ __forceinline__ float key_score(uint32_t k) {
-  if (k == kNoKey) return __int_as_float(0x7f800000);
-  return __uint_as_float(k ^ ((k >> 31) ? 0x80000000u : 0xffffffffu));
-}
-// Block-free argmin over the 32 lanes of a warp: (best key, its lowest rank, second key),
-// where a lane offers (key, rank, key of its own runner-up).
-__device__ __forceinline__ void warp_argmin_keys(uint32_t& key, uint32_t& rank, uint32_t& key2) {
-  const uint32_t bk = __reduce_min_sync(0xffffffffu, key);
-  const uint32_t br = __reduce_min_sync(0xffffffffu, key == bk ? rank : kNone);
-  // the winning lane offers its runner-up; every other lane its best
-  const uint32_t sk = __reduce_min_sync(0xffffffffu, (key == bk && rank == br) ? key2 : key);
-  key = bk;
-  rank = br;
-  key2 = sk;
-}
 
 template <int NPT, int BLOCK, int STAGES>
 __global__ void __launch_bounds__(BLOCK) schedule_staged_kernel(
@@ -1084,6 +1241,340 @@ __global__ void __launch_bounds__(BLOCK) schedule_staged_kernel(
   }
 }
 
+// ---- listed greedy: one warp per stream, candidate lists from the base pass ---------
+// The stream's per-decode state lives in shared memory: load[d] (active tokens) and
+// hl[d] = (headroom cap - load clamped to 32 bits, theta * load) for one 8-byte gather per
+// candidate.  An arrival rescores only its listed candidates (4 per lane: lane i takes
+// entries 4i .. 4i + 3, chunk i / 8) and checks the chunks' bounds against lmin, a lower
+// bound on every decode's load: exact at the start and after every full scan, lowered by
+// departures and left unchanged by dispatches (which only raise a load).  An arrival the
+// bounds do not certify is scanned in full from its base-score row, which also makes lmin
+// exact again.  Certification needs w_load >= 0 and theta >= 0; a stream with other
+// weights scans every arrival.
+// Events go in windows of 32, double-buffered.  A window's records (code, length, prefill
+// and snapshot, or for a departure the decision in global memory) and its arrivals' lists
+// are copied with cp.async one window ahead, the copies of a departure's decision after the
+// decisions of the window before were written back.  Before a window is walked, lane i
+// prepares its event i: an arrival's validity and the smallest of its chunks' bounds; a
+// departure's decision, taken from the window before when its arrival is there, or marked
+// as the slot of its arrival when that is earlier in the same window.  The arrival's
+// certification threshold LB is prepared too, from lmin as the window starts; should a
+// departure lower lmin during the window, the rest of the window computes it afresh.
+// Decisions and scores are kept in the window buffer and written back when the window
+// after starts.
+struct __align__(16) ListWindow {
+  uint4 rec[32];                                  // code, length, prefill | decision, snapshot
+  uint2 bnd[32][kListMaxChunks];                  // (tau rank, tau key) of each chunk
+  uint2 ent[32][kListMaxChunks * kListLen];       // (rank, base bits) of each chunk's list
+  int32_t wd[32];                                 // decisions of the window's arrivals
+  uint32_t wbk[32], wsk[32];                      // their best and second-best keys
+  uint32_t lb[32];                                // an arrival's LB key from the prepared lmin
+};
+constexpr uint32_t kInWindow = 0x40000000u;  // departure decision: the slot of its arrival
+
+// The full argmin of one arrival from its base-score row (the listed walk's fallback), and
+// the exact minimum load.  Kept out of line: the walk's fast path stays small.
+struct ScanResult {
+  uint32_t kb, bi, ks;  // best key, its rank, second-best key
+  int64_t lmin;         // the exact minimum load
+};
+__device__ __noinline__ ScanResult listed_full_scan(const float* __restrict__ row, uint32_t D,
+                                                    bool vec, uint32_t l, float w_load,
+                                                    const uint2* s_hl, const int64_t* s_load,
+                                                    uint32_t lane) {
+  float b = __int_as_float(0x7f800000), s2 = b;
+  uint32_t ci = kNone;
+  int64_t lm = INT64_MAX;
+  auto visit = [&](uint32_t d, float bs) {
+    const uint2 hl = s_hl[d];
+    const int64_t ld = s_load[d];
+    lm = ld < lm ? ld : lm;
+    if (l <= hl.x) {
+      const float sc = __fmaf_rn(w_load, __uint_as_float(hl.y), bs);
+      const bool take = ci == kNone || sc < b;
+      s2 = take ? b : fminf(s2, sc);
+      b = take ? sc : b;
+      ci = take ? d : ci;
+    }
+  };
+  if (vec) {
+#pragma unroll 4
+    for (uint32_t d = 4 * lane; d < D; d += 128) {
+      const float4 v = __ldcs(reinterpret_cast<const float4*>(row + d));
+      visit(d, v.x);
+      visit(d + 1, v.y);
+      visit(d + 2, v.z);
+      visit(d + 3, v.w);
+    }
+  } else {
+#pragma unroll 4
+    for (uint32_t d = lane; d < D; d += 32) visit(d, __ldcs(row + d));
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    const int64_t x = __shfl_xor_sync(0xffffffffu, lm, o);
+    lm = x < lm ? x : lm;
+  }
+  uint32_t kb = ci == kNone ? kNoKey : score_key(b), bi = ci, ks = score_key(s2);
+  warp_argmin_keys(kb, bi, ks);
+  return ScanResult{kb, bi, ks, lm};
+}
+
+__global__ void __launch_bounds__(32) schedule_listed_kernel(
+    TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
+    const float* __restrict__ base, const uint2* __restrict__ lists,
+    const uint2* __restrict__ bounds, const uint32_t* __restrict__ len,
+    const uint32_t* __restrict__ prefill, const uint32_t* __restrict__ snap, uint32_t n_snap,
+    const uint32_t* __restrict__ events, const uint64_t* __restrict__ event_off,
+    const int64_t* __restrict__ load_init, int32_t* dec, float* __restrict__ best,
+    float* __restrict__ second, int64_t* __restrict__ load_final, int* status) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  constexpr uint32_t kBad = 0xffffffffu;
+  const uint32_t lane = threadIdx.x;
+  const uint32_t stream = blockIdx.x;
+  if (stream >= n_streams) return;
+  const uint32_t D = t.D;
+  const uint32_t n_ch = (D + kListChunk - 1) / kListChunk;
+  const bool has_ent = lane < 8u * n_ch;
+  ListWindow* win = reinterpret_cast<ListWindow*>(smem_raw);  // [2]
+  int64_t* s_load = reinterpret_cast<int64_t*>(win + 2);
+  uint2* s_hl = reinterpret_cast<uint2*>(s_load + D);  // [D + 1]: s_hl[D] fits no request
+  const netkv_weights w = W[stream];
+  const bool listed = w.w_load >= 0.0f && w.theta_s_per_token >= 0.0f;
+  const bool vec = (D % 4u == 0) && ((reinterpret_cast<uintptr_t>(base) & 15u) == 0);
+
+  auto hl_of = [&](int64_t ld) -> uint2 {
+    const int64_t h = w.cap_tokens - ld;
+    const uint32_t hr = h <= 0 ? 0u : h >= 0xffffffffll ? 0xffffffffu : (uint32_t)h;
+    return make_uint2(hr, __float_as_uint(w.theta_s_per_token * (float)ld));
+  };
+  int64_t lmin = INT64_MAX;
+  for (uint32_t d = lane; d < D; d += 32) {
+    const int64_t ld = load_init ? load_init[(uint64_t)stream * D + d] : 0;
+    s_load[d] = ld;
+    s_hl[d] = hl_of(ld);
+    lmin = ld < lmin ? ld : lmin;
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    const int64_t x = __shfl_xor_sync(0xffffffffu, lmin, o);
+    lmin = x < lmin ? x : lmin;
+  }
+  float lt_min = w.theta_s_per_token * (float)lmin;
+  if (lane == 0) s_hl[D] = make_uint2(0u, 0u);
+  __syncwarp();
+
+  const uint64_t e0 = event_off[stream], e1 = event_off[stream + 1];
+  const uint64_t n_win = (e1 - e0 + 31) / 32;
+  auto codes_of = [&](uint64_t k) -> uint32_t {  // lane i: code of event i of window k
+    const uint64_t e = e0 + 32 * k + lane;
+    return e < e1 ? __ldg(events + e) : kBad;
+  };
+  // copies of window k (codes c) into buffer k & 1, as one cp.async group
+  auto issue = [&](uint64_t k, uint32_t c) {
+    ListWindow& wb = win[k & 1];
+    const uint32_t r = c & 0x7fffffffu;
+    const bool valid = c != kBad && r < R;
+    wb.rec[lane].x = c;
+    if (valid) {
+      cp_async4(&wb.rec[lane].y, len + r);
+      if (c >> 31) {
+        cp_async4(&wb.rec[lane].z, dec + r);
+      } else {
+        cp_async4(&wb.rec[lane].z, prefill + r);
+        cp_async4(&wb.rec[lane].w, snap + r);
+      }
+    }
+    uint32_t arr = __ballot_sync(0xffffffffu, valid && !(c >> 31));
+    while (arr) {
+      const uint32_t i = __ffs(arr) - 1;
+      arr &= arr - 1;
+      const uint64_t lo = (uint64_t)__shfl_sync(0xffffffffu, r, i) * n_ch;
+      if (has_ent) {
+        cp_async16(&wb.ent[i][4 * lane], lists + lo * kListLen + 4 * lane);
+        cp_async16(&wb.ent[i][4 * lane + 2], lists + lo * kListLen + 4 * lane + 2);
+      }
+      if (lane < n_ch) cp_async8(&wb.bnd[i][lane], bounds + lo + lane);
+    }
+    cp_async_commit();
+  };
+  // decisions and scores of window k's arrivals to global memory (lane i: event i)
+  auto write_back = [&](const ListWindow& wb) {
+    const uint32_t c = wb.rec[lane].x, r = c & 0x7fffffffu;
+    if (c != kBad && !(c >> 31) && r < R) {
+      dec[r] = wb.wd[lane];
+      best[r] = key_score(wb.wbk[lane]);
+      second[r] = key_score(wb.wsk[lane]);
+    }
+  };
+  // add `delta` tokens to decode dd (every lane computes the load, lane 0 stores it)
+  auto adjust = [&](uint32_t dd, int64_t delta) -> int64_t {
+    const int64_t ld = s_load[dd] + delta;
+    __syncwarp();
+    if (lane == 0) {
+      s_load[dd] = ld;
+      s_hl[dd] = hl_of(ld);
+    }
+    __syncwarp();
+    return ld;
+  };
+
+  uint32_t cn = codes_of(0);
+  if (n_win > 0) issue(0, cn);
+  cn = codes_of(1);
+  uint32_t prev_code = kBad;  // lane j: event j of the window before and its decision
+  int32_t prev_dec = -1;
+  for (uint64_t k = 0; k < n_win; ++k) {
+    if (k > 0) {  // the window before: remember its arrivals, write its results back
+      const ListWindow& pb = win[(k - 1) & 1];
+      prev_code = pb.rec[lane].x;
+      prev_dec = pb.wd[lane];
+      write_back(pb);
+    }
+    __syncwarp();  // every lane is done with buffer (k + 1) & 1
+    if (k + 1 < n_win) issue(k + 1, cn);
+    else cp_async_commit();
+    cn = codes_of(k + 2);
+    cp_async_wait<1>();  // window k's copies have landed
+    __syncwarp();
+    ListWindow& wb = win[k & 1];
+    const uint32_t n_ev = (uint32_t)min((uint64_t)32, e1 - e0 - 32 * k);
+    {  // lane i prepares event i
+      uint4 f = wb.rec[lane];
+      const uint32_t c = f.x, r = c & 0x7fffffffu;
+      // a departure's arrival in the window before, or earlier in this one (every lane
+      // takes part in the shuffles; a lane's r matches only an arrival's code)
+      int32_t dd = (int32_t)f.z;
+      for (uint32_t j = 0; j < 32; ++j) {
+        const uint32_t pc = __shfl_sync(0xffffffffu, prev_code, j);
+        const int32_t pd = __shfl_sync(0xffffffffu, prev_dec, j);
+        if (pc == r) dd = pd;
+      }
+      for (uint32_t j = 0; j < 32; ++j) {
+        const uint32_t cc = __shfl_sync(0xffffffffu, c, j);
+        if (j < lane && cc == r) dd = (int32_t)(kInWindow | j);
+      }
+      bool skip = true;  // out of range, or an invalid arrival (prepared here)
+      if (c == kBad) {
+      } else if (r >= R) {
+        flag_status(status, NETKV_DEV_ERANGE);
+      } else if (c >> 31) {
+        f.z = (uint32_t)dd;
+        skip = f.y == 0u;  // a zero-length request released nothing
+      } else {
+        const uint32_t l = f.y;
+        if (f.z < t.P && f.w < n_snap && l != 0) {
+          uint2 b = lane < 32 ? wb.bnd[lane][0] : make_uint2(kNone, kNoKey);
+          for (uint32_t ch = 1; ch < n_ch; ++ch) {
+            const uint2 x = wb.bnd[lane][ch];
+            if (x.y < b.y || (x.y == b.y && x.x < b.x)) b = x;
+          }
+          f.z = b.y;
+          f.w = b.x;
+          wb.lb[lane] = b.y == kNoKey || b.y == kBoundInvalid
+                            ? b.y
+                            : score_key(__fmaf_rn(w.w_load, lt_min, key_score(b.y)));
+          skip = false;
+        } else {
+          flag_status(status, l == 0 ? NETKV_DEV_EDOMAIN : NETKV_DEV_ERANGE);
+          wb.wd[lane] = -1;
+          wb.wbk[lane] = kNoKey;
+          wb.wsk[lane] = kNoKey;
+        }
+      }
+      if (skip) f.y = 0u;  // the walk skips events of length 0
+      wb.rec[lane] = f;
+    }
+    __syncwarp();
+    bool moved = false;  // lmin fell below the value the thresholds were prepared with
+    const bool tie_ok = lmin >= 0;
+    for (uint32_t i = 0; i < n_ev; ++i) {
+      const uint4 f = wb.rec[i];
+      const uint32_t l = f.y;
+      if (l == 0u) continue;  // out of range, an invalid arrival (prepared), or nothing to release
+      if (f.x >> 31) {  // departure: release the tokens of a dispatched request
+        int32_t dd = (int32_t)f.z;
+        if (dd >= 0 && ((uint32_t)dd & kInWindow)) dd = wb.wd[(uint32_t)dd & 31u];
+        if (dd >= 0 && (uint32_t)dd < D) {
+          const int64_t ld = adjust((uint32_t)dd, -(int64_t)l);
+          if (ld < lmin) {
+            lmin = ld;
+            lt_min = w.theta_s_per_token * (float)lmin;
+            moved = true;
+          }
+        }
+        continue;
+      }
+      // the listed candidates as (key << 32 | rank), infeasible ones all ones: the lane's
+      // best pair and second key by a two-level tree of 64-bit minima
+      uint32_t lk = kNoKey, li = kNone, lk2 = kNoKey;
+      if (has_ent) {
+        const uint4 e01 = *reinterpret_cast<const uint4*>(&wb.ent[i][4 * lane]);
+        const uint4 e23 = *reinterpret_cast<const uint4*>(&wb.ent[i][4 * lane + 2]);
+        const uint32_t dr[4] = {e01.x, e01.z, e23.x, e23.z};
+        const uint32_t bs[4] = {e01.y, e01.w, e23.y, e23.w};
+        unsigned long long pk[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const uint2 hl = s_hl[min(dr[j], D)];  // s_hl[D]: a sentinel no request fits
+          pk[j] = l <= hl.x
+              ? ((unsigned long long)score_key(__fmaf_rn(w.w_load, __uint_as_float(hl.y),
+                                                          __uint_as_float(bs[j]))) << 32) | dr[j]
+              : ~0ull;
+        }
+        const unsigned long long a = min(pk[0], pk[1]), a2 = max(pk[0], pk[1]);
+        const unsigned long long b = min(pk[2], pk[3]), b2 = max(pk[2], pk[3]);
+        const unsigned long long bp = min(a, b), sp = min(max(a, b), min(a2, b2));
+        lk = (uint32_t)(bp >> 32);
+        li = (uint32_t)bp;
+        lk2 = (uint32_t)(sp >> 32);
+      }
+      // (key, rank) argmin and second key: the rank and the second depend only on the key
+      uint32_t kb = __reduce_min_sync(0xffffffffu, lk);
+      uint32_t bi = __reduce_min_sync(0xffffffffu, lk == kb ? li : kNone);
+      const uint32_t ties = __popc(__ballot_sync(0xffffffffu, lk == kb));
+      const uint32_t ks_one = __reduce_min_sync(0xffffffffu, lk == kb ? lk2 : lk);
+      uint32_t ks = ties >= 2 ? kb : ks_one;
+      const uint32_t tk = f.z, ti = f.w;
+      bool cert = listed && tk != kBoundInvalid;
+      if (cert && tk != kNoKey) {
+        const uint32_t klb =
+            moved ? score_key(__fmaf_rn(w.w_load, lt_min, key_score(tk))) : wb.lb[i];
+        const bool tie = moved ? lmin >= 0 : tie_ok;
+        cert = (kb < klb || (kb == tk && tie && bi < ti)) && ks <= klb;
+      }
+      // the listed decision is taken at once; an arrival the bounds did not certify (rare)
+      // takes it back and is decided by the full scan
+      int32_t dstar = kb == kNoKey ? -1 : (int32_t)bi;
+      if (dstar >= 0) adjust((uint32_t)dstar, (int64_t)l);
+      if (lane == 0) {
+        wb.wd[i] = dstar;
+        wb.wbk[i] = kb;
+        wb.wsk[i] = ks;
+      }
+      if (!cert) {
+        if (dstar >= 0) adjust((uint32_t)dstar, -(int64_t)l);
+        const ScanResult sr = listed_full_scan(base + (uint64_t)(f.x & 0x7fffffffu) * D, D, vec,
+                                               l, w.w_load, s_hl, s_load, lane);
+        lmin = sr.lmin;
+        lt_min = w.theta_s_per_token * (float)lmin;
+        dstar = sr.kb == kNoKey ? -1 : (int32_t)sr.bi;
+        if (dstar >= 0) adjust((uint32_t)dstar, (int64_t)l);
+        if (lane == 0) {
+          wb.wd[i] = dstar;
+          wb.wbk[i] = sr.kb;
+          wb.wsk[i] = sr.ks;
+        }
+      }
+    }
+  }
+  __syncwarp();
+  if (n_win > 0) write_back(win[(n_win - 1) & 1]);
+  cp_async_wait<0>();
+  __syncwarp();
+  for (uint32_t d = lane; d < D; d += 32) load_final[(uint64_t)stream * D + d] = s_load[d];
+}
+
 constexpr int kStages = 8;
 constexpr uint32_t kHeapPerStream = 4096;       // pending completions, one stream per CTA
 constexpr uint32_t kHeapPerPackedStream = 256;  // pending completions, packed streams
@@ -1108,6 +1599,25 @@ netkv_status launch_staged(const TopoArgs& t, uint32_t n_streams, const netkv_we
   return netkv_launch_status();
 }
 
+// The listed walk: one warp per stream, its decode state in dynamic shared memory.
+netkv_status launch_listed(const TopoArgs& t, uint32_t n_streams, const netkv_weights* d_w,
+                           uint32_t R, const uint32_t* d_len, const uint32_t* d_prefill,
+                           const uint32_t* d_snap, uint32_t n_snap, const uint32_t* d_events,
+                           const uint64_t* d_event_off, const int64_t* d_load_init,
+                           int32_t* d_dec, float* d_best, float* d_second,
+                           int64_t* d_load_final, const float* d_base, const uint2* d_lists,
+                           const uint2* d_bounds, int* d_status, cudaStream_t s) {
+  const size_t smem = sizeof(ListWindow) * 2 + (size_t)t.D * (sizeof(int64_t) + sizeof(uint2)) +
+                      sizeof(uint2);
+  if (smem > 48u * 1024u)  // per device: set before every launch that needs it
+    NETKV_CUDA_TRY(cudaFuncSetAttribute(schedule_listed_kernel,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+  schedule_listed_kernel<<<n_streams, 32, smem, s>>>(
+      t, n_streams, d_w, R, d_base, d_lists, d_bounds, d_len, d_prefill, d_snap, n_snap,
+      d_events, d_event_off, d_load_init, d_dec, d_best, d_second, d_load_final, d_status);
+  return netkv_launch_status();
+}
+
 // The base-score pre-pass over every arrival (and, with d_X, the factor s_eff / Bbot that
 // self-contention scales).
 template <bool kUtil = false>
@@ -1115,7 +1625,8 @@ netkv_status launch_base(const TopoArgs& t, uint32_t n_streams, const netkv_weig
                          uint32_t R, const uint32_t* d_len, const uint32_t* d_prefill,
                          const uint32_t* d_snap, const uint16_t* d_M, const float* d_UB,
                          uint32_t n_snap, const uint32_t* d_events, const uint64_t* d_event_off,
-                         float* d_base, float* d_X, int* d_status, cudaStream_t s) {
+                         float* d_base, float* d_X, int* d_status, cudaStream_t s,
+                         uint2* d_lists = nullptr, uint2* d_bounds = nullptr) {
     const uint32_t D = t.D;
     const unsigned gy = n_streams >= 1024u ? 1u : (1024u + n_streams - 1) / n_streams;
     const dim3 bgrid(n_streams < (1u << 20) ? n_streams : (1u << 20), gy);
@@ -1142,6 +1653,10 @@ netkv_status launch_base(const TopoArgs& t, uint32_t n_streams, const netkv_weig
         base_wide_kernel<1, kUtil><<<dim3(wx, wy), 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill,
                                                          d_snap, d_M, d_UB, n_snap, d_events,
                                                          d_event_off, d_base, d_status, d_X);
+      else if (d_lists)
+        base_wide_kernel<4, kUtil, true><<<dim3(wx, wy), 256, 0, s>>>(
+            t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events,
+            d_event_off, d_base, d_status, d_X, d_lists, d_bounds);
       else
         base_wide_kernel<4, kUtil><<<dim3(wx, wy), 256, 0, s>>>(t, n_streams, d_w, R, d_len, d_prefill,
                                                          d_snap, d_M, d_UB, n_snap, d_events,
@@ -1156,13 +1671,20 @@ netkv_status launch(const TopoArgs& t, uint32_t n_streams, const netkv_weights* 
                     const uint16_t* d_M, const float* d_UB, uint32_t n_snap,
                     const uint32_t* d_events, const uint64_t* d_event_off,
                     const int64_t* d_load_init, int32_t* d_dec, float* d_best, float* d_second,
-                    int64_t* d_load_final, float* d_base, int* d_status, cudaStream_t s) {
+                    int64_t* d_load_final, float* d_base, int* d_status, cudaStream_t s,
+                    uint2* d_lists = nullptr, uint2* d_bounds = nullptr) {
   const uint32_t per_cta = LPS == 32 ? 1u : 32u / LPS;
   const unsigned grid = (n_streams + per_cta - 1) / per_cta;
   if (d_base) {
+    const bool lists = LPS == 32 && d_lists != nullptr;
     if (launch_base<kUtil>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M, d_UB, n_snap,
-                           d_events, d_event_off, d_base, nullptr, d_status, s) != NETKV_OK)
+                           d_events, d_event_off, d_base, nullptr, d_status, s,
+                           lists ? d_lists : nullptr, lists ? d_bounds : nullptr) != NETKV_OK)
       return NETKV_ECUDA;
+    if (lists)
+      return launch_listed(t, n_streams, d_w, R, d_len, d_prefill, d_snap, n_snap, d_events,
+                           d_event_off, d_load_init, d_dec, d_best, d_second, d_load_final,
+                           d_base, d_lists, d_bounds, d_status, s);
     if (LPS == 32) {
       // one CTA per stream: the walk is bound by each warp's chain of dependent
       // instructions per event; 16 warps (4 per scheduler) measured best on 4,096 decodes
@@ -1241,9 +1763,32 @@ netkv_status launch_inflight(const TopoArgs& t, uint32_t n_streams, const netkv_
 
 }  // namespace
 
+namespace {
+size_t round256(size_t b) { return (b + 255) / 256 * 256; }
+// the base-score rows [R][D], always part of a workspace
+size_t base_ws_bytes(uint32_t R, uint32_t D) { return round256((size_t)R * D * sizeof(float)); }
+// the candidate lists and bounds of pools of 1,025 .. 4,096 decodes (listed walk)
+uint32_t list_chunks(uint32_t D) {
+  return D > kListChunk && D <= kListMaxChunks * kListChunk ? (D + kListChunk - 1) / kListChunk : 0u;
+}
+size_t list_ws_bytes(uint32_t R, uint32_t D) {
+  const size_t nc = list_chunks(D);
+  return nc ? round256((size_t)R * nc * kListLen * sizeof(uint2)) + round256((size_t)R * nc * sizeof(uint2))
+            : 0;
+}
+// lists and bounds inside a workspace of `bytes` bytes, or nulls (the staged walk)
+void list_ws(void* ws, size_t bytes, uint32_t R, uint32_t D, uint2*& lists, uint2*& bounds) {
+  lists = bounds = nullptr;
+  if (!ws || R == 0 || list_ws_bytes(R, D) == 0 || bytes < base_ws_bytes(R, D) + list_ws_bytes(R, D))
+    return;
+  char* p = reinterpret_cast<char*>(ws) + base_ws_bytes(R, D);
+  lists = reinterpret_cast<uint2*>(p);
+  bounds = reinterpret_cast<uint2*>(p + round256((size_t)R * list_chunks(D) * kListLen * sizeof(uint2)));
+}
+}  // namespace
+
 extern "C" size_t netkv_schedule_workspace_size(uint32_t R, uint32_t D) {
-  const size_t b = (size_t)R * D * sizeof(float);
-  return (b + 255) / 256 * 256;
+  return base_ws_bytes(R, D) + list_ws_bytes(R, D);
 }
 
 extern "C" netkv_status netkv_schedule_streams(
@@ -1265,14 +1810,15 @@ extern "C" netkv_status netkv_schedule_streams(
   const TopoArgs t = topo_args(topo);
   const uint32_t D = t.D;
   cudaStream_t s = (cudaStream_t)stream;
-  if (d_workspace && (!aligned_to(d_workspace, 256) ||
-                      workspace_bytes < netkv_schedule_workspace_size(R, D)))
+  if (d_workspace && (!aligned_to(d_workspace, 256) || workspace_bytes < base_ws_bytes(R, D)))
     return NETKV_EINVAL;
   float* d_base = (d_workspace && R > 0) ? reinterpret_cast<float*>(d_workspace) : nullptr;
+  uint2 *d_lists, *d_bounds;
+  list_ws(d_base ? d_workspace : nullptr, workspace_bytes, R, D, d_lists, d_bounds);
 #define NETKV_SCHED(NPT, BLOCK, LPS)                                                             \
   return launch<NPT, BLOCK, LPS>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, \
                             d_events, d_event_off, d_load_init, d_dec, d_best, d_second,       \
-                            d_load_final, d_base, d_status, s)
+                            d_load_final, d_base, d_status, s, d_lists, d_bounds)
   if (D <= 8) NETKV_SCHED(1, 32, 8);
   if (D <= 16) NETKV_SCHED(1, 32, 16);
   if (D <= 32) NETKV_SCHED(1, 32, 32);
@@ -1305,18 +1851,20 @@ extern "C" netkv_status netkv_schedule_streams_util(
   const TopoArgs t = topo_args(topo);
   const uint32_t D = t.D;
   cudaStream_t s = (cudaStream_t)stream;
-  if (!d_workspace || !aligned_to(d_workspace, 256) ||
-      workspace_bytes < netkv_schedule_workspace_size(R, D))
+  if (!d_workspace || !aligned_to(d_workspace, 256) || workspace_bytes < base_ws_bytes(R, D))
     return NETKV_EINVAL;
   if (R == 0)  // no request: the walk only reports out-of-range events and copies the loads
     return netkv_schedule_streams(topo, n_streams, d_w, 0, d_len, d_prefill, d_snap, d_M,
                                   nullptr, n_snap, d_events, d_event_off, d_load_init, d_dec,
                                   d_best, d_second, d_load_final, nullptr, 0, d_status, stream);
   float* d_base = reinterpret_cast<float*>(d_workspace);
+  uint2 *d_lists, *d_bounds;
+  list_ws(d_workspace, workspace_bytes, R, D, d_lists, d_bounds);
 #define NETKV_SCHED_U(NPT, BLOCK, LPS)                                                           \
   return launch<NPT, BLOCK, LPS, true>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,     \
                                        d_util, n_snap, d_events, d_event_off, d_load_init,      \
-                                       d_dec, d_best, d_second, d_load_final, d_base, d_status, s)
+                                       d_dec, d_best, d_second, d_load_final, d_base, d_status, \
+                                       s, d_lists, d_bounds)
   if (D <= 8) NETKV_SCHED_U(1, 32, 8);
   if (D <= 16) NETKV_SCHED_U(1, 32, 16);
   if (D <= 32) NETKV_SCHED_U(1, 32, 32);
