@@ -281,8 +281,8 @@ typedef struct {
  *                parallel and the sequential walk only adds the load term; without one
  *                the walk computes every term itself.  For pools of 1,025 .. 4,096 decodes
  *                a workspace of netkv_schedule_workspace_size(R, D) bytes also holds, per
- *                arrival and chunk of 1,024 decodes, the 32 smallest (base score, rank)
- *                pairs and a bound on the rest: the walk then rescores only those and falls
+ *                arrival, the pool's 32 smallest (base score, rank) pairs and a bound on
+ *                the rest: the walk then rescores only those and falls
  *                back to the arrival's full row when the bound does not certify the argmin
  *                (the same decisions and scores, bit for bit).  A workspace of only the
  *                rows runs the walk over every candidate.  Overlapping calls need distinct

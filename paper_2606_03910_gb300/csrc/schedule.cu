@@ -242,9 +242,9 @@ __global__ void __launch_bounds__(256, 8) base_kernel(
 // ---- candidate lists: a bound on every decode a walk need not rescore ----------------
 // The load term of a score is w_load * theta * load >= 0, so a decode's score is never below
 // its base score, and the fp32 score fma(w_load, theta * load, base) is monotone in both the
-// load and the base.  For each arrival and chunk of kListChunk decodes the base pass lists the
-// kListLen smallest (base, rank) pairs in that order and a bound (tau, tau_rank): every decode
-// of the chunk not listed has (base, rank) >= (tau, tau_rank).  A walk that knows a lower bound
+// load and the base.  For each arrival the base pass lists the pool's kListLen smallest
+// (base, rank) pairs in that order and a bound (tau, tau_rank): every decode not listed has
+// (base, rank) >= (tau, tau_rank).  A walk that knows a lower bound
 // L on every decode's current load then has, for every unlisted decode d,
 //     score(d) >= fma(w_load, theta * L, base(d)) >= fma(w_load, theta * L, tau) =: LB,
 // so the best listed (score, rank) is the argmin of all decodes when its score is below LB, or
@@ -252,33 +252,40 @@ __global__ void __launch_bounds__(256, 8) base_kernel(
 // base); the second-best listed score is the second-best of all when it is <= LB.  Otherwise
 // the walk rescans the arrival's full row.  The result is the full argmin in every case.
 //
-// Bound keys: score_key(tau), or kNoKey when every decode of the chunk is listed, or
-// kBoundInvalid (below every float's key) when the chunk cannot bound anything (a NaN score).
-constexpr int kListLen = 32;             // (rank, base) pairs listed per chunk
-constexpr uint32_t kListChunk = 1024;    // decodes per chunk: base_wide_kernel<4>'s block
-constexpr uint32_t kListMaxChunks = 4;   // pools of up to 4,096 decodes
+// Bound keys: score_key(tau), or kNoKey when every decode of the pool is listed, or
+// kBoundInvalid (below every float's key) when the list cannot bound anything (a NaN score).
+constexpr int kListLen = 32;             // (rank, base) pairs listed per arrival: one a lane
+constexpr uint32_t kListChunk = 1024;    // decodes per base-pass block (256 threads, 4 each)
+constexpr uint32_t kListMinD = 1025;     // listed pools: 1,025 .. 4,096 decodes, whose
+constexpr uint32_t kListMaxD = 4096;     // 2 .. 4 chunk lists are merged into the pool's
+// The list arrays of a workspace (all null: the staged walk runs).
+struct ListWs {
+  uint2 *chunk_lists = nullptr, *chunk_bounds = nullptr, *lists = nullptr, *bounds = nullptr;
+};
 constexpr int kListLevels = 8;           // distinct base scores a block walks up per arrival
 constexpr uint32_t kBoundInvalid = 0u;
 
-// Per-level exchange of a block's warps, double-buffered by barrier phase.
+// Per-level exchange of a block's NW <= 32 warps, double-buffered by barrier phase.
+template <int NW>
 struct ListShared {
-  uint32_t cnt[2][8];  // pairs of the warp at the current key
-  uint32_t nxt[2][8];  // the warp's smallest key above it
+  uint32_t cnt[2][NW];  // pairs of the warp at the current key
+  uint32_t nxt[2][NW];  // the warp's smallest key above it
 };
 
-// The chunk's list and bound for one arrival, by the whole block: walking up the distinct
-// keys of the chunk (at most kListLevels of them), the pairs of each key are listed in rank
+// The pool's list and bound for one arrival, by the whole block: walking up the distinct
+// keys of the pool (at most kListLevels of them), the pairs of each key are listed in rank
 // order until kListLen are listed; the next pair is the bound.  Every warp first finds its
 // smallest key and how many of its pairs hold it, so that after one block barrier the
-// chunk's smallest key and its pairs are placed: when there are more than kListLen of them
+// pool's smallest key and its pairs are placed: when there are more than kListLen of them
 // (ties, the common case) that barrier is the only one.  Each further level costs one
 // barrier: every warp counts its pairs at the key and finds its smallest key above it, and
 // after the barrier each thread places its own pairs by the counts of the warps before it.
 // When the levels run out first, the bound is (next key, rank 0) or, with no key left, the
-// chunk is listed entirely (kNoKey).  k: the thread's NPT = 4 keys (kNoKey past D) of
+// pool is listed entirely (kNoKey).  k: the thread's NPT = 4 keys (kNoKey past D) of
 // decodes d0 .. d0 + 3 (lane-major within a warp, warps in rank order).  `phase` counts the
-// block's barrier phases (uniform).  NaN scores make the chunk's bound kBoundInvalid.
-__device__ __forceinline__ void block_levels(ListShared& S, uint32_t& phase, const uint32_t (&k)[4],
+// block's barrier phases (uniform).  NaN scores make the bound kBoundInvalid.
+template <int NW>
+__device__ __forceinline__ void block_levels(ListShared<NW>& S, uint32_t& phase, const uint32_t (&k)[4],
                                              bool nan, uint32_t d0, uint2* __restrict__ out,
                                              uint2* __restrict__ bound) {
   const uint32_t tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
@@ -315,8 +322,8 @@ __device__ __forceinline__ void block_levels(ListShared& S, uint32_t& phase, con
   uint32_t v, cum;
   {
     const uint32_t b = phase & 1;
-    const uint32_t mw = lane < 8 ? S.nxt[b][lane] : kNoKey;
-    const uint32_t cw = lane < 8 ? S.cnt[b][lane] : 0u;
+    const uint32_t mw = lane < (uint32_t)NW ? S.nxt[b][lane] : kNoKey;
+    const uint32_t cw = lane < (uint32_t)NW ? S.cnt[b][lane] : 0u;
     ++phase;
     if (__reduce_or_sync(0xffffffffu, cw & 0x80000000u)) {
       if (tid < (uint32_t)kListLen) out[tid] = make_uint2(kNone, 0x7f800000u);
@@ -324,7 +331,7 @@ __device__ __forceinline__ void block_levels(ListShared& S, uint32_t& phase, con
       return;
     }
     v = __reduce_min_sync(0xffffffffu, mw);
-    if (v == kNoKey) {  // no decode in the chunk
+    if (v == kNoKey) {  // no decode at all
       if (tid < (uint32_t)kListLen) out[tid] = make_uint2(kNone, 0x7f800000u);
       if (tid == 0) *bound = make_uint2(kNone, kNoKey);
       return;
@@ -349,8 +356,8 @@ __device__ __forceinline__ void block_levels(ListShared& S, uint32_t& phase, con
       S.cnt[b][wid] = c;
     }
     __syncthreads();
-    const uint32_t mw = lane < 8 ? S.nxt[b][lane] : kNoKey;
-    const uint32_t cw = lane < 8 ? S.cnt[b][lane] : 0u;
+    const uint32_t mw = lane < (uint32_t)NW ? S.nxt[b][lane] : kNoKey;
+    const uint32_t cw = lane < (uint32_t)NW ? S.cnt[b][lane] : 0u;
     ++phase;
     v = __reduce_min_sync(0xffffffffu, mw);
     if (v == kNoKey) break;  // every pair is listed
@@ -372,6 +379,86 @@ __device__ __forceinline__ void block_levels(ListShared& S, uint32_t& phase, con
   }
 }
 
+// The pool's list and bound from its chunks' (one warp per request).  Every chunk list is
+// sorted by (key, rank); in 64-bit form (key << 32 | rank) a chunk's list is its real pairs,
+// then all ones.  With B the smallest chunk bound, a pair x < B is the pool's
+// p-th smallest, p = the number of pairs below x in every chunk list (its own position in its
+// own list, a binary search by shuffles in the others'), and is listed when p < kListLen;
+// the pool's bound is the pair with p == kListLen if there is one, else B.  Requests whose
+// arrival the base pass skipped merge whatever their slots hold; the walk never reads them.
+__device__ __forceinline__ unsigned long long list_pair(uint2 e) {  // (rank, base bits)
+  return e.x == kNone ? ~0ull
+                      : ((unsigned long long)score_key(__uint_as_float(e.y)) << 32) | e.x;
+}
+__global__ void __launch_bounds__(256) merge_lists_kernel(
+    const uint2* __restrict__ chunk_lists, const uint2* __restrict__ chunk_bounds, uint32_t n_ch,
+    uint32_t R, uint2* __restrict__ lists, uint2* __restrict__ bounds) {
+  constexpr uint32_t kMaxCh = kListMaxD / kListChunk;
+  const uint32_t lane = threadIdx.x & 31;
+  const uint64_t n_warps = ((uint64_t)gridDim.x * blockDim.x) >> 5;
+  for (uint64_t r = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; r < R; r += n_warps) {
+    unsigned long long x[kMaxCh], bd[kMaxCh];
+    uint32_t xb[kMaxCh];
+    unsigned long long B = ~0ull;
+#pragma unroll
+    for (uint32_t c = 0; c < kMaxCh; ++c) {
+      x[c] = bd[c] = ~0ull;
+      xb[c] = 0x7f800000u;
+      if (c < n_ch) {
+        const uint2 e = __ldcs(chunk_lists + ((r * n_ch + c) * kListLen + lane));
+        const uint2 b = chunk_bounds[r * n_ch + c];
+        x[c] = list_pair(e);
+        xb[c] = e.y;
+        bd[c] = ((unsigned long long)b.y << 32) | b.x;
+        B = min(B, bd[c]);
+      }
+    }
+    uint2 mine = make_uint2(kNone, 0x7f800000u);
+    bool has_bound = false;  // some pair is the (kListLen + 1)-th below B
+    unsigned long long pb = 0;
+#pragma unroll
+    for (uint32_t c = 0; c < kMaxCh; ++c) {
+      const unsigned long long v = x[c];
+      uint32_t p = lane;  // pairs below v in its own list
+#pragma unroll
+      for (uint32_t o = 0; o < kMaxCh; ++o) {
+        if (o == c || o >= n_ch) continue;
+        uint32_t lo = 0;  // pairs of list o below v, by binary search over its 32 lanes
+#pragma unroll
+        for (uint32_t step = 16; step; step >>= 1) {
+          const unsigned long long u = __shfl_sync(0xffffffffu, x[o], lo + step - 1);
+          if (u < v) lo += step;
+        }
+        const unsigned long long u31 = __shfl_sync(0xffffffffu, x[o], 31);
+        if (lo == 31 && u31 < v) lo = 32;  // every pair of list o is below v
+        p += lo;
+      }
+      const bool real = c < n_ch && v < B && (uint32_t)(v & 0xffffffffu) != kNone;
+      // the real pair at lane `lane` sits at pool position p: list it or make it the bound
+      if (real && p < (uint32_t)kListLen) {
+        lists[r * kListLen + p] = make_uint2((uint32_t)v, xb[c]);
+      }
+      const bool is_b = real && p == (uint32_t)kListLen;
+      if (__any_sync(0xffffffffu, is_b)) {
+        const uint32_t src = __ffs(__ballot_sync(0xffffffffu, is_b)) - 1;
+        pb = __shfl_sync(0xffffffffu, v, src);
+        has_bound = true;
+      }
+    }
+    // how many pairs were listed: positions beyond them are empty
+    uint32_t n_listed = 0;
+#pragma unroll
+    for (uint32_t c = 0; c < kMaxCh; ++c)
+      n_listed += __popc(__ballot_sync(0xffffffffu, c < n_ch && x[c] < B &&
+                                                         (uint32_t)(x[c] & 0xffffffffu) != kNone));
+    if (lane >= n_listed) lists[r * kListLen + lane] = mine;
+    if (lane == 0) {
+      const unsigned long long b = has_bound ? pb : B;
+      bounds[r] = make_uint2((uint32_t)b, (uint32_t)(b >> 32));
+    }
+  }
+}
+
 // Base scores for pools of more than 32 decodes.  A block takes one chunk of 256 * NPT
 // decodes of one stream and a contiguous range of its events; each thread owns NPT
 // consecutive decodes.  Arrivals in a range mostly share their telemetry snapshot, so a
@@ -387,10 +474,11 @@ __device__ __forceinline__ void block_levels(ListShared& S, uint32_t& phase, con
 // read 8 bytes and scores written 16 bytes at a time when the rows allow it.
 // kUtil: as for base_kernel (UB holds the utilisation rows).  X (self-contention) keeps
 // the per-candidate division s_eff / Bbot.
-// kList: the block also writes each arrival's candidate list and bound for its chunk
-// (lists[r][chunk][kListLen], bounds[r][chunk]) with block_levels.
-template <int NPT, bool kUtil = false, bool kList = false>
-__global__ void __launch_bounds__(256, kList ? 3 : 4) base_wide_kernel(
+// kList: the block also writes each arrival's candidate list and bound for its chunk of
+// decodes (lists[r][chunk][kListLen], bounds[r][chunk]) with block_levels; merge_lists_kernel
+// then merges the chunks' lists into the pool's.
+template <int NPT, bool kUtil = false, bool kList = false, int BT = 256>
+__global__ void __launch_bounds__(BT, 1024 / BT) base_wide_kernel(
     TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
     const uint32_t* __restrict__ len, const uint32_t* __restrict__ prefill,
     const uint32_t* __restrict__ snap, const uint16_t* __restrict__ M,
@@ -398,10 +486,11 @@ __global__ void __launch_bounds__(256, kList ? 3 : 4) base_wide_kernel(
     const uint64_t* __restrict__ event_off, float* __restrict__ base, int* status,
     float* __restrict__ X = nullptr, uint2* __restrict__ lists = nullptr,
     uint2* __restrict__ bounds = nullptr) {
-  static_assert(!kList || (NPT == 4 && 256u * NPT == kListChunk), "lists need 1,024-decode chunks");
-  __shared__ std::conditional_t<kList, ListShared, char> S;
+  static_assert(!kList || NPT == 4, "lists take 4 decodes a thread");
+  static_assert(BT % 32 == 0 && BT <= 1024, "block of whole warps");
+  __shared__ std::conditional_t<kList, ListShared<BT / 32>, char> S;
   uint32_t phase = 0;  // block barrier phases of the list selection (buffer parity)
-  constexpr uint32_t kChunk = 256u * NPT;
+  constexpr uint32_t kChunk = (uint32_t)BT * NPT;
   constexpr uint32_t kBad = 0xffffffffu;
   const uint32_t D = t.D, N = t.N;
   const uint32_t n_chunks = (D + kChunk - 1) / kChunk;
@@ -1244,8 +1333,8 @@ __global__ void __launch_bounds__(BLOCK) schedule_staged_kernel(
 // ---- listed greedy: one warp per stream, candidate lists from the base pass ---------
 // The stream's per-decode state lives in shared memory: load[d] (active tokens) and
 // hl[d] = (headroom cap - load clamped to 32 bits, theta * load) for one 8-byte gather per
-// candidate.  An arrival rescores only its listed candidates (4 per lane: lane i takes
-// entries 4i .. 4i + 3, chunk i / 8) and checks the chunks' bounds against lmin, a lower
+// candidate.  An arrival rescores only its listed candidates (lane i takes entry i) and
+// checks the list's bound against lmin, a lower
 // bound on every decode's load: exact at the start and after every full scan, lowered by
 // departures and left unchanged by dispatches (which only raise a load).  An arrival the
 // bounds do not certify is scanned in full from its base-score row, which also makes lmin
@@ -1255,7 +1344,7 @@ __global__ void __launch_bounds__(BLOCK) schedule_staged_kernel(
 // and snapshot, or for a departure the decision in global memory) and its arrivals' lists
 // are copied with cp.async one window ahead, the copies of a departure's decision after the
 // decisions of the window before were written back.  Before a window is walked, lane i
-// prepares its event i: an arrival's validity and the smallest of its chunks' bounds; a
+// prepares its event i: an arrival's validity and its certification threshold; a
 // departure's decision, taken from the window before when its arrival is there, or marked
 // as the slot of its arrival when that is earlier in the same window.  The arrival's
 // certification threshold LB is prepared too, from lmin as the window starts; should a
@@ -1264,8 +1353,8 @@ __global__ void __launch_bounds__(BLOCK) schedule_staged_kernel(
 // after starts.
 struct __align__(16) ListWindow {
   uint4 rec[32];                                  // code, length, prefill | decision, snapshot
-  uint2 bnd[32][kListMaxChunks];                  // (tau rank, tau key) of each chunk
-  uint2 ent[32][kListMaxChunks * kListLen];       // (rank, base bits) of each chunk's list
+  uint2 bnd[32];                                  // (tau rank, tau key) of each arrival
+  uint2 ent[32][kListLen];                        // (rank, base bits): each arrival's list
   int32_t wd[32];                                 // decisions of the window's arrivals
   uint32_t wbk[32], wsk[32];                      // their best and second-best keys
   uint32_t lb[32];                                // an arrival's LB key from the prepared lmin
@@ -1334,8 +1423,6 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
   const uint32_t stream = blockIdx.x;
   if (stream >= n_streams) return;
   const uint32_t D = t.D;
-  const uint32_t n_ch = (D + kListChunk - 1) / kListChunk;
-  const bool has_ent = lane < 8u * n_ch;
   ListWindow* win = reinterpret_cast<ListWindow*>(smem_raw);  // [2]
   int64_t* s_load = reinterpret_cast<int64_t*>(win + 2);
   uint2* s_hl = reinterpret_cast<uint2*>(s_load + D);  // [D + 1]: s_hl[D] fits no request
@@ -1389,12 +1476,9 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
     while (arr) {
       const uint32_t i = __ffs(arr) - 1;
       arr &= arr - 1;
-      const uint64_t lo = (uint64_t)__shfl_sync(0xffffffffu, r, i) * n_ch;
-      if (has_ent) {
-        cp_async16(&wb.ent[i][4 * lane], lists + lo * kListLen + 4 * lane);
-        cp_async16(&wb.ent[i][4 * lane + 2], lists + lo * kListLen + 4 * lane + 2);
-      }
-      if (lane < n_ch) cp_async8(&wb.bnd[i][lane], bounds + lo + lane);
+      const uint64_t ri = __shfl_sync(0xffffffffu, r, i);
+      cp_async8(&wb.ent[i][lane], lists + ri * kListLen + lane);
+      if (lane == 0) cp_async8(&wb.bnd[i], bounds + ri);
     }
     cp_async_commit();
   };
@@ -1407,16 +1491,14 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
       second[r] = key_score(wb.wsk[lane]);
     }
   };
-  // add `delta` tokens to decode dd (every lane computes the load, lane 0 stores it)
-  auto adjust = [&](uint32_t dd, int64_t delta) -> int64_t {
-    const int64_t ld = s_load[dd] + delta;
-    __syncwarp();
+  // add `delta` tokens to decode dd (lane 0; dispatches never lower lmin)
+  auto adjust = [&](uint32_t dd, int64_t delta) {
     if (lane == 0) {
+      const int64_t ld = s_load[dd] + delta;
       s_load[dd] = ld;
       s_hl[dd] = hl_of(ld);
     }
     __syncwarp();
-    return ld;
   };
 
   uint32_t cn = codes_of(0);
@@ -1438,7 +1520,10 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
     cp_async_wait<1>();  // window k's copies have landed
     __syncwarp();
     ListWindow& wb = win[k & 1];
-    const uint32_t n_ev = (uint32_t)min((uint64_t)32, e1 - e0 - 32 * k);
+    bool my_dep = false;   // lane i: event i is a departure to apply: its length and decode
+    uint32_t my_l = 0;
+    int32_t my_dd = -1;
+    bool my_arr = false;   // event i is an arrival to decide
     {  // lane i prepares event i
       uint4 f = wb.rec[lane];
       const uint32_t c = f.x, r = c & 0x7fffffffu;
@@ -1454,27 +1539,23 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
         const uint32_t cc = __shfl_sync(0xffffffffu, c, j);
         if (j < lane && cc == r) dd = (int32_t)(kInWindow | j);
       }
-      bool skip = true;  // out of range, or an invalid arrival (prepared here)
       if (c == kBad) {
       } else if (r >= R) {
         flag_status(status, NETKV_DEV_ERANGE);
       } else if (c >> 31) {
-        f.z = (uint32_t)dd;
-        skip = f.y == 0u;  // a zero-length request released nothing
+        my_dep = f.y != 0u;  // a zero-length request released nothing
+        my_l = f.y;
+        my_dd = dd;
       } else {
         const uint32_t l = f.y;
         if (f.z < t.P && f.w < n_snap && l != 0) {
-          uint2 b = lane < 32 ? wb.bnd[lane][0] : make_uint2(kNone, kNoKey);
-          for (uint32_t ch = 1; ch < n_ch; ++ch) {
-            const uint2 x = wb.bnd[lane][ch];
-            if (x.y < b.y || (x.y == b.y && x.x < b.x)) b = x;
-          }
+          const uint2 b = wb.bnd[lane];
           f.z = b.y;
           f.w = b.x;
           wb.lb[lane] = b.y == kNoKey || b.y == kBoundInvalid
                             ? b.y
                             : score_key(__fmaf_rn(w.w_load, lt_min, key_score(b.y)));
-          skip = false;
+          my_arr = true;
         } else {
           flag_status(status, l == 0 ? NETKV_DEV_EDOMAIN : NETKV_DEV_ERANGE);
           wb.wd[lane] = -1;
@@ -1482,59 +1563,69 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
           wb.wsk[lane] = kNoKey;
         }
       }
-      if (skip) f.y = 0u;  // the walk skips events of length 0
       wb.rec[lane] = f;
     }
     __syncwarp();
     bool moved = false;  // lmin fell below the value the thresholds were prepared with
     const bool tie_ok = lmin >= 0;
-    for (uint32_t i = 0; i < n_ev; ++i) {
-      const uint4 f = wb.rec[i];
-      const uint32_t l = f.y;
-      if (l == 0u) continue;  // out of range, an invalid arrival (prepared), or nothing to release
-      if (f.x >> 31) {  // departure: release the tokens of a dispatched request
-        int32_t dd = (int32_t)f.z;
+    const uint32_t dep_mask = __ballot_sync(0xffffffffu, my_dep);
+    uint32_t arr_mask = __ballot_sync(0xffffffffu, my_arr);
+    uint32_t done = 0;  // events before `done` are applied
+    // the departures between the last arrival and event `upto`, all at once: they commute
+    // (each lowers one load), and lmin only needs the loads they leave
+    auto depart = [&](uint32_t upto) {
+      const uint32_t lo = done >= 32 ? 0u : ~0u << done;
+      const uint32_t hi = upto >= 32 ? ~0u : (1u << upto) - 1u;
+      const uint32_t bm = dep_mask & lo & hi;
+      done = upto;
+      if (!bm) return;
+      uint32_t d = kNone;
+      if ((bm >> lane) & 1u) {
+        int32_t dd = my_dd;
         if (dd >= 0 && ((uint32_t)dd & kInWindow)) dd = wb.wd[(uint32_t)dd & 31u];
         if (dd >= 0 && (uint32_t)dd < D) {
-          const int64_t ld = adjust((uint32_t)dd, -(int64_t)l);
-          if (ld < lmin) {
-            lmin = ld;
-            lt_min = w.theta_s_per_token * (float)lmin;
-            moved = true;
-          }
+          d = (uint32_t)dd;
+          atomicAdd(reinterpret_cast<unsigned long long*>(s_load + d),
+                    (unsigned long long)(-(int64_t)my_l));
         }
-        continue;
       }
-      // the listed candidates as (key << 32 | rank), infeasible ones all ones: the lane's
-      // best pair and second key by a two-level tree of 64-bit minima
-      uint32_t lk = kNoKey, li = kNone, lk2 = kNoKey;
-      if (has_ent) {
-        const uint4 e01 = *reinterpret_cast<const uint4*>(&wb.ent[i][4 * lane]);
-        const uint4 e23 = *reinterpret_cast<const uint4*>(&wb.ent[i][4 * lane + 2]);
-        const uint32_t dr[4] = {e01.x, e01.z, e23.x, e23.z};
-        const uint32_t bs[4] = {e01.y, e01.w, e23.y, e23.w};
-        unsigned long long pk[4];
+      __syncwarp();
+      int64_t ld = INT64_MAX;
+      if (d != kNone) {
+        ld = s_load[d];
+        s_hl[d] = hl_of(ld);  // lanes of the same decode store the same value
+      }
+      if (__any_sync(0xffffffffu, ld < lmin)) {
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const uint2 hl = s_hl[min(dr[j], D)];  // s_hl[D]: a sentinel no request fits
-          pk[j] = l <= hl.x
-              ? ((unsigned long long)score_key(__fmaf_rn(w.w_load, __uint_as_float(hl.y),
-                                                          __uint_as_float(bs[j]))) << 32) | dr[j]
-              : ~0ull;
+        for (int o = 16; o; o >>= 1) {
+          const int64_t x = __shfl_xor_sync(0xffffffffu, ld, o);
+          ld = x < ld ? x : ld;
         }
-        const unsigned long long a = min(pk[0], pk[1]), a2 = max(pk[0], pk[1]);
-        const unsigned long long b = min(pk[2], pk[3]), b2 = max(pk[2], pk[3]);
-        const unsigned long long bp = min(a, b), sp = min(max(a, b), min(a2, b2));
-        lk = (uint32_t)(bp >> 32);
-        li = (uint32_t)bp;
-        lk2 = (uint32_t)(sp >> 32);
+        lmin = ld < lmin ? ld : lmin;
+        lt_min = w.theta_s_per_token * (float)lmin;
+        moved = true;
       }
+      __syncwarp();
+    };
+    while (arr_mask) {
+      const uint32_t i = __ffs(arr_mask) - 1;
+      arr_mask &= arr_mask - 1;
+      depart(i);
+      done = i + 1;
+      const uint4 f = wb.rec[i];
+      const uint32_t l = f.y;
+      // the lane's listed candidate (s_hl[D]: a sentinel no request fits, for empty entries)
+      const uint2 e = wb.ent[i][lane];
+      const uint2 hl = s_hl[min(e.x, D)];
+      const uint32_t lk = l <= hl.x
+          ? score_key(__fmaf_rn(w.w_load, __uint_as_float(hl.y), __uint_as_float(e.y)))
+          : kNoKey;
       // (key, rank) argmin and second key: the rank and the second depend only on the key
-      uint32_t kb = __reduce_min_sync(0xffffffffu, lk);
-      uint32_t bi = __reduce_min_sync(0xffffffffu, lk == kb ? li : kNone);
+      const uint32_t kb = __reduce_min_sync(0xffffffffu, lk);
+      const uint32_t bi = __reduce_min_sync(0xffffffffu, lk == kb ? e.x : kNone);
       const uint32_t ties = __popc(__ballot_sync(0xffffffffu, lk == kb));
-      const uint32_t ks_one = __reduce_min_sync(0xffffffffu, lk == kb ? lk2 : lk);
-      uint32_t ks = ties >= 2 ? kb : ks_one;
+      const uint32_t ks_one = __reduce_min_sync(0xffffffffu, lk == kb ? kNoKey : lk);
+      const uint32_t ks = ties >= 2 ? kb : ks_one;
       const uint32_t tk = f.z, ti = f.w;
       bool cert = listed && tk != kBoundInvalid;
       if (cert && tk != kNoKey) {
@@ -1567,6 +1658,7 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
         }
       }
     }
+    depart(32);  // departures after the window's last arrival
   }
   __syncwarp();
   if (n_win > 0) write_back(win[(n_win - 1) & 1]);
@@ -1608,7 +1700,7 @@ netkv_status launch_listed(const TopoArgs& t, uint32_t n_streams, const netkv_we
                            int64_t* d_load_final, const float* d_base, const uint2* d_lists,
                            const uint2* d_bounds, int* d_status, cudaStream_t s) {
   const size_t smem = sizeof(ListWindow) * 2 + (size_t)t.D * (sizeof(int64_t) + sizeof(uint2)) +
-                      sizeof(uint2);
+                      sizeof(uint2);  // s_hl[D], the sentinel
   if (smem > 48u * 1024u)  // per device: set before every launch that needs it
     NETKV_CUDA_TRY(cudaFuncSetAttribute(schedule_listed_kernel,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
@@ -1672,19 +1764,30 @@ netkv_status launch(const TopoArgs& t, uint32_t n_streams, const netkv_weights* 
                     const uint32_t* d_events, const uint64_t* d_event_off,
                     const int64_t* d_load_init, int32_t* d_dec, float* d_best, float* d_second,
                     int64_t* d_load_final, float* d_base, int* d_status, cudaStream_t s,
-                    uint2* d_lists = nullptr, uint2* d_bounds = nullptr) {
+                    const ListWs* lw = nullptr) {
   const uint32_t per_cta = LPS == 32 ? 1u : 32u / LPS;
   const unsigned grid = (n_streams + per_cta - 1) / per_cta;
   if (d_base) {
-    const bool lists = LPS == 32 && d_lists != nullptr;
+    const bool lists = LPS == 32 && lw != nullptr && lw->lists != nullptr;
     if (launch_base<kUtil>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M, d_UB, n_snap,
                            d_events, d_event_off, d_base, nullptr, d_status, s,
-                           lists ? d_lists : nullptr, lists ? d_bounds : nullptr) != NETKV_OK)
+                           lists ? lw->chunk_lists : nullptr,
+                           lists ? lw->chunk_bounds : nullptr) != NETKV_OK)
       return NETKV_ECUDA;
-    if (lists)
+    if (lists) {
+      int dev = 0, sms = 0;
+      cudaGetDevice(&dev);
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+      const uint64_t blocks = ((uint64_t)R * 32 + 255) / 256;
+      const uint64_t cap = (uint64_t)(sms > 0 ? sms : 1) * 64;
+      merge_lists_kernel<<<(unsigned)(blocks < cap ? blocks : cap), 256, 0, s>>>(
+          lw->chunk_lists, lw->chunk_bounds, (t.D + kListChunk - 1) / kListChunk, R, lw->lists,
+          lw->bounds);
+      if (netkv_launch_status() != NETKV_OK) return NETKV_ECUDA;
       return launch_listed(t, n_streams, d_w, R, d_len, d_prefill, d_snap, n_snap, d_events,
                            d_event_off, d_load_init, d_dec, d_best, d_second, d_load_final,
-                           d_base, d_lists, d_bounds, d_status, s);
+                           d_base, lw->lists, lw->bounds, d_status, s);
+    }
     if (LPS == 32) {
       // one CTA per stream: the walk is bound by each warp's chain of dependent
       // instructions per event; 16 warps (4 per scheduler) measured best on 4,096 decodes
@@ -1767,23 +1870,31 @@ namespace {
 size_t round256(size_t b) { return (b + 255) / 256 * 256; }
 // the base-score rows [R][D], always part of a workspace
 size_t base_ws_bytes(uint32_t R, uint32_t D) { return round256((size_t)R * D * sizeof(float)); }
-// the candidate lists and bounds of pools of 1,025 .. 4,096 decodes (listed walk)
-uint32_t list_chunks(uint32_t D) {
-  return D > kListChunk && D <= kListMaxChunks * kListChunk ? (D + kListChunk - 1) / kListChunk : 0u;
-}
+// pools of 1,025 .. 4,096 decodes: the chunks' candidate lists [R][n_ch][kListLen] and bounds
+// [R][n_ch], then the pool's [R][kListLen] and [R] (listed walk)
+bool listed_pool(uint32_t D) { return D >= kListMinD && D <= kListMaxD; }
+uint32_t list_chunks(uint32_t D) { return (D + kListChunk - 1) / kListChunk; }
 size_t list_ws_bytes(uint32_t R, uint32_t D) {
+  if (!listed_pool(D)) return 0;
   const size_t nc = list_chunks(D);
-  return nc ? round256((size_t)R * nc * kListLen * sizeof(uint2)) + round256((size_t)R * nc * sizeof(uint2))
-            : 0;
+  return round256((size_t)R * nc * kListLen * sizeof(uint2)) + round256((size_t)R * nc * sizeof(uint2)) +
+         round256((size_t)R * kListLen * sizeof(uint2)) + round256((size_t)R * sizeof(uint2));
 }
-// lists and bounds inside a workspace of `bytes` bytes, or nulls (the staged walk)
-void list_ws(void* ws, size_t bytes, uint32_t R, uint32_t D, uint2*& lists, uint2*& bounds) {
-  lists = bounds = nullptr;
+// the list arrays inside a workspace of `bytes` bytes, or nulls (the staged walk)
+ListWs list_ws(void* ws, size_t bytes, uint32_t R, uint32_t D) {
+  ListWs l;
   if (!ws || R == 0 || list_ws_bytes(R, D) == 0 || bytes < base_ws_bytes(R, D) + list_ws_bytes(R, D))
-    return;
+    return l;
+  const size_t nc = list_chunks(D);
   char* p = reinterpret_cast<char*>(ws) + base_ws_bytes(R, D);
-  lists = reinterpret_cast<uint2*>(p);
-  bounds = reinterpret_cast<uint2*>(p + round256((size_t)R * list_chunks(D) * kListLen * sizeof(uint2)));
+  l.chunk_lists = reinterpret_cast<uint2*>(p);
+  p += round256((size_t)R * nc * kListLen * sizeof(uint2));
+  l.chunk_bounds = reinterpret_cast<uint2*>(p);
+  p += round256((size_t)R * nc * sizeof(uint2));
+  l.lists = reinterpret_cast<uint2*>(p);
+  p += round256((size_t)R * kListLen * sizeof(uint2));
+  l.bounds = reinterpret_cast<uint2*>(p);
+  return l;
 }
 }  // namespace
 
@@ -1813,12 +1924,11 @@ extern "C" netkv_status netkv_schedule_streams(
   if (d_workspace && (!aligned_to(d_workspace, 256) || workspace_bytes < base_ws_bytes(R, D)))
     return NETKV_EINVAL;
   float* d_base = (d_workspace && R > 0) ? reinterpret_cast<float*>(d_workspace) : nullptr;
-  uint2 *d_lists, *d_bounds;
-  list_ws(d_base ? d_workspace : nullptr, workspace_bytes, R, D, d_lists, d_bounds);
+  const ListWs lw = list_ws(d_base ? d_workspace : nullptr, workspace_bytes, R, D);
 #define NETKV_SCHED(NPT, BLOCK, LPS)                                                             \
   return launch<NPT, BLOCK, LPS>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, \
                             d_events, d_event_off, d_load_init, d_dec, d_best, d_second,       \
-                            d_load_final, d_base, d_status, s, d_lists, d_bounds)
+                            d_load_final, d_base, d_status, s, &lw)
   if (D <= 8) NETKV_SCHED(1, 32, 8);
   if (D <= 16) NETKV_SCHED(1, 32, 16);
   if (D <= 32) NETKV_SCHED(1, 32, 32);
@@ -1858,13 +1968,12 @@ extern "C" netkv_status netkv_schedule_streams_util(
                                   nullptr, n_snap, d_events, d_event_off, d_load_init, d_dec,
                                   d_best, d_second, d_load_final, nullptr, 0, d_status, stream);
   float* d_base = reinterpret_cast<float*>(d_workspace);
-  uint2 *d_lists, *d_bounds;
-  list_ws(d_workspace, workspace_bytes, R, D, d_lists, d_bounds);
+  const ListWs lw = list_ws(d_workspace, workspace_bytes, R, D);
 #define NETKV_SCHED_U(NPT, BLOCK, LPS)                                                           \
   return launch<NPT, BLOCK, LPS, true>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, d_M,     \
                                        d_util, n_snap, d_events, d_event_off, d_load_init,      \
                                        d_dec, d_best, d_second, d_load_final, d_base, d_status, \
-                                       s, d_lists, d_bounds)
+                                       s, &lw)
   if (D <= 8) NETKV_SCHED_U(1, 32, 8);
   if (D <= 16) NETKV_SCHED_U(1, 32, 16);
   if (D <= 32) NETKV_SCHED_U(1, 32, 32);

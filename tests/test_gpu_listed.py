@@ -1,13 +1,13 @@
 """The listed walk of pools of 1,025 .. 4,096 decodes against the staged walk, bit for bit.
 
 With a workspace of netkv_schedule_workspace_size(R, D) bytes the base-score pass also
-writes each arrival's candidate lists and bounds and the greedy rescans only arrivals the
-bounds do not certify; a workspace holding only the base-score rows (R * D * 4 bytes) runs
-the staged walk over every candidate.  Both are the exact argmin of Algorithm 1 on the same
+writes each arrival's candidate list (the pool's 32 smallest base scores) and bound, and the
+greedy rescans only arrivals the bound does not certify; a workspace holding only the
+base-score rows (R * D * 4 bytes) runs the staged walk over every candidate.  Both are the exact argmin of Algorithm 1 on the same
 fp32 scores, so decisions, best and second scores and final loads must agree exactly, on
 workloads that certify almost every arrival and on ones built to defeat the bounds: a load
 weight that dominates the score, a tight capacity, initial loads (negative ones too), zero
-and negative load weights, and ragged pools whose last chunk is short.  Oracle parity of the
+and negative load weights, and pools of 2 to 4 chunks of 1,024 decodes, ragged ones too.  Oracle parity of the
 listed walk is covered where the bench shapes run (tests/test_gpu_parity.py,
 tests/test_gpu_fused.py, tests/test_gpu_configs.py)."""
 import numpy as np
@@ -35,7 +35,7 @@ def nk():
 
 SHAPES = [((1, 7, 11, 17), 1047),   # two chunks, the second of 23 decodes; D % 4 != 0
           ((1, 8, 8, 40), 2048),
-          ((1, 7, 11, 49), 3018),   # ragged, scalar row reads in the full scans
+          ((1, 7, 11, 49), 3018),   # ragged: scalar row reads in the full scans
           ((1, 8, 8, 80), 4096)]
 
 
@@ -138,7 +138,8 @@ def test_workspace_size_grows_only_for_listed_pools():
     netkv = nk()
     for D in (8, 32, 256, 1024):
         assert netkv.netkv_schedule_workspace_size(1000, D) == (1000 * D * 4 + 255) // 256 * 256
+    r256 = lambda b: (b + 255) // 256 * 256
     for D in (1025, 4096):
-        nc = (D + 1023) // 1024
-        lists = (1000 * nc * 32 * 8 + 255) // 256 * 256 + (1000 * nc * 8 + 255) // 256 * 256
+        nc = (D + 1023) // 1024  # chunk lists of the base pass, then the pool's merged list
+        lists = r256(1000 * nc * 32 * 8) + r256(1000 * nc * 8) + r256(1000 * 32 * 8) + r256(1000 * 8)
         assert netkv.netkv_schedule_workspace_size(1000, D) == (1000 * D * 4 + 255) // 256 * 256 + lists
