@@ -1430,10 +1430,16 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
   const bool listed = w.w_load >= 0.0f && w.theta_s_per_token >= 0.0f;
   const bool vec = (D % 4u == 0) && ((reinterpret_cast<uintptr_t>(base) & 15u) == 0);
 
+  // (float)x of a load: through int32 when it fits (the same value, without the slow 64-bit
+  // conversion)
+  auto to_f = [](int64_t x) -> float {
+    if (__builtin_expect(x == (int64_t)(int32_t)x, 1)) return (float)(int32_t)x;
+    return (float)x;
+  };
   auto hl_of = [&](int64_t ld) -> uint2 {
     const int64_t h = w.cap_tokens - ld;
     const uint32_t hr = h <= 0 ? 0u : h >= 0xffffffffll ? 0xffffffffu : (uint32_t)h;
-    return make_uint2(hr, __float_as_uint(w.theta_s_per_token * (float)ld));
+    return make_uint2(hr, __float_as_uint(w.theta_s_per_token * to_f(ld)));
   };
   int64_t lmin = INT64_MAX;
   for (uint32_t d = lane; d < D; d += 32) {
@@ -1447,7 +1453,7 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
     const int64_t x = __shfl_xor_sync(0xffffffffu, lmin, o);
     lmin = x < lmin ? x : lmin;
   }
-  float lt_min = w.theta_s_per_token * (float)lmin;
+  float lt_min = w.theta_s_per_token * to_f(lmin);
   if (lane == 0) s_hl[D] = make_uint2(0u, 0u);
   __syncwarp();
 
@@ -1491,12 +1497,14 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
       second[r] = key_score(wb.wsk[lane]);
     }
   };
-  // add `delta` tokens to decode dd (lane 0; dispatches never lower lmin)
+  // add `delta` tokens to decode dd: every lane computes the new state (no divergence), lane
+  // 0 stores it (dispatches never lower lmin)
   auto adjust = [&](uint32_t dd, int64_t delta) {
+    const int64_t ld = s_load[dd] + delta;
+    const uint2 h = hl_of(ld);
     if (lane == 0) {
-      const int64_t ld = s_load[dd] + delta;
       s_load[dd] = ld;
-      s_hl[dd] = hl_of(ld);
+      s_hl[dd] = h;
     }
     __syncwarp();
   };
@@ -1583,17 +1591,30 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
       if ((bm >> lane) & 1u) {
         int32_t dd = my_dd;
         if (dd >= 0 && ((uint32_t)dd & kInWindow)) dd = wb.wd[(uint32_t)dd & 31u];
-        if (dd >= 0 && (uint32_t)dd < D) {
-          d = (uint32_t)dd;
-          atomicAdd(reinterpret_cast<unsigned long long*>(s_load + d),
-                    (unsigned long long)(-(int64_t)my_l));
-        }
+        if (dd >= 0 && (uint32_t)dd < D) d = (uint32_t)dd;
       }
-      __syncwarp();
+      // each lane releases its own decode; two departures of one decode (rare) go one by one
+      const uint32_t peers = __match_any_sync(0xffffffffu, d);
       int64_t ld = INT64_MAX;
-      if (d != kNone) {
-        ld = s_load[d];
-        s_hl[d] = hl_of(ld);  // lanes of the same decode store the same value
+      if (__any_sync(0xffffffffu, d != kNone && __popc(peers) > 1)) {
+        uint32_t rest = __ballot_sync(0xffffffffu, d != kNone);
+        while (rest) {
+          const uint32_t src = __ffs(rest) - 1;
+          rest &= rest - 1;
+          const uint32_t ds = __shfl_sync(0xffffffffu, d, src);
+          const uint32_t ls = __shfl_sync(0xffffffffu, my_l, src);
+          if (lane == 0) {
+            const int64_t x = s_load[ds] - (int64_t)ls;
+            s_load[ds] = x;
+            s_hl[ds] = hl_of(x);
+          }
+          __syncwarp();
+        }
+        if (d != kNone) ld = s_load[d];
+      } else if (d != kNone) {
+        ld = s_load[d] - (int64_t)my_l;
+        s_load[d] = ld;
+        s_hl[d] = hl_of(ld);
       }
       if (__any_sync(0xffffffffu, ld < lmin)) {
 #pragma unroll
@@ -1602,7 +1623,7 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
           ld = x < ld ? x : ld;
         }
         lmin = ld < lmin ? ld : lmin;
-        lt_min = w.theta_s_per_token * (float)lmin;
+        lt_min = w.theta_s_per_token * to_f(lmin);
         moved = true;
       }
       __syncwarp();
@@ -1648,7 +1669,7 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
         const ScanResult sr = listed_full_scan(base + (uint64_t)(f.x & 0x7fffffffu) * D, D, vec,
                                                l, w.w_load, s_hl, s_load, lane);
         lmin = sr.lmin;
-        lt_min = w.theta_s_per_token * (float)lmin;
+        lt_min = w.theta_s_per_token * to_f(lmin);
         dstar = sr.kb == kNoKey ? -1 : (int32_t)sr.bi;
         if (dstar >= 0) adjust((uint32_t)dstar, (int64_t)l);
         if (lane == 0) {
