@@ -624,10 +624,13 @@ def run_netkv(args):
 
     R, D = x.R, sc.D
     # level bottlenecks 1; prefix match 4 (group insert, group resolve, leaders, members)
-    # with a workspace or 1 without; greedy 2 (base scores + walk) with a workspace or 1
+    # with a workspace or 1 without; greedy 2 (base scores + walk) with a workspace, 3 for
+    # pools of 1,025 .. 4,096 decodes (base scores with chunk lists, list merge, listed
+    # walk), or 1
+    plain_greedy = not (sc.inflight_cap > 0 or sc.load_model is not None)
+    listed = plain_greedy and sc.precompute_scores and 1025 <= sc.D <= 4096
     launches_per_step = (0 if fused else 1) + (4 if sc.share_prefixes else 1) + (
-        1 if (sc.inflight_cap > 0 or sc.load_model is not None)
-        else (2 if sc.precompute_scores else 1))
+        1 if not plain_greedy else (3 if listed else 2) if sc.precompute_scores else 1)
     n_input_tensors = sum(1 for f in dataclasses.fields(StepInputs)
                           if isinstance(getattr(x, f.name), torch.Tensor))
     decisions = R * world
@@ -643,9 +646,14 @@ def run_netkv(args):
         # per snapshot: the utilisation row (L floats), 16-byte UB of every instance
         "oracle_build": 0 if fused else x.n_snap * (16 + 16 * sc.N) if args.tiers else
                         x.n_snap * ((8 if x.util_down is not None else 4) * w.L + 16 * sc.N),
-        # per arrival: event, len/prefill/snap, per candidate base score (4 B) + the
-        # dec/best/second stores; per departure: event, len, dec
-        "schedule": R * (4 + 12 + 4 * D + 12) + R * 12 + 2 * 8 * D * x.n_streams,
+        # per arrival: event, len/prefill/snap and the dec/best/second stores; per
+        # departure: event, len, dec; the loads in and out.  With a workspace the base pass
+        # reads M (2 B) and writes the base score (4 B) of every candidate, and the walk
+        # reads the row (staged walk) or the candidate list and bound (listed walk: the
+        # chunk lists written and merged, 264 B each); without one the walk reads M.
+        "schedule": R * (4 + 12 + 12) + R * 12 + 2 * 8 * D * x.n_streams + (
+            (R * 6 * D + (R * 264 * (2 * ((D + 1023) // 1024) + 2) if listed else R * 4 * D))
+            if sc.precompute_scores else R * 2 * D),
     }
     dom = max(per_kernel, key=per_kernel.get)
     peak, peak_src = measured_peaks()
@@ -665,8 +673,10 @@ def run_netkv(args):
                 "per_unit": {"prefix_match": "8 B per (request, chain block examined up to its "
                                              "last first miss) + 2 B per M entry",
                              "oracle_build": "per snapshot: the utilisation row + 16 B per instance",
-                             "schedule": "per arrival: event, request fields, 4 B base score per "
-                                         "candidate, dec/best/second; per departure: event, len, dec"}[dom],
+                             "schedule": "per arrival: event, request fields, dec/best/second, "
+                                         "M read and base score written per candidate (2 + 4 B), "
+                                         "then the row (staged walk) or the 264 B candidate list "
+                                         "(listed walk); per departure: event, len, dec"}[dom],
                 "examined_blocks_per_launch": examined,
                 "survey_probe_bytes_per_launch": 16 * probes + 2 * R * D,
                 "survey_probes_per_launch": probes,
