@@ -1478,13 +1478,11 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
         cp_async4(&wb.rec[lane].w, snap + r);
       }
     }
-    uint32_t arr = __ballot_sync(0xffffffffu, valid && !(c >> 31));
-    while (arr) {
-      const uint32_t i = __ffs(arr) - 1;
-      arr &= arr - 1;
-      const uint64_t ri = __shfl_sync(0xffffffffu, r, i);
-      cp_async8(&wb.ent[i][lane], lists + ri * kListLen + lane);
-      if (lane == 0) cp_async8(&wb.bnd[i], bounds + ri);
+    if (valid && !(c >> 31)) {  // the lane's arrival: its list (16 x 16 B) and bound
+      const uint2* src = lists + (uint64_t)r * kListLen;
+#pragma unroll
+      for (int q = 0; q < kListLen; q += 2) cp_async16(&wb.ent[lane][q], src + q);
+      cp_async8(&wb.bnd[lane], bounds + r);
     }
     cp_async_commit();
   };
@@ -1509,6 +1507,13 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
     __syncwarp();
   };
 
+  // departures find their arrival in the window before (decision) or in their own window
+  // (slot) through tables keyed by r mod 128; a window whose arrivals collide in a table
+  // searches by shuffles instead
+  __shared__ uint2 s_prev[128];  // (r, decision)
+  __shared__ uint2 s_cur[128];   // (r, window << 5 | slot)
+  for (uint32_t q = lane; q < 128; q += 32) s_prev[q] = s_cur[q] = make_uint2(kBad, 0u);
+  __syncwarp();
   uint32_t cn = codes_of(0);
   if (n_win > 0) issue(0, cn);
   cn = codes_of(1);
@@ -1535,17 +1540,33 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
     {  // lane i prepares event i
       uint4 f = wb.rec[lane];
       const uint32_t c = f.x, r = c & 0x7fffffffu;
-      // a departure's arrival in the window before, or earlier in this one (every lane
-      // takes part in the shuffles; a lane's r matches only an arrival's code)
+      // a departure's arrival in the window before, or earlier in this one (a lane's r
+      // matches only an arrival's code)
       int32_t dd = (int32_t)f.z;
-      for (uint32_t j = 0; j < 32; ++j) {
-        const uint32_t pc = __shfl_sync(0xffffffffu, prev_code, j);
-        const int32_t pd = __shfl_sync(0xffffffffu, prev_dec, j);
-        if (pc == r) dd = pd;
-      }
-      for (uint32_t j = 0; j < 32; ++j) {
-        const uint32_t cc = __shfl_sync(0xffffffffu, c, j);
-        if (j < lane && cc == r) dd = (int32_t)(kInWindow | j);
+      const uint32_t tag = (uint32_t)(k << 5);
+      const bool prev_arr = prev_code != kBad && !(prev_code >> 31);
+      const bool cur_arr = c != kBad && !(c >> 31);
+      if (prev_arr) s_prev[prev_code & 127u] = make_uint2(prev_code, (uint32_t)prev_dec);
+      if (cur_arr) s_cur[c & 127u] = make_uint2(c, tag | lane);
+      __syncwarp();
+      const bool clash = (prev_arr && s_prev[prev_code & 127u].x != prev_code) ||
+                         (cur_arr && s_cur[c & 127u].x != c);
+      if (__any_sync(0xffffffffu, clash)) {
+        for (uint32_t j = 0; j < 32; ++j) {
+          const uint32_t pc = __shfl_sync(0xffffffffu, prev_code, j);
+          const int32_t pd = __shfl_sync(0xffffffffu, prev_dec, j);
+          if (pc == r) dd = pd;
+        }
+        for (uint32_t j = 0; j < 32; ++j) {
+          const uint32_t cc = __shfl_sync(0xffffffffu, c, j);
+          if (j < lane && cc == r) dd = (int32_t)(kInWindow | j);
+        }
+      } else if (c != kBad && (c >> 31) && r < R) {
+        const uint2 pe = s_prev[r & 127u];
+        if (pe.x == r) dd = (int32_t)pe.y;
+        const uint2 ce = s_cur[r & 127u];
+        if (ce.x == r && (ce.y & ~31u) == tag && (ce.y & 31u) < lane)
+          dd = (int32_t)(kInWindow | (ce.y & 31u));
       }
       if (c == kBad) {
       } else if (r >= R) {
@@ -1587,6 +1608,7 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
       const uint32_t bm = dep_mask & lo & hi;
       done = upto;
       if (!bm) return;
+      __syncwarp();  // lane 0's decisions of this window are visible
       uint32_t d = kNone;
       if ((bm >> lane) & 1u) {
         int32_t dd = my_dd;
