@@ -1653,12 +1653,14 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
     while (arr_mask) {
       const uint32_t i = __ffs(arr_mask) - 1;
       arr_mask &= arr_mask - 1;
+      // the arrival's record, list entry and threshold do not change: read them first
+      const uint4 f = wb.rec[i];
+      const uint2 e = wb.ent[i][lane];
+      const uint32_t lb_i = wb.lb[i];
       depart(i);
       done = i + 1;
-      const uint4 f = wb.rec[i];
       const uint32_t l = f.y;
       // the lane's listed candidate (s_hl[D]: a sentinel no request fits, for empty entries)
-      const uint2 e = wb.ent[i][lane];
       const uint2 hl = s_hl[min(e.x, D)];
       const uint32_t lk = l <= hl.x
           ? score_key(__fmaf_rn(w.w_load, __uint_as_float(hl.y), __uint_as_float(e.y)))
@@ -1669,18 +1671,28 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
       const uint32_t ties = __popc(__ballot_sync(0xffffffffu, lk == kb));
       const uint32_t ks_one = __reduce_min_sync(0xffffffffu, lk == kb ? kNoKey : lk);
       const uint32_t ks = ties >= 2 ? kb : ks_one;
+      // the listed decision is taken at once; an arrival the bounds did not certify (rare)
+      // takes it back and is decided by the full scan.  The dispatch's load is read before
+      // the certification test, whose arithmetic then covers its latency.
+      int32_t dstar = kb == kNoKey ? -1 : (int32_t)bi;
+      const int64_t ld_star = s_load[dstar >= 0 ? (uint32_t)dstar : 0u];
       const uint32_t tk = f.z, ti = f.w;
       bool cert = listed && tk != kBoundInvalid;
       if (cert && tk != kNoKey) {
         const uint32_t klb =
-            moved ? score_key(__fmaf_rn(w.w_load, lt_min, key_score(tk))) : wb.lb[i];
+            moved ? score_key(__fmaf_rn(w.w_load, lt_min, key_score(tk))) : lb_i;
         const bool tie = moved ? lmin >= 0 : tie_ok;
         cert = (kb < klb || (kb == tk && tie && bi < ti)) && ks <= klb;
       }
-      // the listed decision is taken at once; an arrival the bounds did not certify (rare)
-      // takes it back and is decided by the full scan
-      int32_t dstar = kb == kNoKey ? -1 : (int32_t)bi;
-      if (dstar >= 0) adjust((uint32_t)dstar, (int64_t)l);
+      if (dstar >= 0) {
+        const int64_t ld = ld_star + (int64_t)l;
+        const uint2 h = hl_of(ld);
+        if (lane == 0) {
+          s_load[dstar] = ld;
+          s_hl[dstar] = h;
+        }
+        __syncwarp();
+      }
       if (lane == 0) {
         wb.wd[i] = dstar;
         wb.wbk[i] = kb;
