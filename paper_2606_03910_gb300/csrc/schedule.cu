@@ -1363,6 +1363,8 @@ constexpr uint32_t kInWindow = 0x40000000u;  // departure decision: the slot of 
 
 // The full argmin of one arrival from its base-score row (the listed walk's fallback), and
 // the exact minimum load.  Kept out of line: the walk's fast path stays small.
+__device__ __noinline__ float wide_to_float(int64_t x) { return (float)x; }
+
 struct ScanResult {
   uint32_t kb, bi, ks;  // best key, its rank, second-best key
   int64_t lmin;         // the exact minimum load
@@ -1431,10 +1433,10 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
   const bool vec = (D % 4u == 0) && ((reinterpret_cast<uintptr_t>(base) & 15u) == 0);
 
   // (float)x of a load: through int32 when it fits (the same value, without the slow 64-bit
-  // conversion)
+  // conversion, which stays out of line so that it is not evaluated on the common path)
   auto to_f = [](int64_t x) -> float {
     if (__builtin_expect(x == (int64_t)(int32_t)x, 1)) return (float)(int32_t)x;
-    return (float)x;
+    return wide_to_float(x);
   };
   auto hl_of = [&](int64_t ld) -> uint2 {
     const int64_t h = w.cap_tokens - ld;
