@@ -1724,6 +1724,290 @@ __global__ void __launch_bounds__(32) schedule_listed_kernel(
   for (uint32_t d = lane; d < D; d += 32) load_final[(uint64_t)stream * D + d] = s_load[d];
 }
 
+// ---- windowed greedy of small pools (D <= LPS <= 16) with precomputed base scores -----
+// 32 / LPS streams per warp, one segment of LPS lanes each; lane sl owns decode sl's load
+// (and theta * load) in registers.  A stream's events go in windows of 32, double-buffered
+// in shared memory: each event's record (code, length, prefill | decision, snapshot) and an
+// arrival's base-score row are copied with cp.async one window ahead by the lane that
+// prepares the event (event j of a window: lane j % LPS).  Before a window is walked, each
+// departure's decision is found: from the window before or as the slot of its arrival in
+// this window, through tables keyed by request index mod 64 (a window whose arrivals collide
+// there searches by shuffles), else the copy of the global decision (written back one window
+// earlier).  The window is then walked arrival by arrival, the segments of a warp side by
+// side: the departures since a segment's last arrival are applied one after another (a
+// broadcast and the owner lane's update each), then every lane scores its decode exactly as
+// schedule_kernel does, and a segment butterfly takes the (score, rank) argmin with the
+// second score.  Decisions and scores go back to global memory when the next window starts.
+template <int LPS>
+struct WinSeg {              // one stream's window buffer
+  uint4 rec[32];             // code, length, prefill | decision, snapshot
+  float bs[32][LPS];         // base scores of an arrival's row
+  int32_t wd[32];            // decisions
+  float wb[32], ws[32];      // best and second scores
+};
+constexpr int kWinWarps = 4;  // warps per block (independent)
+
+template <int LPS>
+__global__ void __launch_bounds__(32 * kWinWarps) schedule_window_kernel(
+    TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
+    const float* __restrict__ base, const uint32_t* __restrict__ len,
+    const uint32_t* __restrict__ prefill, const uint32_t* __restrict__ snap, uint32_t n_snap,
+    const uint32_t* __restrict__ events, const uint64_t* __restrict__ event_off,
+    const int64_t* __restrict__ load_init, int32_t* dec, float* __restrict__ best,
+    float* __restrict__ second, int64_t* __restrict__ load_final, int* status) {
+  static_assert(LPS == 8 || LPS == 16, "segments of 8 or 16 lanes");
+  constexpr int S = 32 / LPS;  // streams per warp
+  constexpr int E = 32 / LPS;  // events a lane prepares per window
+  constexpr uint32_t kBad = 0xffffffffu;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const uint32_t lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+  const uint32_t seg = lane / LPS, sl = lane % LPS, seg0 = seg * LPS;
+  const uint32_t smask = ((1u << LPS) - 1u) << seg0;
+  const uint32_t stream = ((uint32_t)blockIdx.x * kWinWarps + wib) * S + seg;
+  const bool live = stream < n_streams;
+  WinSeg<LPS>* wsb = reinterpret_cast<WinSeg<LPS>*>(smem_raw) + ((size_t)wib * S + seg) * 2;
+  uint2* tabs = reinterpret_cast<uint2*>(reinterpret_cast<WinSeg<LPS>*>(smem_raw) +
+                                         (size_t)kWinWarps * S * 2) +
+                ((size_t)wib * S + seg) * 128;
+  uint2* tab_prev = tabs;       // (r, decision) of the window before's arrivals
+  uint2* tab_cur = tabs + 64;   // (r, window << 5 | slot) of this window's arrivals
+  const uint32_t D = t.D;
+  const netkv_weights w = live ? W[stream] : W[0];
+  const float inf = __int_as_float(0x7f800000);
+  const bool mine = live && sl < D;
+
+  int64_t load = 0;
+  if (mine && load_init) load = load_init[(uint64_t)stream * D + sl];
+  float ltf = w.theta_s_per_token * (float)load;
+  for (uint32_t q = sl; q < 128; q += LPS) tabs[q] = make_uint2(kBad, 0u);
+
+  const uint64_t e0 = live ? event_off[stream] : 0, e1 = live ? event_off[stream + 1] : 0;
+  const uint32_t my_win = (uint32_t)((e1 - e0 + 31) / 32);
+  const uint32_t n_win = __reduce_max_sync(0xffffffffu, my_win);
+  auto codes_of = [&](uint32_t k, uint32_t* c) {
+#pragma unroll
+    for (int q = 0; q < E; ++q) {
+      const uint64_t e = e0 + 32ull * k + (uint32_t)q * LPS + sl;
+      c[q] = e < e1 ? __ldg(events + e) : kBad;
+    }
+  };
+  // window k's copies (codes c) into buffer k & 1, one cp.async group
+  auto issue = [&](uint32_t k, const uint32_t* c) {
+    WinSeg<LPS>& b = wsb[k & 1];
+#pragma unroll
+    for (int q = 0; q < E; ++q) {
+      const uint32_t j = (uint32_t)q * LPS + sl, code = c[q], r = code & 0x7fffffffu;
+      b.rec[j].x = code;
+      if (code != kBad && r < R) {
+        cp_async4(&b.rec[j].y, len + r);
+        if (code >> 31) {
+          cp_async4(&b.rec[j].z, dec + r);
+        } else {
+          cp_async4(&b.rec[j].z, prefill + r);
+          cp_async4(&b.rec[j].w, snap + r);
+          const float* row = base + (uint64_t)r * D;
+          for (uint32_t d = 0; d < D; ++d) cp_async4(&b.bs[j][d], row + d);
+        }
+      }
+    }
+    cp_async_commit();
+  };
+
+  uint32_t cn[E], cc[E], pc[E];  // codes of the next window, this one, the one before
+  int32_t pd[E];                 // decisions of the window before (its arrivals)
+#pragma unroll
+  for (int q = 0; q < E; ++q) {
+    pc[q] = kBad;
+    pd[q] = -1;
+  }
+  codes_of(0, cc);
+  if (n_win > 0) issue(0, cc);
+  codes_of(1, cn);
+  for (uint32_t k = 0; k < n_win; ++k) {
+    if (k > 0) {  // the window before (codes pc): write its results back, remember them
+      const WinSeg<LPS>& pb = wsb[(k - 1) & 1];
+#pragma unroll
+      for (int q = 0; q < E; ++q) {
+        const uint32_t j = (uint32_t)q * LPS + sl, code = pc[q], r = code & 0x7fffffffu;
+        pd[q] = -1;
+        if (code != kBad && !(code >> 31) && r < R) {
+          pd[q] = pb.wd[j];
+          dec[r] = pb.wd[j];
+          best[r] = pb.wb[j];
+          second[r] = pb.ws[j];
+          tab_prev[r & 63u] = make_uint2(r, (uint32_t)pd[q]);
+        }
+      }
+    }
+    __syncwarp();  // every lane is done with buffer (k + 1) & 1 and the tables
+    if (k + 1 < n_win) issue(k + 1, cn);
+    else cp_async_commit();
+    uint32_t cn2[E];  // the window after next
+    codes_of(k + 2, cn2);
+    cp_async_wait<1>();
+    __syncwarp();
+    WinSeg<LPS>& b = wsb[k & 1];
+    // prepare: this window's arrivals into the current table, then every departure's decision
+    bool clash = false;
+#pragma unroll
+    for (int q = 0; q < E; ++q) {
+      const uint32_t j = (uint32_t)q * LPS + sl, code = cc[q], r = code & 0x7fffffffu;
+      if (code != kBad && !(code >> 31) && r < R) tab_cur[r & 63u] = make_uint2(r, (k << 5) | j);
+      if (k > 0 && pc[q] != kBad && !(pc[q] >> 31) && (pc[q] & 0x7fffffffu) < R)
+        clash |= tab_prev[pc[q] & 63u].x != pc[q];
+    }
+    __syncwarp();
+#pragma unroll
+    for (int q = 0; q < E; ++q) {
+      const uint32_t j = (uint32_t)q * LPS + sl, code = cc[q], r = code & 0x7fffffffu;
+      if (code != kBad && !(code >> 31) && r < R) clash |= tab_cur[r & 63u].y != ((k << 5) | j);
+    }
+    const bool seg_clash = (__ballot_sync(0xffffffffu, clash) & smask) != 0;
+    uint32_t l_ev[E], dd_ev[E];  // per prepared event: length, departure's decode or marker
+    uint32_t arr_bits = 0, dep_bits = 0;  // this lane's events, bit q
+#pragma unroll
+    for (int q = 0; q < E; ++q) {
+      const uint32_t j = (uint32_t)q * LPS + sl, code = cc[q], r = code & 0x7fffffffu;
+      const uint4 f = b.rec[j];
+      l_ev[q] = f.y;
+      dd_ev[q] = kBad;
+      if (code == kBad) continue;
+      if (r >= R) {
+        flag_status(status, NETKV_DEV_ERANGE);
+        continue;
+      }
+      if (code >> 31) {
+        int32_t dd = (int32_t)f.z;
+        if (!seg_clash) {
+          const uint2 pe = tab_prev[r & 63u];
+          if (pe.x == r) dd = (int32_t)pe.y;
+          const uint2 ce = tab_cur[r & 63u];
+          if (ce.x == r && (ce.y >> 5) == (k & 0x7ffffffu) && (ce.y & 31u) < j)
+            dd = (int32_t)(kInWindow | (ce.y & 31u));
+        }
+        dd_ev[q] = (uint32_t)dd;
+        if (f.y != 0u) dep_bits |= 1u << q;
+      } else {
+        if (f.z < t.P && f.w < n_snap && f.y != 0u) {
+          arr_bits |= 1u << q;
+        } else {
+          flag_status(status, f.y == 0u ? NETKV_DEV_EDOMAIN : NETKV_DEV_ERANGE);
+          b.wd[j] = -1;
+          b.wb[j] = inf;
+          b.ws[j] = inf;
+        }
+      }
+    }
+    if (__any_sync(0xffffffffu, seg_clash)) {  // collisions: search the windows by shuffles
+#pragma unroll
+      for (int q = 0; q < E; ++q) {
+        const uint32_t j = (uint32_t)q * LPS + sl, r = cc[q] & 0x7fffffffu;
+        const bool dep = cc[q] != kBad && (cc[q] >> 31) && r < R;
+#pragma unroll
+        for (int qq = 0; qq < E; ++qq) {
+          for (uint32_t m = 0; m < (uint32_t)LPS; ++m) {
+            const uint32_t pcs = __shfl_sync(0xffffffffu, pc[qq], seg0 + m);
+            const int32_t pds = __shfl_sync(0xffffffffu, pd[qq], seg0 + m);
+            const uint32_t ccs = __shfl_sync(0xffffffffu, cc[qq], seg0 + m);
+            const uint32_t jj = (uint32_t)qq * LPS + m;
+            if (seg_clash && dep) {
+              if (pcs == r) dd_ev[q] = (uint32_t)pds;
+              if (ccs == r && jj < j) dd_ev[q] = kInWindow | jj;
+            }
+          }
+        }
+      }
+    }
+    // the segment's arrival and departure slots (bit j of the window)
+    uint32_t arr_mask = 0, dep_mask = 0;
+#pragma unroll
+    for (int q = 0; q < E; ++q) {
+      const uint32_t ba = __ballot_sync(0xffffffffu, (arr_bits >> q) & 1u);
+      const uint32_t bd = __ballot_sync(0xffffffffu, (dep_bits >> q) & 1u);
+      arr_mask |= ((ba >> seg0) & ((1u << LPS) - 1u)) << (q * LPS);
+      dep_mask |= ((bd >> seg0) & ((1u << LPS) - 1u)) << (q * LPS);
+    }
+    __syncwarp();  // prepared results of invalid arrivals are visible
+    // the departures of slots in `bits` (segment-uniform), in slot order
+    auto apply = [&](uint32_t bits) {
+      uint32_t n = __popc(bits);
+      const uint32_t rounds = __reduce_max_sync(0xffffffffu, n);
+      for (uint32_t it = 0; it < rounds; ++it) {
+        const bool has = bits != 0;
+        const uint32_t j = has ? __ffs(bits) - 1 : 0u;
+        if (has) bits &= bits - 1;
+        const uint32_t qj = j / LPS, holder = seg0 + j % LPS;
+        uint32_t pv = 0, pl = 0;
+#pragma unroll
+        for (int q = 0; q < E; ++q)
+          if ((uint32_t)q == qj) {
+            pv = dd_ev[q];
+            pl = l_ev[q];
+          }
+        uint32_t dd = __shfl_sync(0xffffffffu, pv, holder);
+        const uint32_t l = __shfl_sync(0xffffffffu, pl, holder);
+        if (has && dd != kBad && (dd & kInWindow) && (int32_t)dd >= 0) dd = (uint32_t)b.wd[dd & 31u];
+        if (has && mine && dd == sl) {
+          load -= (int64_t)l;
+          ltf = w.theta_s_per_token * (float)load;
+        }
+      }
+    };
+    uint32_t done = 0;  // slots below `done` are applied or decided
+    const uint32_t rounds = __reduce_max_sync(0xffffffffu, __popc(arr_mask));
+    for (uint32_t it = 0; it < rounds; ++it) {
+      __syncwarp();  // decisions stored by earlier rounds are visible
+      const bool has = arr_mask != 0;
+      const uint32_t a = has ? __ffs(arr_mask) - 1 : 0u;
+      if (has) arr_mask &= arr_mask - 1;
+      apply(has ? dep_mask & ((1u << a) - 1u) & ~((1u << done) - 1u) : 0u);
+      if (has) done = a + 1;
+      const uint4 f = b.rec[a];
+      const uint32_t l = f.y;
+      float bsc = inf, s2 = inf;
+      uint32_t bi = kNone;
+      if (has && mine && load + (int64_t)l <= w.cap_tokens) {
+        bsc = __fmaf_rn(w.w_load, ltf, b.bs[a][sl]);
+        bi = sl;
+      }
+      seg_argmin<LPS>(bsc, bi, s2, 0xffffffffu);
+      const int32_t dstar = bi == kNone ? -1 : (int32_t)bi;
+      if (has && mine && dstar == (int32_t)sl) {
+        load += (int64_t)l;
+        ltf = w.theta_s_per_token * (float)load;
+      }
+      if (has && sl == 0) {
+        b.wd[a] = dstar;
+        b.wb[a] = bsc;
+        b.ws[a] = s2;
+      }
+    }
+    __syncwarp();
+    apply(dep_mask & ~((1u << done) - 1u) & (done >= 32 ? 0u : ~0u));  // after the last arrival
+#pragma unroll
+    for (int q = 0; q < E; ++q) {  // the codes move on by one window
+      pc[q] = cc[q];
+      cc[q] = cn[q];
+      cn[q] = cn2[q];
+    }
+  }
+  __syncwarp();
+  if (n_win > 0) {  // the last window's results (its codes are pc now)
+    const WinSeg<LPS>& pb = wsb[(n_win - 1) & 1];
+#pragma unroll
+    for (int q = 0; q < E; ++q) {
+      const uint32_t j = (uint32_t)q * LPS + sl, code = pc[q], r = code & 0x7fffffffu;
+      if (code != kBad && !(code >> 31) && r < R) {
+        dec[r] = pb.wd[j];
+        best[r] = pb.wb[j];
+        second[r] = pb.ws[j];
+      }
+    }
+  }
+  cp_async_wait<0>();
+  if (mine) load_final[(uint64_t)stream * D + sl] = load;
+}
+
 constexpr int kStages = 8;
 constexpr uint32_t kHeapPerStream = 4096;       // pending completions, one stream per CTA
 constexpr uint32_t kHeapPerPackedStream = 256;  // pending completions, packed streams
@@ -1743,6 +2027,28 @@ netkv_status launch_staged(const TopoArgs& t, uint32_t n_streams, const netkv_we
     NETKV_CUDA_TRY(cudaFuncSetAttribute(schedule_staged_kernel<NPT, BLOCK, kStages>,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
   schedule_staged_kernel<NPT, BLOCK, kStages><<<n_streams, BLOCK, smem, s>>>(
+      t, n_streams, d_w, R, d_base, d_len, d_prefill, d_snap, n_snap, d_events, d_event_off,
+      d_load_init, d_dec, d_best, d_second, d_load_final, d_status);
+  return netkv_launch_status();
+}
+
+// The windowed walk of pools of at most LPS decodes: 32 / LPS streams per warp.
+template <int LPS>
+netkv_status launch_window(const TopoArgs& t, uint32_t n_streams, const netkv_weights* d_w,
+                           uint32_t R, const uint32_t* d_len, const uint32_t* d_prefill,
+                           const uint32_t* d_snap, uint32_t n_snap, const uint32_t* d_events,
+                           const uint64_t* d_event_off, const int64_t* d_load_init,
+                           int32_t* d_dec, float* d_best, float* d_second,
+                           int64_t* d_load_final, const float* d_base, int* d_status,
+                           cudaStream_t s) {
+  constexpr uint32_t S = 32 / LPS;
+  const size_t smem = (size_t)kWinWarps * S * (2 * sizeof(WinSeg<LPS>) + 128 * sizeof(uint2));
+  if (smem > 48u * 1024u)  // per device: set before every launch that needs it
+    NETKV_CUDA_TRY(cudaFuncSetAttribute(schedule_window_kernel<LPS>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+  const uint64_t warps = ((uint64_t)n_streams + S - 1) / S;
+  const unsigned grid = (unsigned)((warps + kWinWarps - 1) / kWinWarps);
+  schedule_window_kernel<LPS><<<grid, 32 * kWinWarps, smem, s>>>(
       t, n_streams, d_w, R, d_base, d_len, d_prefill, d_snap, n_snap, d_events, d_event_off,
       d_load_init, d_dec, d_best, d_second, d_load_final, d_status);
   return netkv_launch_status();
@@ -1864,6 +2170,11 @@ netkv_status launch(const TopoArgs& t, uint32_t n_streams, const netkv_weights* 
       return launch_staged<8, 512>(t, n_streams, d_w, R, d_len, d_prefill, d_snap, n_snap,
                                    d_events, d_event_off, d_load_init, d_dec, d_best, d_second,
                                    d_load_final, d_base, d_status, s);
+    } else if (LPS == 8 || LPS == 16) {
+      return launch_window<(LPS == 16 ? 16 : 8)>(t, n_streams, d_w, R, d_len, d_prefill, d_snap,
+                                                 n_snap, d_events, d_event_off, d_load_init,
+                                                 d_dec, d_best, d_second, d_load_final, d_base,
+                                                 d_status, s);
     } else {
       schedule_kernel<NPT, BLOCK, LPS, true><<<grid, BLOCK, 0, s>>>(
           t, n_streams, d_w, R, d_base, d_len, d_prefill, d_snap, d_M, d_UB, n_snap, d_events,
