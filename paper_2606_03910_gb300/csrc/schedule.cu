@@ -1771,6 +1771,11 @@ __global__ void __launch_bounds__(32 * kWinWarps) schedule_window_kernel(
                 ((size_t)wib * S + seg) * 128;
   uint2* tab_prev = tabs;       // (r, decision) of the window before's arrivals
   uint2* tab_cur = tabs + 64;   // (r, window << 5 | slot) of this window's arrivals
+  // tokens released before the segment's b-th arrival of the window, per decode: rel[b][d]
+  uint32_t* rel = reinterpret_cast<uint32_t*>(reinterpret_cast<uint2*>(
+                      reinterpret_cast<WinSeg<LPS>*>(smem_raw) + (size_t)kWinWarps * S * 2) +
+                  (size_t)kWinWarps * S * 128) +
+                  ((size_t)wib * S + seg) * 33 * LPS;
   const uint32_t D = t.D;
   const netkv_weights w = live ? W[stream] : W[0];
   const float inf = __int_as_float(0x7f800000);
@@ -1780,6 +1785,7 @@ __global__ void __launch_bounds__(32 * kWinWarps) schedule_window_kernel(
   if (mine && load_init) load = load_init[(uint64_t)stream * D + sl];
   float ltf = w.theta_s_per_token * (float)load;
   for (uint32_t q = sl; q < 128; q += LPS) tabs[q] = make_uint2(kBad, 0u);
+  for (uint32_t q = sl; q < 33u * LPS; q += LPS) rel[q] = 0u;
 
   const uint64_t e0 = live ? event_off[stream] : 0, e1 = live ? event_off[stream + 1] : 0;
   const uint32_t my_win = (uint32_t)((e1 - e0 + 31) / 32);
@@ -1927,7 +1933,43 @@ __global__ void __launch_bounds__(32 * kWinWarps) schedule_window_kernel(
       arr_mask |= ((ba >> seg0) & ((1u << LPS) - 1u)) << (q * LPS);
       dep_mask |= ((bd >> seg0) & ((1u << LPS) - 1u)) << (q * LPS);
     }
-    __syncwarp();  // prepared results of invalid arrivals are visible
+    // a departure whose decode is known now (not an arrival of this window) adds its tokens
+    // to rel[number of the segment's arrivals before it][decode]; the rest (and any of more
+    // than 2^27 tokens, so that a sum of 32 fits in 32 bits) are released one by one
+    uint32_t slow_bits = 0;
+#pragma unroll
+    for (int q = 0; q < E; ++q) {
+      const uint32_t j = (uint32_t)q * LPS + sl;
+      bool slow = false;
+      if ((dep_bits >> q) & 1u) {
+        const uint32_t dd = dd_ev[q];
+        if ((dd & kInWindow) && (int32_t)dd >= 0) {
+          slow = true;
+        } else if (dd < D) {
+          if (l_ev[q] < (1u << 27)) atomicAdd(&rel[__popc(arr_mask & ((1u << j) - 1u)) * LPS + dd], l_ev[q]);
+          else slow = true;
+        }
+      }
+      slow_bits |= (slow ? 1u : 0u) << q;
+    }
+    uint32_t slow_mask = 0;
+#pragma unroll
+    for (int q = 0; q < E; ++q) {
+      const uint32_t bs_ = __ballot_sync(0xffffffffu, (slow_bits >> q) & 1u);
+      slow_mask |= ((bs_ >> seg0) & ((1u << LPS) - 1u)) << (q * LPS);
+    }
+    __syncwarp();  // prepared results of invalid arrivals and the releases are visible
+    // the segment's released tokens of batch `bi` (the departures before its bi-th arrival)
+    auto release = [&](uint32_t bi) {
+      if (mine) {
+        const uint32_t x = rel[bi * LPS + sl];
+        if (x != 0u) {
+          rel[bi * LPS + sl] = 0u;
+          load -= (int64_t)x;
+          ltf = w.theta_s_per_token * (float)load;
+        }
+      }
+    };
     // the departures of slots in `bits` (segment-uniform), in slot order
     auto apply = [&](uint32_t bits) {
       uint32_t n = __popc(bits);
@@ -1960,7 +2002,8 @@ __global__ void __launch_bounds__(32 * kWinWarps) schedule_window_kernel(
       const bool has = arr_mask != 0;
       const uint32_t a = has ? __ffs(arr_mask) - 1 : 0u;
       if (has) arr_mask &= arr_mask - 1;
-      apply(has ? dep_mask & ((1u << a) - 1u) & ~((1u << done) - 1u) : 0u);
+      release(it);
+      apply(has ? slow_mask & ((1u << a) - 1u) & ~((1u << done) - 1u) : 0u);
       if (has) done = a + 1;
       const uint4 f = b.rec[a];
       const uint32_t l = f.y;
@@ -1983,7 +2026,8 @@ __global__ void __launch_bounds__(32 * kWinWarps) schedule_window_kernel(
       }
     }
     __syncwarp();
-    apply(dep_mask & ~((1u << done) - 1u) & (done >= 32 ? 0u : ~0u));  // after the last arrival
+    release(rounds);  // after the last arrival
+    apply(slow_mask & ~((1u << done) - 1u) & (done >= 32 ? 0u : ~0u));
 #pragma unroll
     for (int q = 0; q < E; ++q) {  // the codes move on by one window
       pc[q] = cc[q];
@@ -2042,7 +2086,8 @@ netkv_status launch_window(const TopoArgs& t, uint32_t n_streams, const netkv_we
                            int64_t* d_load_final, const float* d_base, int* d_status,
                            cudaStream_t s) {
   constexpr uint32_t S = 32 / LPS;
-  const size_t smem = (size_t)kWinWarps * S * (2 * sizeof(WinSeg<LPS>) + 128 * sizeof(uint2));
+  const size_t smem = (size_t)kWinWarps * S *
+                      (2 * sizeof(WinSeg<LPS>) + 128 * sizeof(uint2) + 33 * LPS * sizeof(uint32_t));
   if (smem > 48u * 1024u)  // per device: set before every launch that needs it
     NETKV_CUDA_TRY(cudaFuncSetAttribute(schedule_window_kernel<LPS>,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
