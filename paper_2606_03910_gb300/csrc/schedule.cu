@@ -1780,6 +1780,7 @@ __global__ void __launch_bounds__(32 * kWinWarps) schedule_window_kernel(
   const netkv_weights w = live ? W[stream] : W[0];
   const float inf = __int_as_float(0x7f800000);
   const bool mine = live && sl < D;
+  const bool vec4 = (D % 4u == 0) && ((reinterpret_cast<uintptr_t>(base) & 15u) == 0);
 
   int64_t load = 0;
   if (mine && load_init) load = load_init[(uint64_t)stream * D + sl];
@@ -1812,7 +1813,11 @@ __global__ void __launch_bounds__(32 * kWinWarps) schedule_window_kernel(
           cp_async4(&b.rec[j].z, prefill + r);
           cp_async4(&b.rec[j].w, snap + r);
           const float* row = base + (uint64_t)r * D;
-          for (uint32_t d = 0; d < D; ++d) cp_async4(&b.bs[j][d], row + d);
+          if (vec4) {  // 16-byte copies: D % 4 == 0 and an aligned base
+            for (uint32_t d = 0; d < D; d += 4) cp_async16(&b.bs[j][d], row + d);
+          } else {
+            for (uint32_t d = 0; d < D; ++d) cp_async4(&b.bs[j][d], row + d);
+          }
         }
       }
     }
