@@ -140,13 +140,13 @@ def workload_config(streams, world, extra=None, kind="replicas"):
                            "telemetry",
                "streams_per_gpu": 16, "requests_per_stream": 100_000, "decodes": 4096,
                "prefills": 1024, "parallelism": f"replicas{world}",
-               "l2": "inputs larger than L2 (cache index 64 GiB, M 13 GB per GPU)"}
+               "l2": "inputs larger than L2 (cache index 4 GiB, M 13 GB per GPU)"}
     else:
         cfg = {"workload": f"{streams} replicas x 64-GPU four-tier tree (8P+8D, TP=4), "
                            "1,000 requests/stream, decode caches of 200K blocks",
                "streams_per_gpu": streams, "requests_per_stream": 1000, "decodes": 8,
                "prefills": 8, "parallelism": f"replicas{world}",
-               "l2": "inputs larger than L2 (cache index 64 GiB + chains 27 GB per GPU)"}
+               "l2": "inputs larger than L2 (cache index 100 GiB + chains 27 GB per GPU)"}
     if extra:
         cfg.update(extra)
     return cfg
@@ -228,9 +228,9 @@ KERNEL_CODE = {
 #   prefix_match: bytes per request, from the 64-replica case of the bench workload
 #   oracle_build: bytes per snapshot of the oracle-build sweep
 MEASURED_TRAFFIC = {
-    # 64 replicas (64,000 requests): group_insert 8.97 MB, group_resolve 9.11 MB,
-    # match_leaders 129.31 MB, match_kernel<members> 243.13 MB (read + write)
-    "prefix_match": {"code_sha256_16": "25b21a15533a1bcf", "bytes_per_unit": 390_518_016 / 64_000,
+    # 64 replicas (64,000 requests): group_insert 8.96 MB, group_resolve 9.11 MB,
+    # match_leaders 92.63 MB, match_members_kernel 235.99 MB (read + write)
+    "prefix_match": {"code_sha256_16": "81aee53484a5a95a", "bytes_per_unit": 346_683_392 / 64_000,
                      "unit": "request", "captured": "64-replica case, one launch per kernel"},
     "oracle_build": {"code_sha256_16": "ed437e71560780e2", "bytes_per_unit": 67_155_930,
                      "unit": "snapshot", "captured": "1,000-snapshot sweep, one launch"},

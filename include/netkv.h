@@ -154,11 +154,13 @@ netkv_status netkv_oracle_build_tiers(netkv_topology_t topo, const float* d_c, u
 /* ------------------------------------------------------------------ caches
  * Decode caches K_d (Sec. III-C), the sets of block hashes each decode instance holds.
  * Decodes are taken in groups of 64 (decode ranks 64q .. 64q+63 form group q); each
- * (table set g, group q) has one index of 2^log2_capacity hash slots followed by
- * 2^log2_capacity run entries, index number g * G + q with G = ceil(D / 64):
- *   run entries  {uint64 hash, uint64 mask}: the group's distinct cached hashes in list
- *                order (decode by decode, first appearance); bit (d mod 64) of the mask
- *                says that decode d caches the hash;
+ * (table set g, group q) has one index, index number g * G + q with G = ceil(D / 64), of
+ * 2^log2_capacity hash slots, then 2^log2_capacity run keys, then 2^log2_capacity run
+ * masks, padded to a multiple of 256 bytes:
+ *   run keys     uint64: the group's distinct cached hashes in list order (decode by
+ *                decode, first appearance);
+ *   run masks    W bytes each, W = 1, 2, 4 or 8 for D <= 8, <= 16, <= 32 or more: bit
+ *                (d mod 64) says that decode d caches the run key at that position;
  *   hash slots   {uint64 hash, uint64 run position}, open addressing with linear probing
  *                from a multiplicative hash; hash 0 marks an empty slot (block hash 0 is
  *                reserved).
@@ -213,7 +215,7 @@ netkv_status netkv_prefix_match(const void* d_index, uint32_t D, uint32_t log2_c
  * serves callers that cannot allocate device memory at scoring time, for example a
  * scheduler plugin that runs inside a serving engine whose memory pool owns the whole
  * GPU, or code that must not call cudaMalloc on its request path.  It computes exactly
- * what netkv_prefix_match computes with a workspace, using instead a fixed 24 MiB
+ * what netkv_prefix_match computes with a workspace, using instead a fixed 32 MiB
  * device array compiled into the library (every GPU that loads the library keeps it
  * until the process exits).
  *   - Arguments are those of netkv_prefix_match without the workspace.

@@ -3,9 +3,10 @@
 // that are all cached on decode d.
 //
 // Cache index.  The caches of a table set are indexed per group of up to 64 decodes:
-//   run array   the group's distinct cached hashes in the order the key lists give them
-//               (decode by decode, first appearance), each with a 64-bit mask of the
-//               group's decodes that cache it;
+//   run keys    the group's distinct cached hashes in the order the key lists give them
+//               (decode by decode, first appearance);
+//   run masks   beside each run key, the mask of the group's decodes that cache it, in
+//               1, 2, 4 or 8 bytes by the pool's size;
 //   hash table  open addressing, 16-byte slots {hash, position in the run array}.
 // Caches are filled with whole prefixes of chains, so a cached prefix sits in the run
 // array as a contiguous run in chain order.
@@ -15,9 +16,9 @@
 //
 // Match.  One warp per (request, decode group).  The warp looks up the block at the
 // current position in the hash table (one random access), then compares the chain with
-// the run array from that position on, 32 blocks per step (a 256-byte chain load and a
-// 512-byte run load, both coalesced): every block that equals the next run entry is
-// cached exactly on the decodes of that entry's mask, and one ballot per live decode
+// the run keys from that position on, 32 blocks per step (coalesced loads of 256 chain
+// bytes, 256 key bytes and 32 .. 256 mask bytes): every block that equals the next run key
+// is cached exactly on the decodes of that position's mask, and one ballot per live decode
 // finds its first missing block.  Where chain and run part, the next block is looked up
 // in the hash table again; a block absent from the table is missing on every decode.
 // The answer never depends on the run order (any key order is exact); the order only
@@ -28,10 +29,11 @@
 // on those blocks, so with a workspace the match runs in three steps:
 //   group_insert_kernel / group_resolve_kernel: requests are grouped by (table set,
 //     first block hash) in an open-addressing table; each group's leader is its
-//     longest chain (lowest index among equals); leaders go to a compact list.
+//     longest chain (lowest index among equals); leaders go to a compact list, and each
+//     member gets a record of its own and its leader's chain offsets and lengths.
 //   match_leaders_kernel: leaders (and ungrouped requests) run the full match, one task
 //     per (leader, decode group) taken in order from a counter.
-//   match_kernel<kMembers>: a member r with leader L compares chains to get
+//   match_members_kernel: a member r with leader L compares chains to get
 //     lcp = |common prefix of h_r and h_L| (capped at max_d M_L[d] + 1).  For a decode
 //     with M_L[d] < lcp the first missing block of L lies inside the common prefix, so
 //     M_r[d] = M_L[d] exactly; otherwise blocks [0, lcp) are all cached and the walk
@@ -77,12 +79,13 @@ __global__ void __launch_bounds__(kBuildBlock) cache_build_kernel(
   __shared__ uint32_t chunk_new;
   const uint64_t cap = 1ull << log2_cap, mask = cap - 1;
   const uint32_t n_dgroups = (D + kGroup - 1) / kGroup;
+  const uint32_t mb = mask_bytes_of(D);
   const uint64_t n_index = (uint64_t)n_sets * n_dgroups;
   for (uint64_t idx = blockIdx.x; idx < n_index; idx += gridDim.x) {
     const uint64_t g = idx / n_dgroups;
     const uint32_t q = (uint32_t)(idx - g * n_dgroups);
-    IndexSlot* hash = index_hash(index, idx, log2_cap);
-    RunEntry* run = reinterpret_cast<RunEntry*>(hash + cap);
+    const IndexView v = index_view(index, idx, log2_cap, mb);
+    IndexSlot* hash = v.hash;
     uint32_t run_len = 0;  // same value in every thread
     for (uint32_t d = q * kGroup; d < min(D, (q + 1) * kGroup); ++d) {
       const uint64_t t = g * D + d;
@@ -115,13 +118,13 @@ __global__ void __launch_bounds__(kBuildBlock) cache_build_kernel(
         const uint32_t pos = run_len + block_scan(is_new ? 1u : 0u, warp_sums, &chunk_new);
         if (is_new) {
           hash[slot].pos = pos;
-          run[pos].key = key;
-          run[pos].mask = bit;
+          v.keys[pos] = key;
+          run_mask_or(v, pos, bit);  // masks share 32-bit words: set by atomics only
         }
         __syncthreads();
         if (placed && !is_new) {
           const uint64_t p = *((volatile unsigned long long*)&hash[slot].pos);
-          atomicOr(&run[p].mask, bit);
+          run_mask_or(v, p, bit);
         }
         run_len += chunk_new;
         __syncthreads();
@@ -162,13 +165,14 @@ __device__ __forceinline__ void miss_all(GroupHits& h, uint32_t lane, unsigned l
 // First-miss scan of blocks [start, n) of one chain for the `alive` decodes of a group.
 // Decodes found missing at position p get p; decodes never missing keep their value.
 // start_pos: the run position of block `start` when the caller has already looked it up.
-__device__ __forceinline__ void scan_chain(const IndexSlot* __restrict__ hash, uint32_t log2_cap,
+__device__ __forceinline__ void scan_chain(const IndexView& ix, uint32_t log2_cap,
                                            const uint64_t* __restrict__ chain, uint64_t start,
                                            uint64_t n, unsigned long long alive, GroupHits& h,
                                            uint32_t lane, int* status,
                                            unsigned long long start_pos = kNotFound) {
   const uint64_t cap = 1ull << log2_cap;
-  const RunEntry* __restrict__ run = reinterpret_cast<const RunEntry*>(hash + cap);
+  const IndexSlot* __restrict__ hash = ix.hash;
+  const unsigned long long* __restrict__ run_keys = ix.keys;
   uint64_t p = start;
   uint64_t seg_run = 0, seg_p = 0;  // run position matched with chain position seg_p
   bool in_run = false, fresh = false;
@@ -201,14 +205,17 @@ __device__ __forceinline__ void scan_chain(const IndexSlot* __restrict__ hash, u
     const uint64_t rp = seg_run + (i - seg_p);
     const bool in = i < n;
     const uint64_t ck = in ? __ldcs(chain + i) : 0ull;
-    ulonglong2 re = make_ulonglong2(0ull, 0ull);
-    if (in && rp < cap) re = __ldg(reinterpret_cast<const ulonglong2*>(run + rp));
-    const bool same = in && ck != 0ull && re.x == ck;
+    unsigned long long rkey = 0ull, rmask = 0ull;
+    if (in && rp < cap) {
+      rkey = __ldg(run_keys + rp);
+      rmask = run_mask(ix, rp);
+    }
+    const bool same = in && ck != 0ull && rkey == ck;
     const uint32_t run_ok = __ballot_sync(0xffffffffu, same);
     const uint32_t lead = (~run_ok) ? (uint32_t)(__ffs(~run_ok) - 1) : 32u;  // leading matches
     const bool counted = lane < lead;
     // decodes missing at some counted position of this step (usually none)
-    const unsigned long long nm = counted ? (alive & ~re.y) : 0ull;
+    const unsigned long long nm = counted ? (alive & ~rmask) : 0ull;
     unsigned long long a = ((unsigned long long)__reduce_or_sync(0xffffffffu, (uint32_t)(nm >> 32))
                             << 32) |
                            __reduce_or_sync(0xffffffffu, (uint32_t)nm);
@@ -231,7 +238,6 @@ __device__ __forceinline__ void scan_chain(const IndexSlot* __restrict__ hash, u
   }
 }
 
-enum MatchMode { kAll = 0, kMembers = 2 };
 
 // Group key of a request: its table set and first block hash, never zero.
 __device__ __forceinline__ uint64_t group_key(uint64_t h0, uint32_t set) {
@@ -278,12 +284,18 @@ __global__ void group_insert_kernel(GroupSlot* __restrict__ tab, uint32_t log2_s
   }
 }
 
+// A member's record: its chain offset and length (clamped to 65,535 blocks) and its
+// leader's, 48 + 16 bits each, so that the member pass fetches both chains' first blocks
+// and the leader's hits in its first round trip.
+constexpr uint64_t kOff48 = (1ull << 48) - 1;
+
 __global__ void group_resolve_kernel(const GroupSlot* __restrict__ tab, uint32_t log2_slots,
                                      const uint64_t* __restrict__ chains,
                                      const uint64_t* __restrict__ chain_off, uint32_t R,
                                      const uint32_t* __restrict__ set_off, uint32_t n_sets,
                                      uint32_t* __restrict__ leader_of, int32_t* __restrict__ set_of,
-                                     uint32_t* __restrict__ leaders, MatchCounters* counters) {
+                                     uint32_t* __restrict__ leaders, ulonglong2* __restrict__ rec,
+                                     MatchCounters* counters, int* status) {
   const uint64_t mask = (1ull << log2_slots) - 1;
   for (uint32_t r = blockIdx.x * blockDim.x + threadIdx.x; r < R; r += gridDim.x * blockDim.x) {
     const uint64_t c0 = __ldg(chain_off + r), c1 = __ldg(chain_off + r + 1);
@@ -302,6 +314,17 @@ __global__ void group_resolve_kernel(const GroupSlot* __restrict__ tab, uint32_t
         }
         if (k == 0ull) break;
         slot = (slot + 1) & mask;
+      }
+    }
+    if (lead != r) {
+      const uint64_t l0 = __ldg(chain_off + lead), l1 = __ldg(chain_off + lead + 1);
+      if (c1 <= kOff48 && l1 <= kOff48 && l1 > l0) {
+        const uint64_t n = c1 - c0, nl = l1 - l0;
+        if (n > 65535) flag_status(status, NETKV_DEV_EDOMAIN);  // counted up to 65,535 blocks
+        rec[r] = make_ulonglong2(c0 | (min(n, (uint64_t)65535) << 48),
+                                 l0 | (min(nl, (uint64_t)65535) << 48));
+      } else {
+        lead = r;  // offsets beyond 48 bits: matched in full by the leader pass
       }
     }
     leader_of[r] = lead;
@@ -364,19 +387,19 @@ __global__ void __launch_bounds__(kMatchBlock, 8) match_leaders_kernel(
     if (chain_extent(chain_off, set_off, n_sets, set_of, r, lane, status, set, c0, n)) {
       h.lo = h.hi = (uint32_t)n;
       const unsigned long long alive = ng >= 64 ? ~0ull : ((1ull << ng) - 1);
-      const IndexSlot* tab = index_hash(index, (uint64_t)set * n_dgroups + q, log2_cap);
-      scan_chain(tab, log2_cap, chains + c0, 0, n, alive, h, lane, status);
+      const IndexView ix = index_view(index, (uint64_t)set * n_dgroups + q, log2_cap,
+                                      mask_bytes_of(D));
+      scan_chain(ix, log2_cap, chains + c0, 0, n, alive, h, lane, status);
     }
     store_hits(M, (uint64_t)r * D, q0, ng, lane, h);
   }
 }
 
-template <int kMode>
+// Full match without a workspace: one warp per (request, decode group).
 __global__ void __launch_bounds__(kMatchBlock, 8) match_kernel(
     const void* __restrict__ index, uint32_t D, uint32_t log2_cap, uint32_t n_sets,
     const uint64_t* __restrict__ chains, const uint64_t* __restrict__ chain_off, uint32_t R,
-    const uint32_t* __restrict__ set_off, const uint32_t* __restrict__ leader_of,
-    const int32_t* __restrict__ set_of, uint16_t* __restrict__ M, int* status) {
+    const uint32_t* __restrict__ set_off, uint16_t* __restrict__ M, int* status) {
   const uint32_t lane = threadIdx.x & 31;
   const uint64_t warp = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const uint64_t n_warps = ((uint64_t)gridDim.x * blockDim.x) >> 5;
@@ -385,65 +408,94 @@ __global__ void __launch_bounds__(kMatchBlock, 8) match_kernel(
 
   for (uint64_t task = warp; task < total; task += n_warps) {
     const uint32_t r = (uint32_t)(n_dgroups == 1 ? task : task / n_dgroups);
-    uint32_t lead = r;
-    if (kMode == kMembers) {
-      lead = __ldg(leader_of + r);
-      if (lead == r) continue;  // leaders were matched by the leader pass
-    }
     const uint32_t q = (uint32_t)(task - (uint64_t)r * n_dgroups);
     const uint32_t q0 = q * kGroup, ng = min(kGroup, D - q0);
     GroupHits h = {0u, 0u};
     int32_t set;
     uint64_t c0, n;
-    if (!chain_extent(chain_off, set_off, n_sets, set_of, r, lane, status, set, c0, n)) {
-      store_hits(M, (uint64_t)r * D, q0, ng, lane, h);
-      continue;
+    if (chain_extent(chain_off, set_off, n_sets, nullptr, r, lane, status, set, c0, n)) {
+      h.lo = h.hi = (uint32_t)n;
+      const unsigned long long alive = ng >= 64 ? ~0ull : ((1ull << ng) - 1);
+      const IndexView ix = index_view(index, (uint64_t)set * n_dgroups + q, log2_cap,
+                                      mask_bytes_of(D));
+      scan_chain(ix, log2_cap, chains + c0, 0, n, alive, h, lane, status);
     }
-    h.lo = h.hi = (uint32_t)n;
-    unsigned long long alive = ng >= 64 ? ~0ull : ((1ull << ng) - 1);
-    uint64_t start = 0;
-    if (kMode == kMembers) {
-      // the leader's hits for this group and the common prefix of the two chains
-      const uint64_t lrow = (uint64_t)lead * D + q0;
-      const uint32_t mlo = lane < ng ? (uint32_t)__ldg(M + lrow + lane) : 0u;
-      const uint32_t mhi = lane + 32 < ng ? (uint32_t)__ldg(M + lrow + lane + 32) : 0u;
-      uint32_t mmax = max(mlo, mhi);
-#pragma unroll
-      for (int o = 16; o; o >>= 1) mmax = max(mmax, __shfl_xor_sync(0xffffffffu, mmax, o));
-      const uint64_t l0 = __ldg(chain_off + lead), l1 = __ldg(chain_off + lead + 1);
-      const uint64_t cap = min(n, min(l1 - l0, (uint64_t)mmax + 1));
-      uint64_t lcp = cap;  // common prefix, 128 blocks per step
-      for (uint64_t base = 0; base < cap; base += 128) {
-        uint64_t a[4], b[4];
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const uint64_t i = base + 32 * k + lane;
-          a[k] = i < cap ? __ldcs(chains + c0 + i) : 0ull;
-          b[k] = i < cap ? __ldg(chains + l0 + i) : 0ull;
-        }
-        uint64_t found = cap;
-#pragma unroll
-        for (int k = 3; k >= 0; --k) {
-          const uint32_t diff = __ballot_sync(0xffffffffu, a[k] != b[k]);
-          if (diff) found = base + 32 * k + (uint64_t)(__ffs(diff) - 1);
-        }
-        if (found < cap) {
-          lcp = found;
-          break;
-        }
-      }
-      // decodes whose leader missed inside the common prefix copy the leader's answer
-      const uint32_t clo = __ballot_sync(0xffffffffu, lane < ng && (uint64_t)mlo < lcp);
-      const uint32_t chi = __ballot_sync(0xffffffffu, lane + 32 < ng && (uint64_t)mhi < lcp);
-      const unsigned long long copy = (unsigned long long)clo | ((unsigned long long)chi << 32);
-      if ((clo >> lane) & 1u) h.lo = mlo;
-      if ((chi >> lane) & 1u) h.hi = mhi;
-      alive &= ~copy;
-      start = lcp;
-    }
-    const IndexSlot* tab = index_hash(index, (uint64_t)set * n_dgroups + q, log2_cap);
-    scan_chain(tab, log2_cap, chains + c0, start, n, alive, h, lane, status);
     store_hits(M, (uint64_t)r * D, q0, ng, lane, h);
+  }
+}
+
+// Member pass of pools of one decode group (D <= 64): one warp per request.  The record
+// written by the grouping gives both chains' offsets and lengths, so the leader's hits and
+// the first 128 blocks of both chains are fetched in one round trip (the cap on the common
+// prefix, min(n_r, n_L, max_d M_L[d] + 1), is known once the hits arrive).  Then as
+// the leader pass: decodes whose leader missed inside the common prefix take the leader's
+// answer, the rest walk on from the common prefix.
+__global__ void __launch_bounds__(kMatchBlock, 8) match_members_kernel(
+    const void* __restrict__ index, uint32_t D, uint32_t log2_cap,
+    const uint64_t* __restrict__ chains, uint32_t R, const uint32_t* __restrict__ leader_of,
+    const int32_t* __restrict__ set_of, const ulonglong2* __restrict__ rec,
+    uint16_t* __restrict__ M, int* status) {
+  const uint32_t lane = threadIdx.x & 31;
+  const uint64_t warp = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const uint64_t n_warps = ((uint64_t)gridDim.x * blockDim.x) >> 5;
+  const uint32_t ng = D;  // one group
+  for (uint64_t rr = warp; rr < R; rr += n_warps) {
+    const uint32_t r = (uint32_t)rr;
+    // the three loads go out together (a leader's record is not written and not used)
+    const uint32_t lead = __ldg(leader_of + r);
+    const ulonglong2 rc = __ldg(rec + r);
+    const int32_t set = __ldg(set_of + r);
+    if (lead == r) continue;  // leaders were matched by the leader pass
+    const uint64_t c0 = rc.x & kOff48, n = rc.x >> 48;
+    const uint64_t l0 = rc.y & kOff48, nl = rc.y >> 48;
+    const uint64_t capn = min(n, nl);
+    const uint64_t lrow = (uint64_t)lead * D;
+    const uint32_t mlo = lane < ng ? (uint32_t)__ldg(M + lrow + lane) : 0u;
+    const uint32_t mhi = lane + 32 < ng ? (uint32_t)__ldg(M + lrow + lane + 32) : 0u;
+    uint64_t a[4], b[4];
+    const uint64_t first = min(capn, (uint64_t)128);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const uint64_t i = 32 * k + lane;
+      a[k] = i < first ? __ldcs(chains + c0 + i) : 0ull;
+      b[k] = i < first ? __ldg(chains + l0 + i) : 0ull;
+    }
+    uint32_t mmax = max(mlo, mhi);
+#pragma unroll
+    for (int o = 16; o; o >>= 1) mmax = max(mmax, __shfl_xor_sync(0xffffffffu, mmax, o));
+    const uint64_t cap = min(capn, (uint64_t)mmax + 1);
+    uint64_t lcp = cap;  // common prefix, 128 blocks per step
+    for (uint64_t base = 0; base < cap;) {
+      uint64_t found = cap;
+#pragma unroll
+      for (int k = 3; k >= 0; --k) {
+        const uint64_t i = base + 32 * k + lane;
+        const uint32_t diff = __ballot_sync(0xffffffffu, i < cap && a[k] != b[k]);
+        if (diff) found = base + 32 * k + (uint64_t)(__ffs(diff) - 1);
+      }
+      if (found < cap) {
+        lcp = found;
+        break;
+      }
+      base += 128;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint64_t i = base + 32 * k + lane;
+        a[k] = i < cap ? __ldcs(chains + c0 + i) : 0ull;
+        b[k] = i < cap ? __ldg(chains + l0 + i) : 0ull;
+      }
+    }
+    GroupHits h = {(uint32_t)n, (uint32_t)n};
+    // decodes whose leader missed inside the common prefix copy the leader's answer
+    const uint32_t clo = __ballot_sync(0xffffffffu, lane < ng && (uint64_t)mlo < lcp);
+    const uint32_t chi = __ballot_sync(0xffffffffu, lane + 32 < ng && (uint64_t)mhi < lcp);
+    if ((clo >> lane) & 1u) h.lo = mlo;
+    if ((chi >> lane) & 1u) h.hi = mhi;
+    unsigned long long alive = ng >= 64 ? ~0ull : ((1ull << ng) - 1);
+    alive &= ~((unsigned long long)clo | ((unsigned long long)chi << 32));
+    scan_chain(index_view(index, (uint64_t)set, log2_cap, mask_bytes_of(D)), log2_cap,
+               chains + c0, lcp, n, alive, h, lane, status);
+    store_hits(M, (uint64_t)r * D, 0, ng, lane, h);
   }
 }
 
@@ -532,8 +584,9 @@ __global__ void __launch_bounds__(kMatchBlock, 6) match_members_wide_kernel(
       if (lane < n_pend) {
         const uint64_t key = __ldg(own + lcp);
         if (key == 0ull) flag_status(status, NETKV_DEV_EDOMAIN);
-        else pos = lookup(index_hash(index, (uint64_t)set * n_dgroups + pend_q, log2_cap), key,
-                          log2_cap, status);
+        else pos = lookup(index_view(index, (uint64_t)set * n_dgroups + pend_q, log2_cap,
+                                     mask_bytes_of(D)).hash,
+                          key, log2_cap, status);
       }
       uint32_t hit = __ballot_sync(0xffffffffu, lane < n_pend && pos != kNotFound);
       while (hit) {
@@ -550,8 +603,8 @@ __global__ void __launch_bounds__(kMatchBlock, 6) match_members_wide_kernel(
         const uint32_t alo = __ballot_sync(0xffffffffu, lane < ng && (uint64_t)mlo >= lcp);
         const uint32_t ahi = __ballot_sync(0xffffffffu, lane + 32 < ng && (uint64_t)mhi >= lcp);
         const unsigned long long alive = (unsigned long long)alo | ((unsigned long long)ahi << 32);
-        scan_chain(index_hash(index, (uint64_t)set * n_dgroups + q, log2_cap), log2_cap, own, lcp,
-                   n, alive, h, lane, status, pj);
+        scan_chain(index_view(index, (uint64_t)set * n_dgroups + q, log2_cap, mask_bytes_of(D)),
+                   log2_cap, own, lcp, n, alive, h, lane, status, pj);
         store_hits(M, row, q0, ng, lane, h);
       }
       n_pend = 0;
@@ -609,9 +662,10 @@ uint32_t group_log2_slots(uint32_t R) {
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-// Workspace: group table | leader_of [R] | set_of [R] | leader list [R] | counters.
+// Workspace: group table | leader_of [R] | set_of [R] | leader list [R] | member records [R]
+// | counters.
 struct WorkspaceLayout {
-  size_t table, leader_of, set_of, leaders, counters, total;
+  size_t table, leader_of, set_of, leaders, rec, counters, total;
 };
 
 WorkspaceLayout workspace_layout(uint32_t R) {
@@ -620,7 +674,8 @@ WorkspaceLayout workspace_layout(uint32_t R) {
   w.leader_of = align_up(sizeof(GroupSlot) << group_log2_slots(R), 256);
   w.set_of = w.leader_of + align_up(sizeof(uint32_t) * (size_t)R, 256);
   w.leaders = w.set_of + align_up(sizeof(int32_t) * (size_t)R, 256);
-  w.counters = w.leaders + align_up(sizeof(uint32_t) * (size_t)R, 256);
+  w.rec = w.leaders + align_up(sizeof(uint32_t) * (size_t)R, 256);
+  w.counters = w.rec + align_up(sizeof(ulonglong2) * (size_t)R, 256);
   w.total = w.counters + align_up(sizeof(MatchCounters), 256);
   return w;
 }
@@ -638,7 +693,7 @@ int leader_grid() {
 extern "C" size_t netkv_cache_index_bytes(uint32_t n_sets, uint32_t D, uint32_t log2_capacity) {
   if (log2_capacity < 1 || log2_capacity > 31) return 0;
   return (size_t)n_sets * ((D + kGroup - 1) / kGroup) *
-         ((sizeof(IndexSlot) + sizeof(RunEntry)) << log2_capacity);
+         index_stride(log2_capacity, mask_bytes_of(D));
 }
 
 extern "C" netkv_status netkv_cache_build(void* d_index, uint32_t n_sets, uint32_t D,
@@ -688,9 +743,8 @@ extern "C" netkv_status netkv_prefix_match(const void* d_index, uint32_t D,
   const uint64_t blocks = (tasks + warps_per_block - 1) / warps_per_block;
   const unsigned grid = (unsigned)(blocks < (1u << 24) ? blocks : (1u << 24));
   if (!d_workspace) {
-    match_kernel<kAll><<<grid, kMatchBlock, 0, s>>>(index, D, log2_capacity, n_sets, d_chains,
-                                                    d_chain_off, R, d_set_off, nullptr, nullptr,
-                                                    d_M, d_status);
+    match_kernel<<<grid, kMatchBlock, 0, s>>>(index, D, log2_capacity, n_sets, d_chains,
+                                              d_chain_off, R, d_set_off, d_M, d_status);
     return netkv_launch_status();
   }
   const uint32_t lg = group_log2_slots(R);
@@ -700,20 +754,20 @@ extern "C" netkv_status netkv_prefix_match(const void* d_index, uint32_t D,
   uint32_t* leader_of = reinterpret_cast<uint32_t*>(ws + L.leader_of);
   int32_t* set_of = reinterpret_cast<int32_t*>(ws + L.set_of);
   uint32_t* leaders = reinterpret_cast<uint32_t*>(ws + L.leaders);
+  ulonglong2* rec = reinterpret_cast<ulonglong2*>(ws + L.rec);
   MatchCounters* counters = reinterpret_cast<MatchCounters*>(ws + L.counters);
   NETKV_CUDA_TRY(cudaMemsetAsync(tab, 0, sizeof(GroupSlot) << lg, s));
   NETKV_CUDA_TRY(cudaMemsetAsync(counters, 0, sizeof(MatchCounters), s));
   const unsigned rgrid = (unsigned)((R + 255) / 256 < 65535u * 16 ? (R + 255) / 256 : 65535u * 16);
   group_insert_kernel<<<rgrid, 256, 0, s>>>(tab, lg, d_chains, d_chain_off, R, d_set_off, n_sets);
   group_resolve_kernel<<<rgrid, 256, 0, s>>>(tab, lg, d_chains, d_chain_off, R, d_set_off, n_sets,
-                                             leader_of, set_of, leaders, counters);
+                                             leader_of, set_of, leaders, rec, counters, d_status);
   match_leaders_kernel<<<leader_grid(), kMatchBlock, 0, s>>>(
       index, D, log2_capacity, n_sets, d_chains, d_chain_off, d_set_off, set_of, leaders, counters,
       d_M, d_status);
   if (D <= kGroup) {
-    match_kernel<kMembers><<<grid, kMatchBlock, 0, s>>>(index, D, log2_capacity, n_sets, d_chains,
-                                                        d_chain_off, R, d_set_off, leader_of,
-                                                        set_of, d_M, d_status);
+    match_members_kernel<<<grid, kMatchBlock, 0, s>>>(index, D, log2_capacity, d_chains, R,
+                                                      leader_of, set_of, rec, d_M, d_status);
   } else {
     const uint64_t mblocks = ((uint64_t)R + warps_per_block - 1) / warps_per_block;
     const unsigned mgrid = (unsigned)(mblocks < (1u << 24) ? mblocks : (1u << 24));
@@ -736,7 +790,7 @@ extern "C" netkv_status netkv_prefix_match(const void* d_index, uint32_t D,
 
 namespace {
 
-constexpr size_t kStaticScratchBytes = 24ull << 20;  // 24 MiB per device
+constexpr size_t kStaticScratchBytes = 32ull << 20;  // 32 MiB per device
 static __device__ __align__(256) unsigned char g_prefix_scratch[kStaticScratchBytes];
 
 constexpr int kMaxDevices = 64;

@@ -59,7 +59,13 @@ def test_version_and_host_validation(lib):
     so = lib._lib
     assert so.netkv_oracle_build(None, None, 1, 1.0, None, None, None, None) == lib.NETKV_EINVAL
     assert so.netkv_cache_build(None, 1, 1, 4, None, None, None, None) == lib.NETKV_EINVAL
-    assert so.netkv_cache_index_bytes(2, 65, 4) == 2 * 2 * (16 + 16) * 16
+    # per (set, group of 64 decodes): slots (16 B), run keys (8 B) and run masks (1, 2, 4 or
+    # 8 B by pool size) per position, padded to 256 bytes
+    assert so.netkv_cache_index_bytes(2, 65, 4) == 2 * 2 * (16 + 8 + 8) * 16
+    assert so.netkv_cache_index_bytes(3, 8, 10) == 3 * (16 + 8 + 1) * 1024
+    assert so.netkv_cache_index_bytes(1, 16, 10) == (16 + 8 + 2) * 1024
+    assert so.netkv_cache_index_bytes(1, 20, 10) == (16 + 8 + 4) * 1024
+    assert so.netkv_cache_index_bytes(1, 8, 1) == 256
     assert so.netkv_prefix_match(None, 1, 4, 1, None, None, 1, None, None, 0, None, None, None) == lib.NETKV_EINVAL
     assert so.netkv_prefix_match_workspace_size(0) == 0
     assert so.netkv_schedule_streams(None, 1, None, 0, None, None, None, None, None, 0, None, None,

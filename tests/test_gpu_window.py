@@ -43,7 +43,7 @@ SHAPES = [((1, 1, 2, 3), 3, 5),     # 8-lane segments, 5 of 8 lanes idle; 5 stre
 
 
 def _events(rng, r0, r1, gaps):
-    """Arrivals of requests r0..r1-1 in order; request i departs after gaps[i] more events
+    """Arrivals of requests r0..r1-1 in order; request i departs after gaps[i] more arrivals
     (a negative gap: it never departs)."""
     out, pending = [], []          # pending: [events left, r]
     for r in range(r0, r1):
@@ -98,8 +98,9 @@ def _case(fanout, n_streams, rps=300, seed=0, huge=False, bad=False):
     ev = np.array(ev, dtype=np.uint32)
     perm = rng.permutation(R).astype(np.int64)   # request r becomes perm[r]
     return dict(w=w, sc=sc, x=x, out=out, length=length, prefill=prefill, snap=snap,
-                events=ev, event_off=np.array(off, dtype=np.int64), perm=perm,
-                M=out.M, cap=(1 << 40) if huge else 60_000)
+                arrival_us=w.arrival_us.astype(np.int64), events=ev,
+                event_off=np.array(off, dtype=np.int64), perm=perm, M=out.M,
+                cap=(1 << 40) if huge else 60_000)
 
 
 def host32(t):
@@ -117,7 +118,7 @@ def _renumber(c):
     ev2 = ((ev & 0x80000000) | r2).astype(np.uint32)
     M2 = c["M"][torch.from_numpy(inv).to(c["M"].device)]
     return dict(length=c["length"][inv], prefill=c["prefill"][inv], snap=c["snap"][inv],
-                events=ev2, M=M2)
+                arrival_us=c["arrival_us"][inv], events=ev2, M=M2)
 
 
 def _run(c, arrays, walk, load_init=None):
@@ -146,7 +147,9 @@ def _run(c, arrays, walk, load_init=None):
         ws = torch.empty(netkv.netkv_schedule_inflight_workspace_size(R, D), dtype=torch.uint8,
                          device=dev)
         xfer = torch.empty(R, dtype=torch.int32, device=dev)
-        arrival = torch.zeros(R, dtype=torch.int64, device=dev)
+        # arrival times in event order, so that the completion heap drains (a transfer
+        # still pending past the heap's 256 entries would only set EFULL)
+        arrival = torch.from_numpy(arrays["arrival_us"]).to(dev)
         netkv.netkv_schedule_streams_inflight(sc.topo, S, wt, R, length, prefill, snap, arrival,
                                               arrays["M"], out.UB, x.n_snap, events, event_off,
                                               0, load_init, o["dec"], o["best"], o["second"],
@@ -170,8 +173,8 @@ def test_window_equals_packed_walk(fanout, D, n_streams, kind):
         rng = np.random.default_rng(3)
         li = rng.integers(-50, 30_000, (n_streams, D)).astype(np.int64)
         load_init = torch.from_numpy(li).cuda()
-    orig = dict(length=c["length"], prefill=c["prefill"], snap=c["snap"], events=c["events"],
-                M=c["M"])
+    orig = dict(length=c["length"], prefill=c["prefill"], snap=c["snap"],
+                arrival_us=c["arrival_us"], events=c["events"], M=c["M"])
     ren = _renumber(c)
     for arrays in (orig, ren):
         a = _run(c, arrays, "window", load_init)
