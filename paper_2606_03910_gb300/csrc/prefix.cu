@@ -255,8 +255,9 @@ struct GroupSlot {
 
 // Work counters at the end of the workspace.
 struct MatchCounters {
-  unsigned long long n_leaders;  // entries of the leader list
-  unsigned long long next_task;  // next (leader, decode group) task of the leader pass
+  unsigned long long n_leaders;    // entries of the leader list
+  unsigned long long next_task;    // next (leader, decode group) task of the leader pass
+  unsigned long long next_member;  // next chunk of requests of the member pass
 };
 
 __global__ void group_insert_kernel(GroupSlot* __restrict__ tab, uint32_t log2_slots,
@@ -424,78 +425,146 @@ __global__ void __launch_bounds__(kMatchBlock, 8) match_kernel(
   }
 }
 
-// Member pass of pools of one decode group (D <= 64): one warp per request.  The record
-// written by the grouping gives both chains' offsets and lengths, so the leader's hits and
-// the first 128 blocks of both chains are fetched in one round trip (the cap on the common
-// prefix, min(n_r, n_L, max_d M_L[d] + 1), is known once the hits arrive).  Then as
-// the leader pass: decodes whose leader missed inside the common prefix take the leader's
-// answer, the rest walk on from the common prefix.
+// Member pass of pools of one decode group (D <= 64), for member r with leader `lead`.
+// The record written by the grouping gives both chains' offsets and lengths, so the
+// leader's hits and the first 128 blocks of both chains are fetched in one round trip (the
+// cap on the common prefix, min(n_r, n_L, max_d M_L[d] + 1), is known once the hits
+// arrive).  Then as the leader pass: decodes whose leader missed inside the common prefix
+// take the leader's answer, the rest walk on from the common prefix.
+__device__ __forceinline__ void member_match(const void* __restrict__ index, uint32_t D,
+                                             uint32_t log2_cap,
+                                             const uint64_t* __restrict__ chains, uint32_t r,
+                                             uint32_t lead, int32_t set, ulonglong2 rc,
+                                             uint16_t* __restrict__ M, uint32_t lane,
+                                             int* status) {
+  const uint32_t ng = D;  // one group
+  const uint64_t c0 = rc.x & kOff48, n = rc.x >> 48;
+  const uint64_t l0 = rc.y & kOff48, nl = rc.y >> 48;
+  const uint64_t capn = min(n, nl);
+  const uint64_t lrow = (uint64_t)lead * D;
+  const uint32_t mlo = lane < ng ? (uint32_t)__ldg(M + lrow + lane) : 0u;
+  const uint32_t mhi = lane + 32 < ng ? (uint32_t)__ldg(M + lrow + lane + 32) : 0u;
+  uint64_t a[4], b[4];
+  const uint64_t first = min(capn, (uint64_t)128);
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const uint64_t i = 32 * k + lane;
+    a[k] = i < first ? __ldcs(chains + c0 + i) : 0ull;
+    b[k] = i < first ? __ldg(chains + l0 + i) : 0ull;
+  }
+  uint32_t mmax = max(mlo, mhi);
+#pragma unroll
+  for (int o = 16; o; o >>= 1) mmax = max(mmax, __shfl_xor_sync(0xffffffffu, mmax, o));
+  const uint64_t cap = min(capn, (uint64_t)mmax + 1);
+  uint64_t lcp = cap;  // common prefix, 128 blocks per step
+  for (uint64_t base = 0; base < cap;) {
+    uint64_t found = cap;
+#pragma unroll
+    for (int k = 3; k >= 0; --k) {
+      const uint64_t i = base + 32 * k + lane;
+      const uint32_t diff = __ballot_sync(0xffffffffu, i < cap && a[k] != b[k]);
+      if (diff) found = base + 32 * k + (uint64_t)(__ffs(diff) - 1);
+    }
+    if (found < cap) {
+      lcp = found;
+      break;
+    }
+    base += 128;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const uint64_t i = base + 32 * k + lane;
+      a[k] = i < cap ? __ldcs(chains + c0 + i) : 0ull;
+      b[k] = i < cap ? __ldg(chains + l0 + i) : 0ull;
+    }
+  }
+  GroupHits h = {(uint32_t)n, (uint32_t)n};
+  // decodes whose leader missed inside the common prefix copy the leader's answer
+  const uint32_t clo = __ballot_sync(0xffffffffu, lane < ng && (uint64_t)mlo < lcp);
+  const uint32_t chi = __ballot_sync(0xffffffffu, lane + 32 < ng && (uint64_t)mhi < lcp);
+  if ((clo >> lane) & 1u) h.lo = mlo;
+  if ((chi >> lane) & 1u) h.hi = mhi;
+  unsigned long long alive = ng >= 64 ? ~0ull : ((1ull << ng) - 1);
+  alive &= ~((unsigned long long)clo | ((unsigned long long)chi << 32));
+  scan_chain(index_view(index, (uint64_t)set, log2_cap, mask_bytes_of(D)), log2_cap,
+             chains + c0, lcp, n, alive, h, lane, status);
+  store_hits(M, (uint64_t)r * D, 0, ng, lane, h);
+}
+
+constexpr uint32_t kMemberChunk = 8;  // consecutive requests a warp takes at a time
+
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+  const unsigned sa = (unsigned)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(sa), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async4(void* smem, const void* gmem) {
+  const unsigned sa = (unsigned)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;\n" ::"r"(sa), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;\n" ::: "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.wait_group 0;\n" ::: "memory");
+}
+
+// A request's record, leader and table set, staged in shared memory per warp.
+struct __align__(16) MemberSlot {
+  ulonglong2 rc;
+  uint32_t lead;
+  int32_t set;
+  uint32_t pad[2];
+};
+
+// Persistent member pass of pools of one decode group: every warp takes chunks of 8
+// consecutive requests from a global counter (fetched one chunk ahead), so a warp that
+// finishes early takes more work instead of idling until its block ends.  The next
+// request's record, leader and table set are copied into the warp's shared-memory slot
+// with cp.async while the current one is matched, so they cost no round trip of their own.
 __global__ void __launch_bounds__(kMatchBlock, 8) match_members_kernel(
     const void* __restrict__ index, uint32_t D, uint32_t log2_cap,
     const uint64_t* __restrict__ chains, uint32_t R, const uint32_t* __restrict__ leader_of,
     const int32_t* __restrict__ set_of, const ulonglong2* __restrict__ rec,
-    uint16_t* __restrict__ M, int* status) {
+    MatchCounters* counters, uint16_t* __restrict__ M, int* status) {
+  __shared__ MemberSlot slots[kMatchBlock / 32];
+  MemberSlot& slot = slots[threadIdx.x >> 5];
   const uint32_t lane = threadIdx.x & 31;
-  const uint64_t warp = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const uint64_t n_warps = ((uint64_t)gridDim.x * blockDim.x) >> 5;
-  const uint32_t ng = D;  // one group
-  for (uint64_t rr = warp; rr < R; rr += n_warps) {
-    const uint32_t r = (uint32_t)rr;
-    // the three loads go out together (a leader's record is not written and not used)
-    const uint32_t lead = __ldg(leader_of + r);
-    const ulonglong2 rc = __ldg(rec + r);
-    const int32_t set = __ldg(set_of + r);
-    if (lead == r) continue;  // leaders were matched by the leader pass
-    const uint64_t c0 = rc.x & kOff48, n = rc.x >> 48;
-    const uint64_t l0 = rc.y & kOff48, nl = rc.y >> 48;
-    const uint64_t capn = min(n, nl);
-    const uint64_t lrow = (uint64_t)lead * D;
-    const uint32_t mlo = lane < ng ? (uint32_t)__ldg(M + lrow + lane) : 0u;
-    const uint32_t mhi = lane + 32 < ng ? (uint32_t)__ldg(M + lrow + lane + 32) : 0u;
-    uint64_t a[4], b[4];
-    const uint64_t first = min(capn, (uint64_t)128);
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const uint64_t i = 32 * k + lane;
-      a[k] = i < first ? __ldcs(chains + c0 + i) : 0ull;
-      b[k] = i < first ? __ldg(chains + l0 + i) : 0ull;
+  const unsigned long long n_chunks = ((unsigned long long)R + kMemberChunk - 1) / kMemberChunk;
+  // request rr's record into the slot (a leader's record is not written and not used)
+  auto fetch = [&](uint64_t rr) {
+    if (lane == 0) {
+      cp_async16(&slot.rc, rec + rr);
+      cp_async4(&slot.lead, leader_of + rr);
+      cp_async4(&slot.set, set_of + rr);
+      cp_async_commit();
     }
-    uint32_t mmax = max(mlo, mhi);
-#pragma unroll
-    for (int o = 16; o; o >>= 1) mmax = max(mmax, __shfl_xor_sync(0xffffffffu, mmax, o));
-    const uint64_t cap = min(capn, (uint64_t)mmax + 1);
-    uint64_t lcp = cap;  // common prefix, 128 blocks per step
-    for (uint64_t base = 0; base < cap;) {
-      uint64_t found = cap;
-#pragma unroll
-      for (int k = 3; k >= 0; --k) {
-        const uint64_t i = base + 32 * k + lane;
-        const uint32_t diff = __ballot_sync(0xffffffffu, i < cap && a[k] != b[k]);
-        if (diff) found = base + 32 * k + (uint64_t)(__ffs(diff) - 1);
-      }
-      if (found < cap) {
-        lcp = found;
-        break;
-      }
-      base += 128;
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const uint64_t i = base + 32 * k + lane;
-        a[k] = i < cap ? __ldcs(chains + c0 + i) : 0ull;
-        b[k] = i < cap ? __ldg(chains + l0 + i) : 0ull;
-      }
+  };
+  unsigned long long c = 0, c_next = 0;
+  if (lane == 0) c = atomicAdd(&counters->next_member, 1ull);
+  c = __shfl_sync(0xffffffffu, c, 0);
+  if (c >= n_chunks) return;
+  if (lane == 0) c_next = atomicAdd(&counters->next_member, 1ull);  // the chunk after
+  uint64_t r = c * kMemberChunk;
+  uint64_t end = min(r + kMemberChunk, (uint64_t)R);
+  fetch(r);
+  for (;;) {
+    if (lane == 0) cp_async_wait_all();  // request r's record has landed
+    __syncwarp();
+    const ulonglong2 rc = slot.rc;
+    const uint32_t lead = slot.lead;
+    const int32_t set = slot.set;
+    __syncwarp();  // every lane has read the slot before it is refilled
+    uint64_t rn = r + 1;
+    if (rn >= end) {  // this chunk is done: take the one fetched ahead, and fetch the next
+      const unsigned long long cn = __shfl_sync(0xffffffffu, c_next, 0);
+      rn = cn < n_chunks ? cn * kMemberChunk : (uint64_t)R;
+      end = min(rn + kMemberChunk, (uint64_t)R);
+      if (lane == 0 && cn < n_chunks) c_next = atomicAdd(&counters->next_member, 1ull);
     }
-    GroupHits h = {(uint32_t)n, (uint32_t)n};
-    // decodes whose leader missed inside the common prefix copy the leader's answer
-    const uint32_t clo = __ballot_sync(0xffffffffu, lane < ng && (uint64_t)mlo < lcp);
-    const uint32_t chi = __ballot_sync(0xffffffffu, lane + 32 < ng && (uint64_t)mhi < lcp);
-    if ((clo >> lane) & 1u) h.lo = mlo;
-    if ((chi >> lane) & 1u) h.hi = mhi;
-    unsigned long long alive = ng >= 64 ? ~0ull : ((1ull << ng) - 1);
-    alive &= ~((unsigned long long)clo | ((unsigned long long)chi << 32));
-    scan_chain(index_view(index, (uint64_t)set, log2_cap, mask_bytes_of(D)), log2_cap,
-               chains + c0, lcp, n, alive, h, lane, status);
-    store_hits(M, (uint64_t)r * D, 0, ng, lane, h);
+    if (rn < R) fetch(rn);
+    if (lead != (uint32_t)r)  // leaders were matched by the leader pass
+      member_match(index, D, log2_cap, chains, (uint32_t)r, lead, set, rc, M, lane, status);
+    if (rn >= R) break;
+    r = rn;
   }
 }
 
@@ -680,13 +749,17 @@ WorkspaceLayout workspace_layout(uint32_t R) {
   return w;
 }
 
-int leader_grid() {
+// Blocks of a persistent grid: every SM filled to the kernel's occupancy.
+template <typename Kernel>
+int persistent_grid(Kernel kernel) {
   int dev = 0, sms = 0, per_sm = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, match_leaders_kernel, kMatchBlock, 0);
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kMatchBlock, 0);
   return (sms > 0 ? sms : 1) * (per_sm > 0 ? per_sm : 1);
 }
+int leader_grid() { return persistent_grid(match_leaders_kernel); }
+int member_grid() { return persistent_grid(match_members_kernel); }
 
 }  // namespace
 
@@ -766,8 +839,8 @@ extern "C" netkv_status netkv_prefix_match(const void* d_index, uint32_t D,
       index, D, log2_capacity, n_sets, d_chains, d_chain_off, d_set_off, set_of, leaders, counters,
       d_M, d_status);
   if (D <= kGroup) {
-    match_members_kernel<<<grid, kMatchBlock, 0, s>>>(index, D, log2_capacity, d_chains, R,
-                                                      leader_of, set_of, rec, d_M, d_status);
+    match_members_kernel<<<member_grid(), kMatchBlock, 0, s>>>(
+        index, D, log2_capacity, d_chains, R, leader_of, set_of, rec, counters, d_M, d_status);
   } else {
     const uint64_t mblocks = ((uint64_t)R + warps_per_block - 1) / warps_per_block;
     const unsigned mgrid = (unsigned)(mblocks < (1u << 24) ? mblocks : (1u << 24));
