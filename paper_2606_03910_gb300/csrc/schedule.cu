@@ -178,7 +178,7 @@ __device__ __forceinline__ float xfer_factor(const netkv_weights& w, uint32_t l,
 // the utilisation rows [n_snap][n_links] instead of the level bottlenecks, and the
 // bottlenecks are taken from the links' entries.  X (self-contention) gets s_eff / Bbot.
 template <int LPS, bool kUtil = false>
-__global__ void __launch_bounds__(256, 8) base_kernel(
+__global__ void __launch_bounds__(256, 6) base_kernel(
     TopoArgs t, uint32_t n_streams, const netkv_weights* __restrict__ W, uint32_t R,
     const uint32_t* __restrict__ len, const uint32_t* __restrict__ prefill,
     const uint32_t* __restrict__ snap, const uint16_t* __restrict__ M,
@@ -186,12 +186,24 @@ __global__ void __launch_bounds__(256, 8) base_kernel(
     const uint64_t* __restrict__ event_off, float* __restrict__ base, int* status,
     float* __restrict__ X = nullptr) {
   constexpr uint32_t kSegs = 256 / LPS;
+  constexpr uint32_t kNone = 0xffffffffu;  // no event (a departure code: skipped)
   const uint32_t seg = threadIdx.x / LPS, sl = threadIdx.x % LPS;
   const uint32_t D = t.D, N = t.N;
   const bool mine = sl < D;  // D <= LPS: lane sl owns decode sl
   const float4 lat = make_float4(t.lat[0], t.lat[1], t.lat[2], t.lat[3]);
   const uint32_t inst = mine ? __ldg(t.dec + sl) : 0u;
   const uint4 ld = __ldg(t.links + inst);
+  // an arrival's length, prefill rank, snapshot and this lane's prefix hit
+  auto fields = [&](uint32_t code, uint32_t& l, uint32_t& pr, uint32_t& k, uint32_t& m) {
+    const uint32_t r = code & 0x7fffffffu;
+    l = pr = k = m = 0u;
+    if (!(code >> 31) && r < R) {
+      l = __ldg(len + r);
+      pr = __ldg(prefill + r);
+      k = __ldg(snap + r);
+      if (mine) m = __ldg(M + (uint64_t)r * D + sl);
+    }
+  };
   for (uint32_t stream = blockIdx.x; stream < n_streams; stream += gridDim.x) {
     const float w_net = W[stream].w_net, w_prefix = W[stream].w_prefix;
     const float bpt = (float)W[stream].bytes_per_token;
@@ -204,15 +216,21 @@ __global__ void __launch_bounds__(256, 8) base_kernel(
     const uint64_t ee = min(e1, eb + span);
     uint32_t cur_k = 0xffffffffu;
     float4 qd = make_float4(0.f, 0.f, 0.f, 0.f);
-    uint32_t next = eb < ee ? __ldg(events + eb) : 0u;
+    // software pipeline: the next event's fields and the code after it are loaded while
+    // the current arrival is scored, so an arrival waits for one round trip (its
+    // utilisation entries) instead of three
+    uint32_t c_next = eb + 1 < ee ? __ldg(events + eb + 1) : kNone;
+    uint32_t code_n = eb < ee ? __ldg(events + eb) : kNone;
+    uint32_t l_n, pr_n, k_n, m_n;
+    fields(code_n, l_n, pr_n, k_n, m_n);
     for (uint64_t e = eb; e < ee; ++e) {
-      const uint32_t code = next;
-      if (e + 1 < ee) next = __ldg(events + e + 1);
+      const uint32_t code = code_n, l = l_n, pr = pr_n, k = k_n, m = m_n;
+      code_n = c_next;
+      c_next = e + 2 < ee ? __ldg(events + e + 2) : kNone;
+      fields(code_n, l_n, pr_n, k_n, m_n);
       const uint32_t r = code & 0x7fffffffu;
       if ((code >> 31) || r >= R) continue;
-      const uint32_t l = __ldg(len + r), pr = __ldg(prefill + r), k = __ldg(snap + r);
       if (pr >= t.P || k >= n_snap || l == 0 || !mine) continue;
-      const uint32_t m = __ldg(M + (uint64_t)r * D + sl);
       if (k != cur_k) {  // the decode's level bottlenecks of a new snapshot
         cur_k = k;
         const float4 ub = kUtil ? level_bottlenecks_of(t, UB + (uint64_t)k * t.n_links, ld, status)
