@@ -29,8 +29,9 @@
 // on those blocks, so with a workspace the match runs in three steps:
 //   group_insert_kernel / group_resolve_kernel: requests are grouped by (table set,
 //     first block hash) in an open-addressing table; each group's leader is its
-//     longest chain (lowest index among equals); leaders go to a compact list, and each
-//     member gets a record of its own and its leader's chain offsets and lengths.
+//     longest chain (lowest index among equals); leaders go to a compact list (chains of
+//     2,048 blocks or more first), and each member gets a record of its own and its
+//     leader's chain offsets and lengths.
 //   match_leaders_kernel: leaders (and ungrouped requests) run the full match, one task
 //     per (leader, decode group) taken in order from a counter.
 //   match_members_kernel: a member r with leader L compares chains to get
@@ -255,22 +256,33 @@ struct GroupSlot {
 
 // Work counters at the end of the workspace.
 struct MatchCounters {
-  unsigned long long n_leaders;    // entries of the leader list
+  unsigned long long n_long;       // leaders listed from the front of the leader list
+  unsigned long long n_short;      // leaders listed from its back
   unsigned long long next_task;    // next (leader, decode group) task of the leader pass
   unsigned long long next_member;  // next chunk of requests of the member pass
 };
 
+// Leaders with chains of at least this many blocks are listed first, so that the leader
+// pass, which takes its tasks in list order, ends on short chains instead of waiting for
+// a long one started last.
+constexpr uint64_t kLongLeader = 2048;
+
+// One thread per request: its table set (set_of) and group key (in rec[r].x, for the
+// resolve pass) are recorded, and the group's slot keeps the longest chain.
 __global__ void group_insert_kernel(GroupSlot* __restrict__ tab, uint32_t log2_slots,
                                     const uint64_t* __restrict__ chains,
                                     const uint64_t* __restrict__ chain_off, uint32_t R,
-                                    const uint32_t* __restrict__ set_off, uint32_t n_sets) {
+                                    const uint32_t* __restrict__ set_off, uint32_t n_sets,
+                                    int32_t* __restrict__ set_of, ulonglong2* __restrict__ rec) {
   const uint64_t mask = (1ull << log2_slots) - 1;
   for (uint32_t r = blockIdx.x * blockDim.x + threadIdx.x; r < R; r += gridDim.x * blockDim.x) {
     const uint64_t c0 = __ldg(chain_off + r), c1 = __ldg(chain_off + r + 1);
     const int32_t set = find_set(set_off, n_sets, r);
+    set_of[r] = set;
     if (c1 <= c0 || set < 0) continue;
     const uint64_t n = c1 - c0;
     const uint64_t key = group_key(__ldg(chains + c0), (uint32_t)set);
+    rec[r].x = key;
     const unsigned long long code =
         ((unsigned long long)(n < 0xffffffffull ? n : 0xffffffffull) << 32) | (0xffffffffu - r);
     uint64_t slot = home_slot(key, log2_slots);
@@ -291,26 +303,25 @@ __global__ void group_insert_kernel(GroupSlot* __restrict__ tab, uint32_t log2_s
 constexpr uint64_t kOff48 = (1ull << 48) - 1;
 
 __global__ void group_resolve_kernel(const GroupSlot* __restrict__ tab, uint32_t log2_slots,
-                                     const uint64_t* __restrict__ chains,
                                      const uint64_t* __restrict__ chain_off, uint32_t R,
-                                     const uint32_t* __restrict__ set_off, uint32_t n_sets,
-                                     uint32_t* __restrict__ leader_of, int32_t* __restrict__ set_of,
+                                     uint32_t* __restrict__ leader_of,
+                                     const int32_t* __restrict__ set_of,
                                      uint32_t* __restrict__ leaders, ulonglong2* __restrict__ rec,
                                      MatchCounters* counters, int* status) {
   const uint64_t mask = (1ull << log2_slots) - 1;
   for (uint32_t r = blockIdx.x * blockDim.x + threadIdx.x; r < R; r += gridDim.x * blockDim.x) {
     const uint64_t c0 = __ldg(chain_off + r), c1 = __ldg(chain_off + r + 1);
-    const int32_t set = find_set(set_off, n_sets, r);
+    const int32_t set = __ldg(set_of + r);
     uint32_t lead = r;
     if (c1 > c0 && set >= 0) {
-      const uint64_t key = group_key(__ldg(chains + c0), (uint32_t)set);
+      const uint64_t key = rec[r].x;  // written by the insert pass
       uint64_t slot = home_slot(key, log2_slots);
       for (uint64_t step = 0; step <= mask; ++step) {
         const unsigned long long k = tab[slot].key;
         if (k == key) {
           const uint32_t L = 0xffffffffu - (uint32_t)(tab[slot].code & 0xffffffffull);
           // a leader from another table set (64-bit key collision) is never used
-          if (L < R && find_set(set_off, n_sets, L) == set) lead = L;
+          if (L < R && __ldg(set_of + L) == set) lead = L;
           break;
         }
         if (k == 0ull) break;
@@ -329,8 +340,12 @@ __global__ void group_resolve_kernel(const GroupSlot* __restrict__ tab, uint32_t
       }
     }
     leader_of[r] = lead;
-    set_of[r] = set;
-    if (lead == r) leaders[atomicAdd(&counters->n_leaders, 1ull)] = r;
+    if (lead == r) {  // long chains from the front of the list, the rest from its back
+      if (c1 > c0 && c1 - c0 >= kLongLeader)
+        leaders[atomicAdd(&counters->n_long, 1ull)] = r;
+      else
+        leaders[R - 1 - atomicAdd(&counters->n_short, 1ull)] = r;
+    }
   }
 }
 
@@ -365,21 +380,22 @@ __device__ __forceinline__ void store_hits(uint16_t* __restrict__ M, uint64_t ro
 // by whole warps, so long and short chains balance across the GPU.
 __global__ void __launch_bounds__(kMatchBlock, 8) match_leaders_kernel(
     const void* __restrict__ index, uint32_t D, uint32_t log2_cap, uint32_t n_sets,
-    const uint64_t* __restrict__ chains, const uint64_t* __restrict__ chain_off,
+    const uint64_t* __restrict__ chains, const uint64_t* __restrict__ chain_off, uint32_t R,
     const uint32_t* __restrict__ set_off, const int32_t* __restrict__ set_of,
     const uint32_t* __restrict__ leaders, MatchCounters* counters, uint16_t* __restrict__ M,
     int* status) {
   const uint32_t lane = threadIdx.x & 31;
   const uint32_t n_dgroups = (D + kGroup - 1) / kGroup;
+  const unsigned long long n_long = *((volatile unsigned long long*)&counters->n_long);
   const unsigned long long total =
-      *((volatile unsigned long long*)&counters->n_leaders) * n_dgroups;
+      (n_long + *((volatile unsigned long long*)&counters->n_short)) * n_dgroups;
   for (;;) {
     unsigned long long t = 0;
     if (lane == 0) t = atomicAdd(&counters->next_task, 1ull);
     t = __shfl_sync(0xffffffffu, t, 0);
     if (t >= total) break;
     const uint64_t li = n_dgroups == 1 ? t : t / n_dgroups;
-    const uint32_t r = __ldg(leaders + li);
+    const uint32_t r = __ldg(leaders + (li < n_long ? li : (uint64_t)R - 1 - (li - n_long)));
     const uint32_t q = (uint32_t)(t - li * n_dgroups);
     const uint32_t q0 = q * kGroup, ng = min(kGroup, D - q0);
     GroupHits h = {0u, 0u};
@@ -832,12 +848,13 @@ extern "C" netkv_status netkv_prefix_match(const void* d_index, uint32_t D,
   NETKV_CUDA_TRY(cudaMemsetAsync(tab, 0, sizeof(GroupSlot) << lg, s));
   NETKV_CUDA_TRY(cudaMemsetAsync(counters, 0, sizeof(MatchCounters), s));
   const unsigned rgrid = (unsigned)((R + 255) / 256 < 65535u * 16 ? (R + 255) / 256 : 65535u * 16);
-  group_insert_kernel<<<rgrid, 256, 0, s>>>(tab, lg, d_chains, d_chain_off, R, d_set_off, n_sets);
-  group_resolve_kernel<<<rgrid, 256, 0, s>>>(tab, lg, d_chains, d_chain_off, R, d_set_off, n_sets,
-                                             leader_of, set_of, leaders, rec, counters, d_status);
+  group_insert_kernel<<<rgrid, 256, 0, s>>>(tab, lg, d_chains, d_chain_off, R, d_set_off, n_sets,
+                                            set_of, rec);
+  group_resolve_kernel<<<rgrid, 256, 0, s>>>(tab, lg, d_chain_off, R, leader_of, set_of, leaders,
+                                             rec, counters, d_status);
   match_leaders_kernel<<<leader_grid(), kMatchBlock, 0, s>>>(
-      index, D, log2_capacity, n_sets, d_chains, d_chain_off, d_set_off, set_of, leaders, counters,
-      d_M, d_status);
+      index, D, log2_capacity, n_sets, d_chains, d_chain_off, R, d_set_off, set_of, leaders,
+      counters, d_M, d_status);
   if (D <= kGroup) {
     match_members_kernel<<<member_grid(), kMatchBlock, 0, s>>>(
         index, D, log2_capacity, d_chains, R, leader_of, set_of, rec, counters, d_M, d_status);
