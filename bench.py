@@ -229,8 +229,8 @@ KERNEL_CODE = {
 #   oracle_build: bytes per snapshot of the oracle-build sweep
 MEASURED_TRAFFIC = {
     # 64 replicas (64,000 requests): group_insert 8.96 MB, group_resolve 2.20 MB,
-    # match_leaders 92.82 MB, match_members_kernel 240.09 MB (read + write)
-    "prefix_match": {"code_sha256_16": "9d009b971c354783", "bytes_per_unit": 344_069_888 / 64_000,
+    # match_leaders 92.51 MB, match_members_kernel 239.84 MB (read + write)
+    "prefix_match": {"code_sha256_16": "770ae3653abd8151", "bytes_per_unit": 343_515_136 / 64_000,
                      "unit": "request", "captured": "64-replica case, one launch per kernel"},
     "oracle_build": {"code_sha256_16": "ed437e71560780e2", "bytes_per_unit": 67_155_930,
                      "unit": "snapshot", "captured": "1,000-snapshot sweep, one launch"},

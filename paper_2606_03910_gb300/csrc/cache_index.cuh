@@ -56,8 +56,11 @@ __device__ __forceinline__ IndexView index_view(const void* index, uint64_t idx,
   return v;
 }
 
-// Mask of run position p (read-only path).
+// Mask of run position p (read-only path).  kMB: the mask width when the caller knows it
+// at compile time (pools of more than 32 decodes: 8), 0 to read it from the view.
+template <int kMB = 0>
 __device__ __forceinline__ unsigned long long run_mask(const IndexView& v, uint64_t p) {
+  if (kMB == 8) return __ldg(reinterpret_cast<const unsigned long long*>(v.masks) + p);
   switch (v.mask_bytes) {
     case 1: return __ldg(v.masks + p);
     case 2: return __ldg(reinterpret_cast<const unsigned short*>(v.masks) + p);

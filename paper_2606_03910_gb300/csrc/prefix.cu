@@ -166,6 +166,8 @@ __device__ __forceinline__ void miss_all(GroupHits& h, uint32_t lane, unsigned l
 // First-miss scan of blocks [start, n) of one chain for the `alive` decodes of a group.
 // Decodes found missing at position p get p; decodes never missing keep their value.
 // start_pos: the run position of block `start` when the caller has already looked it up.
+// kMB: the run masks' width when known at compile time (see run_mask), else 0.
+template <int kMB = 0>
 __device__ __forceinline__ void scan_chain(const IndexView& ix, uint32_t log2_cap,
                                            const uint64_t* __restrict__ chain, uint64_t start,
                                            uint64_t n, unsigned long long alive, GroupHits& h,
@@ -209,7 +211,7 @@ __device__ __forceinline__ void scan_chain(const IndexView& ix, uint32_t log2_ca
     unsigned long long rkey = 0ull, rmask = 0ull;
     if (in && rp < cap) {
       rkey = __ldg(run_keys + rp);
-      rmask = run_mask(ix, rp);
+      rmask = run_mask<kMB>(ix, rp);
     }
     const bool same = in && ck != 0ull && rkey == ck;
     const uint32_t run_ok = __ballot_sync(0xffffffffu, same);
@@ -669,8 +671,7 @@ __global__ void __launch_bounds__(kMatchBlock, 6) match_members_wide_kernel(
       if (lane < n_pend) {
         const uint64_t key = __ldg(own + lcp);
         if (key == 0ull) flag_status(status, NETKV_DEV_EDOMAIN);
-        else pos = lookup(index_view(index, (uint64_t)set * n_dgroups + pend_q, log2_cap,
-                                     mask_bytes_of(D)).hash,
+        else pos = lookup(index_view(index, (uint64_t)set * n_dgroups + pend_q, log2_cap, 8u).hash,
                           key, log2_cap, status);
       }
       uint32_t hit = __ballot_sync(0xffffffffu, lane < n_pend && pos != kNotFound);
@@ -688,7 +689,7 @@ __global__ void __launch_bounds__(kMatchBlock, 6) match_members_wide_kernel(
         const uint32_t alo = __ballot_sync(0xffffffffu, lane < ng && (uint64_t)mlo >= lcp);
         const uint32_t ahi = __ballot_sync(0xffffffffu, lane + 32 < ng && (uint64_t)mhi >= lcp);
         const unsigned long long alive = (unsigned long long)alo | ((unsigned long long)ahi << 32);
-        scan_chain(index_view(index, (uint64_t)set * n_dgroups + q, log2_cap, mask_bytes_of(D)),
+        scan_chain<8>(index_view(index, (uint64_t)set * n_dgroups + q, log2_cap, 8u),
                    log2_cap, own, lcp, n, alive, h, lane, status, pj);
         store_hits(M, row, q0, ng, lane, h);
       }
